@@ -1,0 +1,411 @@
+"""SelKV oracle: a plain, slow, fp64 CPU statement of what SelKV computes.
+
+TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline
+leg may import or call this module.  The CUDA library never calls it and shares no code with
+it; the two meet only at the seeded inputs of the `synth` module.
+
+What it follows (arxiv 2607.16213, "SelKV: Selective KV Cache Merging with Per-Token
+Merge-or-Drop and Attention Compensation"):
+
+  observation re-pass (Sec. 3.1) -> contribution score (Eq. 1) -> average pooling (Sec. 3.2)
+  -> budget m = floor(rho n), recent window m_r (Sec. 3.1) -> per-KV-head top-m_s, union over
+  KV heads, trim by mean score (Eq. 2, Sec. 3.3 "Union selection") -> bucket-attention routing
+  (Eq. 3) -> soft cosine gate (Eq. 4) -> gated attention-weighted merge (Eq. 5) -> attention
+  ratio (Eq. 6) -> GQA bias alpha*log(mean_kv R) (Sec. 3.5) -> decode with the bias (Alg. 1,
+  last step).  RoPE repositioning (Eq. 7) is off, as in the paper's configuration (Sec. 4.1).
+
+Readings where the paper is silent or garbled (each is a named choice, mirrored by the CUDA
+path):
+  R1  the re-pass is causal: window row i sits at position p_i = n - W + i and sees j <= p_i.
+  R2  softmax scale 1/sqrt(d).
+  R3  query head h uses KV head h // G.
+  R4  per-KV-head scores and cumulative attention are the mean over the G query heads;
+      then c_kv = a_kv * ||v_kv|| (Eq. 1 averaged over the group).
+  R5  pooling: stride 1, zero padding, divide by the kernel size, over the candidate range
+      [0, n - m_r) only (recent-window scores are not pooled in).
+  R6  m = floor(rho * n) in double; m_s = m - m_r must be >= 0.
+  R7  every top-k, trim and argmax orders by value descending, then index ascending.
+  R8  trim key = mean over KV heads of the pooled per-KV-head score, restricted to the union.
+  R9  Eq. 3's argmax uses a_{kv,i}, the cumulative observation-window attention paid to the
+      candidate i (the paper says the lookup uses the window queries' attention); so every
+      evicted token of a bucket shares one target per KV head.
+  R10 bucket(j) = floor(j / B) from position 0; the last bucket may be partial.
+  R11 empty bucket: "expand" looks at the kept tokens of buckets b-r and b+r for r = 1, 2, ...
+      and takes the first non-empty ring; "drop" gives those tokens g = 0 and no target.
+  R12 only values are merged; kept keys are unchanged.
+  R13 the gate uses the original (pre-merge) target value; a zero norm gives sim = 0; g is
+      clamped to [0, 1].
+  R14 decision MERGE iff g > 0, else DROP.
+  R15 a_i = 0 guard: R = 1, and v~ = v_i when the denominator is 0.
+  R16 GQA bias = alpha * ln(mean over KV heads of R) (natural log), per layer.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+from typing import Optional
+
+import numpy as np
+
+GATE_COSINE, GATE_OPEN, GATE_CLOSED = 0, 1, 2
+EMPTY_EXPAND, EMPTY_DROP = 0, 1
+DECISION_DROP, DECISION_MERGE = 0, 1
+
+
+@dataclass
+class Params:
+    """Method hyperparameters (Sec. 4.1 / App. F defaults)."""
+    alpha: float = 0.5
+    pool_kernel: int = 5
+    bucket: int = 32
+    recent: int = 16
+    gate_mode: int = GATE_COSINE
+    empty_bucket: int = EMPTY_EXPAND
+
+
+# ----------------------------------------------------------------------------------------
+# Sec. 3.1: budget
+# ----------------------------------------------------------------------------------------
+def budget(n: int, rho: float, recent: int):
+    """m = floor(rho * n) kept entries; the last m_r = recent are always kept; m_s = m - m_r
+    are chosen by score (Sec. 3.1, reading R6)."""
+    m = int(math.floor(float(rho) * float(n)))
+    return m, m - recent
+
+
+# ----------------------------------------------------------------------------------------
+# Sec. 3.1 two-pass re-pass + Eq. 1: observation-window attention
+# ----------------------------------------------------------------------------------------
+def observation_attention(Q: np.ndarray, K: np.ndarray, n: int) -> np.ndarray:
+    """A[h, i, j]: softmax over keys j <= p_i of q_{h,i} . k_{kv(h),j} / sqrt(d), for the W
+    window rows i at positions p_i = n - W + i (Sec. 3.1; readings R1-R3).
+
+    Q: [Hq][W][d], K: [Hkv][>=n][d] (float64).  Returns [Hq][W][n]."""
+    Hq, W, d = Q.shape
+    Hkv = K.shape[0]
+    G = Hq // Hkv
+    A = np.zeros((Hq, W, n))
+    pos = n - W + np.arange(W)
+    visible = np.arange(n)[None, :] <= pos[:, None]
+    for h in range(Hq):
+        s = (Q[h] @ K[h // G, :n].T) / math.sqrt(d)
+        s = np.where(visible, s, -np.inf)
+        s = s - s.max(axis=1, keepdims=True)
+        e = np.exp(s)
+        A[h] = e / e.sum(axis=1, keepdims=True)
+    return A
+
+
+def cumulative_attention(Q: np.ndarray, K: np.ndarray, n: int) -> np.ndarray:
+    """a[kv, j] = (1/G) sum_{h in group(kv)} sum_i A[h, i, j] (Eq. 5's a, averaged over the
+    query group, reading R4).  Computed one query head at a time.  Returns [Hkv][n]."""
+    Hq, W, d = Q.shape
+    Hkv = K.shape[0]
+    G = Hq // Hkv
+    a = np.zeros((Hkv, n))
+    for h in range(Hq):
+        A_h = observation_attention(Q[h:h + 1], K[h // G:h // G + 1], n)[0]
+        a[h // G] += A_h.sum(axis=0)
+    return a / G
+
+
+def value_norms(V: np.ndarray, n: int) -> np.ndarray:
+    """||v_{kv,j}||_2 for j < n.  V: [Hkv][>=n][d]."""
+    return np.sqrt((V[:, :n] ** 2).sum(axis=2))
+
+
+def contribution_scores(a: np.ndarray, V: np.ndarray, n: int) -> np.ndarray:
+    """Eq. 1 per KV head: c[kv, j] = a[kv, j] * ||v_{kv,j}|| (reading R4)."""
+    return a * value_norms(V, n)
+
+
+def pool_scores(c: np.ndarray, n_cand: int, kernel: int) -> np.ndarray:
+    """Average pooling of the scores over the candidate range [0, n_cand) (Sec. 3.2,
+    reading R5): out[j] = (1/kernel) * sum_{|t| <= kernel//2} c[j + t], with terms outside
+    [0, n_cand) taken as zero.  c: [Hkv][>=n_cand].  Returns [Hkv][n_cand]."""
+    half = kernel // 2
+    out = np.zeros((c.shape[0], n_cand))
+    idx = np.arange(n_cand)
+    for t in range(-half, half + 1):
+        src = idx + t
+        ok = (src >= 0) & (src < n_cand)
+        out[:, ok] += c[:, src[ok]]
+    return out / kernel
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 2 + Sec. 3.3: selection
+# ----------------------------------------------------------------------------------------
+def top_k_mask(values: np.ndarray, k: int) -> np.ndarray:
+    """Boolean mask of the k best entries: larger value first, then lower index (R7)."""
+    order = np.lexsort((np.arange(values.shape[0]), -values))
+    mask = np.zeros(values.shape[0], dtype=bool)
+    mask[order[:k]] = True
+    return mask
+
+
+def kth_gap(values: np.ndarray, k: int) -> float:
+    """Relative gap between the k-th and (k+1)-th best values (0 if either is missing):
+    how far the top-k boundary is from a tie."""
+    if k <= 0 or k >= values.shape[0]:
+        return math.inf
+    s = np.sort(values)[::-1]
+    hi, lo = s[k - 1], s[k]
+    return float((hi - lo) / max(abs(hi), 1e-300))
+
+
+@dataclass
+class Selection:
+    per_kv: np.ndarray        # [Hkv][n_cand] bool: each KV head's top-m_s (Eq. 2)
+    union: np.ndarray         # [n_cand] bool
+    kept_cand: np.ndarray     # [n_cand] bool: union, trimmed to m_s by mean score (Sec. 3.3)
+    kept: np.ndarray          # [n] bool: kept_cand plus the recent window
+    trimmed: bool
+
+
+def select_shared(c_pooled: np.ndarray, n: int, m_s: int, recent: int,
+                  follow_per_kv: Optional[np.ndarray] = None,
+                  follow_kept: Optional[np.ndarray] = None) -> Selection:
+    """GQA union selection (Eq. 2 per KV head, then Sec. 3.3 union and trim; R7, R8).
+
+    follow_per_kv / follow_kept replace the oracle's own per-KV-head choice / final kept
+    set with given ones (used only after a test has checked that they differ from the
+    oracle's own choice at near-ties only)."""
+    Hkv, n_cand = c_pooled.shape
+    if follow_per_kv is not None:
+        per_kv = np.asarray(follow_per_kv[:, :n_cand], dtype=bool)
+    else:
+        per_kv = np.stack([top_k_mask(c_pooled[kv], m_s) for kv in range(Hkv)])
+    union = per_kv.any(axis=0)
+    trimmed = bool(union.sum() > m_s)
+    if trimmed:
+        mean = c_pooled.mean(axis=0)
+        members = np.flatnonzero(union)
+        keep = top_k_mask(mean[members], m_s)
+        kept_cand = np.zeros(n_cand, dtype=bool)
+        kept_cand[members[keep]] = True
+    else:
+        kept_cand = union.copy()
+    kept = np.zeros(n, dtype=bool)
+    kept[:n_cand] = kept_cand
+    kept[n - recent:] = True
+    if follow_kept is not None:
+        kept = np.asarray(follow_kept[:n], dtype=bool).copy()
+        kept_cand = kept[:n_cand].copy()
+    return Selection(per_kv, union, kept_cand, kept, trimmed)
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 3: bucket-attention routing
+# ----------------------------------------------------------------------------------------
+def _best(a_kv: np.ndarray, cands: np.ndarray) -> int:
+    """argmax of a over candidate positions, ties to the lower position (R7)."""
+    best = int(cands[0])
+    for i in cands[1:]:
+        if a_kv[i] > a_kv[best]:
+            best = int(i)
+    return best
+
+
+def route(a_kv: np.ndarray, kept: np.ndarray, bucket: int, empty_policy: int) -> np.ndarray:
+    """Merge target pi(j) for every evicted j of one KV head; -1 for kept tokens and for
+    tokens left without a target (Eq. 3; readings R9-R11).
+
+    The argmax over the kept tokens of bucket(j) of a_kv does not depend on j, so it is
+    found once per bucket."""
+    n = kept.shape[0]
+    nb = (n + bucket - 1) // bucket
+    kept_in = [np.flatnonzero(kept[b * bucket:min(n, (b + 1) * bucket)]) + b * bucket
+               for b in range(nb)]
+    target = np.full(n, -1, dtype=np.int64)
+    for b in range(nb):
+        evicted = [j for j in range(b * bucket, min(n, (b + 1) * bucket)) if not kept[j]]
+        if not evicted:
+            continue
+        t = -1
+        if kept_in[b].size:
+            t = _best(a_kv, kept_in[b])
+        elif empty_policy == EMPTY_EXPAND:
+            r = 1
+            while t < 0 and (b - r >= 0 or b + r < nb):
+                ring = []
+                if b - r >= 0:
+                    ring.extend(kept_in[b - r].tolist())
+                if b + r < nb:
+                    ring.extend(kept_in[b + r].tolist())
+                if ring:
+                    t = _best(a_kv, np.array(sorted(ring)))
+                r += 1
+        for j in evicted:
+            target[j] = t
+    return target
+
+
+def routing_gap(a_kv: np.ndarray, kept: np.ndarray, target: np.ndarray, bucket: int,
+                j: int) -> float:
+    """Relative gap between the chosen target's a and the best other candidate of the same
+    candidate set (used to tell near-ties from real disagreements)."""
+    t = int(target[j])
+    if t < 0:
+        return math.inf
+    b, bt = j // bucket, t // bucket
+    # candidate set: the ring that contains t, at t's bucket distance from j's bucket
+    r = abs(bt - b)
+    n = kept.shape[0]
+    cands = [i for bb in {b - r, b + r} if 0 <= bb * bucket < n
+             for i in range(bb * bucket, min(n, (bb + 1) * bucket)) if kept[i] and i != t]
+    if not cands:
+        return math.inf
+    other = max(a_kv[i] for i in cands)
+    return float((a_kv[t] - other) / max(abs(a_kv[t]), 1e-300))
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 4: soft cosine gate
+# ----------------------------------------------------------------------------------------
+def gate(V_kv: np.ndarray, target: np.ndarray, mode: int):
+    """g_j and sim_j for every routed token (Eq. 4; readings R13, R14).  Tokens without a
+    target get g = 0.  Returns (g, sim, decision) over positions [0, n)."""
+    n = target.shape[0]
+    g = np.zeros(n)
+    sim = np.zeros(n)
+    for j in np.flatnonzero(target >= 0):
+        t = int(target[j])
+        nj = math.sqrt(float(V_kv[j] @ V_kv[j]))
+        nt = math.sqrt(float(V_kv[t] @ V_kv[t]))
+        sim[j] = 0.0 if nj == 0.0 or nt == 0.0 else float(V_kv[j] @ V_kv[t]) / (nj * nt)
+        if mode == GATE_OPEN:
+            g[j] = 1.0
+        elif mode == GATE_CLOSED:
+            g[j] = 0.0
+        else:
+            g[j] = min(max(sim[j], 0.0), 1.0)
+    decision = (g > 0).astype(np.uint8)
+    return g, sim, decision
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 5 + Eq. 6: gated merge and attention ratio
+# ----------------------------------------------------------------------------------------
+def merge(a_kv: np.ndarray, V_kv: np.ndarray, kept_idx: np.ndarray, target: np.ndarray,
+          g: np.ndarray):
+    """For each kept i (in kept_idx order):
+         den_i = a_i + sum_{pi(j)=i} g_j a_j,
+         v~_i  = (a_i v_i + sum_{pi(j)=i} g_j a_j v_j) / den_i          (Eq. 5)
+         R_i   = den_i / a_i                                           (Eq. 6)
+    with the R15 guard.  Returns (V_merged [m][d], R [m])."""
+    m = kept_idx.shape[0]
+    slot = {int(i): s for s, i in enumerate(kept_idx)}
+    num = a_kv[kept_idx][:, None] * V_kv[kept_idx]
+    den = a_kv[kept_idx].copy()
+    for j in np.flatnonzero(target >= 0):
+        s = slot[int(target[j])]
+        w = g[j] * a_kv[j]
+        num[s] += w * V_kv[j]
+        den[s] += w
+    Vm = np.empty_like(num)
+    R = np.ones(m)
+    for s in range(m):
+        i = int(kept_idx[s])
+        Vm[s] = num[s] / den[s] if den[s] > 0 else V_kv[i]
+        if a_kv[i] > 0:
+            R[s] = den[s] / a_kv[i]
+    return Vm, R
+
+
+def gqa_bias(R: np.ndarray, alpha: float) -> np.ndarray:
+    """Sec. 3.5 for GQA: bias_i = alpha * ln(mean over KV heads of R_{kv,i}) (R16).
+    R: [Hkv][m]."""
+    return alpha * np.log(R.mean(axis=0))
+
+
+# ----------------------------------------------------------------------------------------
+# Algorithm 1 for one sequence of one layer
+# ----------------------------------------------------------------------------------------
+@dataclass
+class CompressResult:
+    m: int
+    m_s: int
+    a: np.ndarray             # [Hkv][n] cumulative attention
+    vnorm: np.ndarray         # [Hkv][n]
+    c: np.ndarray             # [Hkv][n] contribution score (Eq. 1)
+    c_pooled: np.ndarray      # [Hkv][n_cand]
+    sel: Selection
+    kept_idx: np.ndarray      # [m] ascending
+    target: np.ndarray        # [Hkv][n]
+    g: np.ndarray             # [Hkv][n]
+    sim: np.ndarray           # [Hkv][n]
+    decision: np.ndarray      # [Hkv][n] uint8 (valid where target >= 0 or policy dropped)
+    K_c: np.ndarray           # [Hkv][m][d]
+    V_c: np.ndarray           # [Hkv][m][d]
+    R: np.ndarray             # [Hkv][m]
+    bias: np.ndarray          # [m]
+    extra: dict = field(default_factory=dict)
+
+
+def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
+             params: Params = Params(), follow_per_kv=None, follow_kept=None,
+             follow_target=None) -> CompressResult:
+    """Algorithm 1, steps 1-6, for one sequence of one layer (step 7, RoPE repositioning, is
+    off).  K, V: [Hkv][>=n][d]; Q: [Hq][W][d]; all float64.
+
+    follow_* replace a discrete choice of the oracle by a given one (per-KV-head top-k
+    masks, final kept mask, merge targets), so that a test can compare the continuous
+    outputs downstream of a near-tie the two sides resolved differently."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Q = np.asarray(Q, dtype=np.float64)
+    Hkv = K.shape[0]
+    m, m_s = budget(n, rho, params.recent)
+    if m_s < 0 or Q.shape[1] > n:
+        raise ValueError("budget below the recent window, or window longer than the sequence")
+    n_cand = n - params.recent
+    a = cumulative_attention(Q, K, n)                         # step 1 (re-pass)
+    vn = value_norms(V, n)
+    c = a * vn                                                # Eq. 1
+    cp = pool_scores(c, n_cand, params.pool_kernel)           # smoothing
+    sel = select_shared(cp, n, m_s, params.recent, follow_per_kv, follow_kept)  # step 2
+    kept_idx = np.flatnonzero(sel.kept)
+    target = np.full((Hkv, n), -1, dtype=np.int64)
+    g = np.zeros((Hkv, n))
+    sim = np.zeros((Hkv, n))
+    decision = np.zeros((Hkv, n), dtype=np.uint8)
+    Vc = np.empty((Hkv, kept_idx.size, K.shape[2]))
+    R = np.ones((Hkv, kept_idx.size))
+    for kv in range(Hkv):
+        t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
+             else route(a[kv], sel.kept, params.bucket, params.empty_bucket))   # step 3
+        target[kv] = t
+        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
+        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # steps 5, 6
+    bias = gqa_bias(R, params.alpha)
+    return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=sel,
+                          kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
+                          K_c=K[:, kept_idx].copy(), V_c=Vc, R=R, bias=bias)
+
+
+# ----------------------------------------------------------------------------------------
+# Decode with the compensated cache (Alg. 1, last step; Sec. 3.5)
+# ----------------------------------------------------------------------------------------
+def decode(q: np.ndarray, K_c: np.ndarray, V_c: np.ndarray, bias: Optional[np.ndarray],
+           length: int) -> np.ndarray:
+    """out[h] = sum_{i < length} softmax_i(q_h . k_{kv(h),i} / sqrt(d) + bias_{kv(h),i}) v_i.
+
+    q: [Hq][d]; K_c, V_c: [Hkv][>=length][d]; bias: None, [>=length] (shared by every head)
+    or [Hkv][>=length].  Returns [Hq][d] float64."""
+    q = np.asarray(q, dtype=np.float64)
+    Hq, d = q.shape
+    Hkv = K_c.shape[0]
+    G = Hq // Hkv
+    out = np.zeros((Hq, d))
+    for h in range(Hq):
+        kv = h // G
+        s = (np.asarray(K_c[kv, :length], dtype=np.float64) @ q[h]) / math.sqrt(d)
+        if bias is not None:
+            b = np.asarray(bias, dtype=np.float64)
+            s = s + (b[kv, :length] if b.ndim == 2 else b[:length])
+        s = s - s.max()
+        p = np.exp(s)
+        p /= p.sum()
+        out[h] = p @ np.asarray(V_c[kv, :length], dtype=np.float64)
+    return out

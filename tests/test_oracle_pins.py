@@ -1,0 +1,375 @@
+"""Pins for the fp64 oracle: closed forms, hand-worked examples (tests/golden/), library
+routines and brute force on tiny inputs, chosen so that a dropped term, a wrong sign or index,
+a transposed operand or a wrong tie-break in the oracle fails at least one of them.
+
+CPU only."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import selkv_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def rng(seed):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- Sec. 3.1: budget
+def test_budget_floor_and_recent_window():
+    # m = floor(rho n), m_s = m - m_r (Sec. 3.1); 25% of 1024 is 256 entries, 240 by score
+    assert O.budget(1024, 0.25, 16) == (256, 240)
+    assert O.budget(1023, 0.25, 16) == (255, 239)      # floor, not round
+    assert O.budget(100000, 0.25, 16) == (25000, 24984)
+    assert O.budget(40, 0.25, 16) == (10, -6)          # below the recent window: invalid
+
+
+# ---------------------------------------------------------------- Sec. 3.1 re-pass
+def test_uniform_keys_closed_form():
+    """With all keys equal every visible score ties, so row i spreads 1/(p_i+1) over
+    j <= p_i = n-W+i.  Then a_j = H_n - H_max(j, n-W) (harmonic numbers): this pins the
+    causal direction, the window's positions and the average over the query group."""
+    n, W, d, Hq, Hkv = 50, 8, 4, 4, 2
+    Q = rng(1).standard_normal((Hq, W, d))
+    K = np.ones((Hkv, n, d))
+    a = O.cumulative_attention(Q, K, n)
+    H = np.concatenate([[0.0], np.cumsum(1.0 / np.arange(1, n + 1))])
+    expect = np.array([H[n] - H[max(j, n - W)] for j in range(n)])
+    for kv in range(Hkv):
+        np.testing.assert_allclose(a[kv], expect, rtol=1e-13, atol=1e-15)
+    assert abs(a.sum(axis=1) - W).max() < 1e-12      # each window row carries mass 1
+
+
+def test_observation_attention_matches_torch_sdpa():
+    """Library pin: torch SDPA in fp64 with identity values returns the attention matrix
+    itself (default scale 1/sqrt(d), boolean mask True = visible)."""
+    n, W, d, Hq, Hkv = 37, 6, 8, 4, 2
+    r = rng(2)
+    Q = r.standard_normal((Hq, W, d)) * 2
+    K = r.standard_normal((Hkv, n, d))
+    A = O.observation_attention(Q, K, n)
+    G = Hq // Hkv
+    pos = n - W + np.arange(W)
+    mask = torch.from_numpy(np.arange(n)[None, :] <= pos[:, None])
+    for h in range(Hq):
+        out = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(Q[h])[None], torch.from_numpy(K[h // G, :n])[None],
+            torch.eye(n, dtype=torch.float64)[None], attn_mask=mask[None])
+        np.testing.assert_allclose(A[h], out[0].numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(A.sum(axis=2), 1.0, rtol=1e-13)
+
+
+def test_cumulative_attention_brute_force():
+    n, W, d, Hq, Hkv = 12, 3, 2, 4, 2
+    r = rng(3)
+    Q, K = r.standard_normal((Hq, W, d)), r.standard_normal((Hkv, n, d))
+    G = Hq // Hkv
+    a = O.cumulative_attention(Q, K, n)
+    brute = np.zeros((Hkv, n))
+    for h in range(Hq):
+        for i in range(W):
+            p = n - W + i
+            logits = [sum(Q[h, i, t] * K[h // G, j, t] for t in range(d)) / math.sqrt(d)
+                      for j in range(p + 1)]
+            mx = max(logits)
+            w = [math.exp(x - mx) for x in logits]
+            z = sum(w)
+            for j in range(p + 1):
+                brute[h // G, j] += w[j] / z / G
+    np.testing.assert_allclose(a, brute, rtol=1e-12)
+
+
+# ---------------------------------------------------------------- Eq. 1 + pooling
+def test_contribution_score_is_attention_times_value_norm():
+    a = np.array([[0.5, 2.0, 0.0]])
+    V = np.array([[[3.0, 4.0], [1.0, 0.0], [7.0, 7.0]]])
+    np.testing.assert_allclose(O.contribution_scores(a, V, 3), [[2.5, 2.0, 0.0]])
+
+
+def test_pool_impulse_and_edges():
+    n_cand, k = 10, 5
+    c = np.zeros((1, 14))
+    c[0, 4] = 1.0
+    np.testing.assert_allclose(O.pool_scores(c, n_cand, k)[0],
+                               [0, 0, .2, .2, .2, .2, .2, 0, 0, 0], atol=1e-15)
+    c = np.zeros((1, 14))
+    c[0, 9] = 1.0          # last candidate: only the left neighbours see it
+    c[0, 10:] = 100.0      # recent window: never pooled in
+    np.testing.assert_allclose(O.pool_scores(c, n_cand, k)[0],
+                               [0, 0, 0, 0, 0, 0, 0, .2, .2, .2], atol=1e-15)
+    ones = np.ones((1, n_cand))
+    np.testing.assert_allclose(O.pool_scores(ones, n_cand, 5)[0],
+                               [.6, .8, 1, 1, 1, 1, 1, 1, .8, .6], atol=1e-15)
+
+
+# ---------------------------------------------------------------- Eq. 2 + Sec. 3.3
+def test_top_k_brute_force_with_ties():
+    r = rng(4)
+    for trial in range(200):
+        n = int(r.integers(1, 30))
+        vals = r.integers(0, 5, size=n).astype(float)    # many ties
+        k = int(r.integers(0, n + 1))
+        chosen, left = [], list(range(n))
+        for _ in range(k):                               # repeated argmax, lowest index
+            best = left[0]
+            for j in left[1:]:
+                if vals[j] > vals[best]:
+                    best = j
+            chosen.append(best)
+            left.remove(best)
+        expect = np.zeros(n, dtype=bool)
+        expect[chosen] = True
+        assert (O.top_k_mask(vals, k) == expect).all()
+
+
+def test_union_trim_worked_example():
+    gd = golden("union_trim.json")
+    cp = np.array(gd["c_pooled"], dtype=float)
+    sel = O.select_shared(cp, gd["n"], gd["m_s"], gd["recent"])
+    for kv, expect in enumerate(gd["per_kv"]):
+        assert np.flatnonzero(sel.per_kv[kv]).tolist() == expect
+    assert np.flatnonzero(sel.union).tolist() == gd["union"]
+    assert sel.trimmed
+    assert np.flatnonzero(sel.kept).tolist() == gd["kept"]
+
+
+def test_union_without_trim_is_shared_topk():
+    cp = np.array([[3, 1, 2, 0], [3, 0, 2, 1]], dtype=float)
+    sel = O.select_shared(cp, 6, 2, 2)
+    assert not sel.trimmed
+    assert np.flatnonzero(sel.kept).tolist() == [0, 2, 4, 5]
+
+
+# ---------------------------------------------------------------- Eq. 3
+def test_routing_worked_example():
+    gd = golden("routing.json")
+    n, B = gd["n"], gd["bucket"]
+    kept = np.zeros(n, dtype=bool)
+    kept[gd["kept"]] = True
+    a = np.full(n, 0.01)
+    for k, v in gd["a"].items():
+        a[int(k)] = v
+    t = O.route(a, kept, B, O.EMPTY_EXPAND)
+    expect = {int(k): v for k, v in gd["expand"].items()}
+    for j in range(n):
+        assert t[j] == (expect[j] if j in expect else -1), j
+    t = O.route(a, kept, B, O.EMPTY_DROP)
+    for j in range(n):
+        if j in gd["drop_policy_untargeted"] or kept[j]:
+            assert t[j] == -1
+        else:
+            assert t[j] == expect[j]
+
+
+def test_routing_brute_force():
+    """Explicit scan: for each evicted j, the kept i of the nearest non-empty ring of
+    buckets with the largest a (lowest index on ties)."""
+    r = rng(5)
+    for trial in range(30):
+        n, B = int(r.integers(8, 90)), int(r.integers(2, 9))
+        kept = r.random(n) < 0.15
+        kept[-1] = True
+        a = r.integers(1, 6, size=n).astype(float)
+        t = O.route(a, kept, B, O.EMPTY_EXPAND)
+        for j in range(n):
+            if kept[j]:
+                assert t[j] == -1
+                continue
+            best = None
+            for dist in range(n):
+                cands = [i for i in range(n) if kept[i] and abs(i // B - j // B) == dist]
+                if cands:
+                    best = min(cands, key=lambda i: (-a[i], i))
+                    break
+            assert t[j] == best
+
+
+# ---------------------------------------------------------------- Eq. 4-6, Sec. 3.5
+def test_gate_merge_ratio_worked_example():
+    gd = golden("gate_merge.json")
+    V = np.array([gd["v_target"]] + gd["contributors"], dtype=float)
+    a = np.array([gd["a_target"]] + gd["a_contrib"])
+    target = np.array([-1] + [0] * len(gd["contributors"]))
+    g, sim, dec = O.gate(V, target, O.GATE_COSINE)
+    np.testing.assert_allclose(g[1:], gd["g"], atol=1e-15)
+    assert dec[1:].tolist() == gd["decision"]
+    Vm, R = O.merge(a, V, np.array([0]), target, g)
+    np.testing.assert_allclose(Vm[0], gd["v_merged"], rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(R[0], gd["R"], rtol=1e-14)
+    np.testing.assert_allclose(O.gqa_bias(R[None], 0.5)[0], gd["bias"], rtol=1e-14)
+
+
+def test_gqa_bias_is_log_of_mean_ratio():
+    gd = golden("gqa_bias.json")
+    np.testing.assert_allclose(O.gqa_bias(np.array(gd["R"]), gd["alpha"]), gd["bias"],
+                               rtol=1e-14, atol=1e-16)
+
+
+def test_gate_modes():
+    V = np.array([[1.0, 0], [-1.0, 0], [0.6, 0.8]])
+    t = np.array([-1, 0, 0])
+    assert O.gate(V, t, O.GATE_OPEN)[0].tolist() == [0, 1, 1]
+    assert O.gate(V, t, O.GATE_CLOSED)[0].tolist() == [0, 0, 0]
+    np.testing.assert_allclose(O.gate(V, t, O.GATE_COSINE)[0], [0, 0, 0.6])
+
+
+# ---------------------------------------------------------------- whole pipeline
+def _tiny(seed=0, **kw):
+    wl = synth.WORKLOADS["tiny"].with_(seed=seed, **kw)
+    x = synth.gen_layer(wl, 0)
+    n = int(x["n_len"][0])
+    return wl, x["K"][0].astype(float), x["V"][0].astype(float), x["Q_obs"][0].astype(float), n
+
+
+def test_gate_closed_is_pure_eviction():
+    """g = 0 everywhere reduces Eq. 5 to dropping (Sec. 3.4; ablation 'eviction only')."""
+    wl, K, V, Q, n = _tiny()
+    r = O.compress(K, V, Q, n, wl.rho, O.Params(gate_mode=O.GATE_CLOSED))
+    # (a_i v_i) / a_i is v_i up to one rounding of fp64
+    np.testing.assert_allclose(r.V_c, V[:, r.kept_idx], rtol=1e-15, atol=0)
+    np.testing.assert_array_equal(r.K_c, K[:, r.kept_idx])
+    np.testing.assert_array_equal(r.R, 1.0)
+    np.testing.assert_array_equal(r.bias, 0.0)
+    assert (r.decision[r.target >= 0] == O.DECISION_DROP).all()
+
+
+def test_gate_open_is_attention_weighted_merge():
+    """g = 1 reduces Eq. 5 to the attention-weighted average of each kept token and the
+    tokens routed to it (Sec. 3.4; ablation 'merge all'), computed here by explicit scans."""
+    wl, K, V, Q, n = _tiny(seed=1)
+    r = O.compress(K, V, Q, n, wl.rho, O.Params(gate_mode=O.GATE_OPEN))
+    for kv in range(K.shape[0]):
+        for s, i in enumerate(r.kept_idx):
+            group = [i] + [j for j in range(n) if r.target[kv, j] == i]
+            w = np.array([r.a[kv, j] for j in group])
+            expect = sum(w[t] * V[kv, j] for t, j in enumerate(group)) / w.sum()
+            np.testing.assert_allclose(r.V_c[kv, s], expect, rtol=1e-12, atol=1e-14)
+            np.testing.assert_allclose(r.R[kv, s], w.sum() / r.a[kv, i], rtol=1e-12)
+
+
+def test_full_budget_is_full_attention():
+    """rho = 1 evicts nothing: the cache is unchanged, R = 1, bias = 0, and decode is
+    exact full attention (checked against torch SDPA in fp64)."""
+    wl, K, V, Q, n = _tiny(seed=2)
+    r = O.compress(K, V, Q, n, 1.0)
+    assert r.kept_idx.tolist() == list(range(n))
+    np.testing.assert_allclose(r.V_c, V[:, :n], rtol=1e-15, atol=0)
+    np.testing.assert_array_equal(r.bias, 0.0)
+    q = rng(6).standard_normal((wl.num_q_heads, wl.head_dim))
+    out = O.decode(q, r.K_c, r.V_c, r.bias, n)
+    G = wl.group
+    for h in range(wl.num_q_heads):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[h])[None, None], torch.from_numpy(K[h // G, :n])[None],
+            torch.from_numpy(V[h // G, :n])[None])
+        np.testing.assert_allclose(out[h], ref[0, 0].numpy(), rtol=1e-11, atol=1e-13)
+
+
+def test_decode_bias_matches_sdpa_additive_mask():
+    r = rng(7)
+    Hq, Hkv, L, d = 4, 2, 23, 8
+    q = r.standard_normal((Hq, d))
+    Kc, Vc = r.standard_normal((Hkv, L, d)), r.standard_normal((Hkv, L, d))
+    bias = r.random(L) * 2
+    out = O.decode(q, Kc, Vc, bias, L)
+    for h in range(Hq):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[h])[None, None], torch.from_numpy(Kc[h // 2])[None],
+            torch.from_numpy(Vc[h // 2])[None], attn_mask=torch.from_numpy(bias)[None, None])
+        np.testing.assert_allclose(out[h], ref[0, 0].numpy(), rtol=1e-12, atol=1e-14)
+
+
+def test_merged_duplicates_recover_softmax_mass():
+    """m identical tokens merged into one kept copy with g = 1 and equal attention give
+    R = m; with alpha = 1 the bias is ln m and decode over the compressed cache equals decode
+    over the full cache exactly (the attention-sag correction of Sec. 3.5)."""
+    r = rng(8)
+    Hq, Hkv, W, d, n, B = 2, 1, 4, 8, 64, 32
+    K = r.standard_normal((Hkv, n, d))
+    V = r.standard_normal((Hkv, n, d))
+    dup = list(range(40, 45))                   # 5 identical tokens in bucket 1
+    K[:, dup] = K[:, dup[:1]]
+    V[:, dup] = V[:, dup[:1]]
+    Q = r.standard_normal((Hq, W, d))
+    kept = np.ones(n, dtype=bool)
+    kept[dup[1:]] = False                       # keep the first copy only
+    rho = kept.sum() / n
+    target = np.full((Hkv, n), -1)
+    target[:, dup[1:]] = dup[0]                 # the copies route to their kept twin
+    res = O.compress(K, V, Q, n, rho, O.Params(alpha=1.0, recent=0, bucket=B),
+                     follow_kept=kept, follow_target=target)
+    s = int(np.flatnonzero(res.kept_idx == dup[0])[0])
+    np.testing.assert_allclose(res.g[0, dup[1:]], 1.0, rtol=1e-15)
+    np.testing.assert_allclose(res.R[0, s], len(dup), rtol=1e-13)
+    np.testing.assert_allclose(res.bias[s], math.log(len(dup)), rtol=1e-13)
+    others = np.delete(np.arange(res.kept_idx.size), s)
+    np.testing.assert_allclose(res.bias[others], 0.0, atol=1e-15)
+    q = r.standard_normal((Hq, d))
+    full = O.decode(q, K, V, None, n)
+    comp = O.decode(q, res.K_c, res.V_c, res.bias, res.kept_idx.size)
+    np.testing.assert_allclose(comp, full, rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("seed,dtype", [(0, "fp32"), (3, "bf16")])
+def test_pipeline_invariants(seed, dtype):
+    wl, K, V, Q, n = _tiny(seed=seed, dtype=dtype)
+    p = O.Params()
+    r = O.compress(K, V, Q, n, wl.rho, p)
+    m, m_s = O.budget(n, wl.rho, p.recent)
+    assert r.kept_idx.size == m and (np.diff(r.kept_idx) > 0).all()
+    assert set(range(n - p.recent, n)) <= set(r.kept_idx.tolist())
+    assert int(r.sel.kept_cand.sum()) == m_s
+    Hkv = K.shape[0]
+    for kv in range(Hkv):
+        ev = np.flatnonzero(~r.sel.kept)
+        t = r.target[kv, ev]
+        assert (t >= 0).all()                                 # everyone has a target
+        assert r.sel.kept[t].all()
+        nonempty = np.array([r.sel.kept[(j // p.bucket) * p.bucket:
+                                        (j // p.bucket + 1) * p.bucket].any() for j in ev])
+        assert (t[nonempty] // p.bucket == ev[nonempty] // p.bucket).all()
+        assert (r.R[kv] >= 1.0 - 1e-15).all()
+        contributed = np.zeros(r.kept_idx.size, dtype=bool)
+        slot = {int(i): s for s, i in enumerate(r.kept_idx)}
+        for j in ev:
+            if r.g[kv, j] > 0:
+                contributed[slot[int(r.target[kv, j])]] = True
+        assert (r.R[kv][~contributed] == 1.0).all()
+        lhs = (r.a[kv, r.kept_idx] * r.R[kv]).sum()            # mass conservation
+        rhs = r.a[kv, r.kept_idx].sum() + (r.g[kv, ev] * r.a[kv, ev]).sum()
+        assert abs(lhs - rhs) <= 1e-12 * rhs
+        for s, i in enumerate(r.kept_idx):                     # convex hull
+            members = [i] + [j for j in ev if r.target[kv, j] == i and r.g[kv, j] > 0]
+            lo, hi = V[kv, members].min(axis=0), V[kv, members].max(axis=0)
+            assert (r.V_c[kv, s] >= lo - 1e-12).all() and (r.V_c[kv, s] <= hi + 1e-12).all()
+    q = rng(9).standard_normal((wl.num_q_heads, wl.head_dim))
+    r0 = O.compress(K, V, Q, n, wl.rho, O.Params(alpha=0.0))
+    np.testing.assert_array_equal(r0.bias, 0.0)                 # alpha = 0: no compensation
+    np.testing.assert_allclose(O.decode(q, r0.K_c, r0.V_c, r0.bias, m),
+                               O.decode(q, r0.K_c, r0.V_c, None, m), rtol=1e-14, atol=1e-15)
+
+
+def test_follow_mode_reproduces_own_choices():
+    wl, K, V, Q, n = _tiny(seed=4)
+    r = O.compress(K, V, Q, n, wl.rho)
+    f = O.compress(K, V, Q, n, wl.rho, follow_per_kv=r.sel.per_kv, follow_kept=r.sel.kept,
+                   follow_target=r.target)
+    np.testing.assert_array_equal(f.V_c, r.V_c)
+    np.testing.assert_array_equal(f.bias, r.bias)
+
+
+def test_rejects_budget_below_recent_window():
+    wl, K, V, Q, n = _tiny()
+    with pytest.raises(ValueError):
+        O.compress(K, V, Q, n, 0.01)
