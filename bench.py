@@ -1,0 +1,475 @@
+"""SelKV benchmark: one-shot compression of a 32-layer GQA cache followed by compensated
+decode, on synthetic inputs of the paper's latency setting (Llama-3-8B attention shape,
+100k-token context, 25% budget, 256 generated tokens).
+
+One step = compress every layer (selkv_compress) + decode_steps tokens, each token running
+selkv_decode_attn on every layer with a fresh query and an appended key/value row.
+`value` = generated tokens / step time (compression included); the decode-only rate,
+compress ms per layer, decode GB/s and the roofline of the decode kernel are reported beside
+it.  Inputs are resident in HBM when the timed region starts; `e2e` repeats the step through
+the public API from pinned host buffers with the copies inside the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload long_100k]
+  python bench.py --impl reference ...    (the fp64 CPU oracle on a bounded sample)
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "compensated decode tokens/s & HBM GB/s (% peak) at 100k ctx; compress ms/layer"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------------------ oracle arm
+def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2):
+    """Time the fp64 oracle on a bounded sample of one step of `wl`: compression of `layers`
+    layers of sequence 0 and `decode_tokens` decode tokens over those layers; the rates are
+    scaled to the whole step (all layers, all sequences, all decode steps)."""
+    from oracle import selkv_oracle as O
+    t_comp = 0.0
+    t_dec = 0.0
+    ncomp = 0
+    ndec = 0
+    for layer in range(layers):
+        x = synth.gen_layer(wl.with_(batch=1), layer, threads=os.cpu_count() or 1)
+        n = int(x["n_len"][0])
+        K, V, Q = (x["K"][0].astype(np.float64), x["V"][0].astype(np.float64),
+                   x["Q_obs"][0].astype(np.float64))
+        t0 = time.perf_counter()
+        r = O.compress(K, V, Q, n, wl.rho)
+        t_comp += time.perf_counter() - t0
+        ncomp += 1
+        dec = synth.gen_decode(wl.with_(batch=1), layer, decode_tokens)
+        Kc, Vc, bias = r.K_c, r.V_c, r.bias
+        for t in range(decode_tokens):
+            Kc = np.concatenate([Kc, dec["k_new"][t, 0][:, None]], axis=1)
+            Vc = np.concatenate([Vc, dec["v_new"][t, 0][:, None]], axis=1)
+            bias = np.concatenate([bias, [0.0]])
+            t0 = time.perf_counter()
+            O.decode(dec["q"][t, 0], Kc, Vc, bias, Kc.shape[1])
+            t_dec += time.perf_counter() - t0
+            ndec += 1
+    per_layer_comp = t_comp / ncomp
+    per_layer_tok = t_dec / ndec
+    step_s = wl.batch * wl.layers * (per_layer_comp + wl.decode_steps * per_layer_tok)
+    tokens = wl.batch * wl.decode_steps
+    sample = ("fp64 oracle: compression of %d layer(s) x 1 sequence (n=%d) and %d decode token(s) "
+              "per layer, scaled to %d layers x %d sequences x %d decode steps"
+              % (layers, wl.n, decode_tokens, wl.layers, wl.batch, wl.decode_steps))
+    return dict(value=tokens / step_s, unit="tokens/s", cores=os.cpu_count(), kind="oracle",
+                sample=sample, compress_s_per_layer=per_layer_comp,
+                decode_s_per_layer_token=per_layer_tok, sample_wall_s=t_comp + t_dec)
+
+
+# ------------------------------------------------------------------------------ GPU arm
+class Layered:
+    """Device-resident inputs and outputs of every layer."""
+
+    def __init__(self, wl, torch, api, S, dev, pinned_host: bool):
+        self.wl = wl
+        B, Hq, Hkv, d, W = wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.obs_window
+        tdt = api.torch_dtype(api.dtype_code(wl.dtype))
+        self.n_len = [int(v) for v in synth.seq_lengths(wl)]
+        self.T = wl.decode_steps
+        self.m_cap = api.capacity(max(self.n_len), wl.rho, extra=self.T + 1)
+        self.shape = api.make_shape(wl.dtype, B, Hq, Hkv, d, W, wl.n, self.m_cap)
+        self.K, self.V, self.Q, self.caches, self.host = [], [], [], [], []
+        threads = os.cpu_count() or 1
+        for layer in range(wl.layers):
+            x = synth.gen_layer(wl, layer, threads=threads)
+            K = torch.from_numpy(x["K"]).to(dev).to(tdt)
+            V = torch.from_numpy(x["V"]).to(dev).to(tdt)
+            Q = torch.from_numpy(x["Q_obs"]).to(dev).to(tdt)
+            self.K.append(K)
+            self.V.append(V)
+            self.Q.append(Q)
+            if pinned_host:
+                self.host.append(tuple(t.cpu().pin_memory() for t in (K, V, Q)))
+            self.caches.append(api.alloc_compressed(self.shape, dev))
+        # decode inputs for every (step, layer): q [T][L][B][Hq][d], k/v [T][L][B][Hkv][d]
+        qs, ks, vs = [], [], []
+        for layer in range(wl.layers):
+            dd = synth.gen_decode(wl, layer, self.T)
+            qs.append(dd["q"])
+            ks.append(dd["k_new"])
+            vs.append(dd["v_new"])
+        self.dq = torch.from_numpy(np.stack(qs, 1)).to(dev).to(tdt)
+        self.dk = torch.from_numpy(np.stack(ks, 1)).to(dev).to(tdt)
+        self.dv = torch.from_numpy(np.stack(vs, 1)).to(dev).to(tdt)
+        self.out = torch.empty((self.T, wl.layers, B, Hq, d), dtype=tdt, device=dev)
+        self.cws = api.Workspace(S.selkv_compress_workspace_size(self.shape), dev)
+        self.dws = api.Workspace(S.selkv_decode_workspace_size(self.shape), dev)
+
+
+def issue_step(L: Layered, S, params, stream_ptr, decode_ranges=None):
+    """Enqueue one step on the stream; returns the number of kernels enqueued."""
+    wl = L.wl
+    k0 = S.selkv_kernel_launches()
+    for layer in range(wl.layers):
+        c = L.caches[layer]
+        S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
+                                 c.K_c, c.V_c, c.bias, c.lengths, None, L.cws.buf, L.cws.nbytes,
+                                 stream_ptr), "compress")
+    if decode_ranges is not None:
+        decode_ranges[0]()
+    for t in range(L.T):
+        for layer in range(wl.layers):
+            c = L.caches[layer]
+            S.check(S.selkv_decode_attn(L.shape, L.dq[t, layer], c.K_c, c.V_c, c.bias, c.lengths,
+                                        L.dk[t, layer], L.dv[t, layer], L.out[t, layer],
+                                        L.dws.buf, L.dws.nbytes, stream_ptr), "decode")
+    return S.selkv_kernel_launches() - k0
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+    import paper_2607_16213_gb300 as S
+    from paper_2607_16213_gb300 import api, build as _build
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    _build.build()
+    S.library()
+    wl = synth.WORKLOADS[args.workload]
+    if args.decode_steps is not None:
+        wl = wl.with_(decode_steps=args.decode_steps)
+    if args.layers is not None:
+        wl = wl.with_(layers=args.layers)
+    params = S.selkv_params.defaults()
+    L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e)
+    stream = torch.cuda.Stream(device=dev)
+    sp = stream.cuda_stream
+    peaks, peak_src = load_peaks()
+
+    with torch.cuda.stream(stream):
+        launches_per_step = issue_step(L, S, params, sp)   # one eager step (also warms up)
+    torch.cuda.synchronize()
+    assert L.cws.errors(sp) == 0 and L.dws.errors(sp) == 0, "device error flags"
+
+    # capture compression and decode as two graphs, so the timed region is launch-free
+    g_comp = torch.cuda.CUDAGraph()
+    g_dec = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_comp, stream=stream):
+        for layer in range(wl.layers):
+            c = L.caches[layer]
+            S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
+                                     c.K_c, c.V_c, c.bias, c.lengths, None, L.cws.buf, L.cws.nbytes,
+                                     stream.cuda_stream), "compress")
+    with torch.cuda.graph(g_dec, stream=stream):
+        for t in range(L.T):
+            for layer in range(wl.layers):
+                c = L.caches[layer]
+                S.check(S.selkv_decode_attn(L.shape, L.dq[t, layer], c.K_c, c.V_c, c.bias, c.lengths,
+                                            L.dk[t, layer], L.dv[t, layer], L.out[t, layer],
+                                            L.dws.buf, L.dws.nbytes, stream.cuda_stream), "decode")
+    n_dec_launch = L.T * wl.layers
+    for _ in range(args.warmup):
+        g_comp.replay()
+        g_dec.replay()
+    torch.cuda.synchronize()
+
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(torch.cuda.current_device() if not os.environ.get("CUDA_VISIBLE_DEVICES") else 0)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_wall = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            g_comp.replay()
+            ev[k][1].record(stream)
+            g_dec.replay()
+            ev[k][2].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t_wall
+    clk = clocks.stop()
+    comp_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
+    dec_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
+    step_ms_total = ev[0][0].elapsed_time(ev[-1][2])
+    if world > 1:
+        t = torch.tensor([step_ms_total], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms_total = float(t.item())
+        dist.barrier()
+    ms_per_step = step_ms_total / args.steps
+    tokens_per_step = wl.batch * L.T
+    value = world * tokens_per_step * args.steps / (step_ms_total / 1e3)
+    dec_ms_avg = sum(dec_ms) / len(dec_ms)
+    comp_ms_avg = sum(comp_ms) / len(comp_ms)
+    decode_tok_s = tokens_per_step / (dec_ms_avg / 1e3)
+
+    # algorithmic bytes of the decode kernel per launch: each cached row of each KV head
+    # reads K_c and V_c (d elements each) and one fp32 bias; plus q, out, k_new, v_new.
+    esz = 2 if wl.dtype == "bf16" else 4
+    d, Hkv, Hq, B = wl.head_dim, wl.num_kv_heads, wl.num_q_heads, wl.batch
+    m_b = [int(math.floor(wl.rho * n)) for n in L.n_len]
+    per_row = Hkv * (2 * d * esz + 4)
+    rows_total = sum(sum(m + t + 1 for t in range(L.T)) for m in m_b)   # over the T steps
+    fixed = L.T * B * (2 * Hq * d * esz + 2 * Hkv * d * esz)
+    dec_bytes_per_layer_step = (rows_total * per_row + fixed) / L.T
+    dec_launch_us = dec_ms_avg * 1e3 / n_dec_launch
+    achieved_gbs = dec_bytes_per_layer_step / (dec_launch_us * 1e-6) / 1e9
+    peak_hbm = float(peaks["hbm_gbs"])
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "decode_traffic.json")
+    if os.path.exists(prof):
+        with open(prof) as f:
+            pj = json.load(f)
+        if pj.get("workload") == wl.name and pj.get("kernel_rev") == kernel_revision():
+            traffic = pj.get("bytes_per_launch")
+
+    # full-cache comparison (same kernel, bias = NULL, uncompressed cache, no append)
+    full_tok_s = None
+    if not args.no_full:
+        fshape = api.make_shape(wl.dtype, B, Hq, Hkv, d, wl.obs_window, wl.n, wl.n)
+        flen = torch.tensor(L.n_len, dtype=torch.int32, device=dev)
+        fws = api.Workspace(S.selkv_decode_workspace_size(fshape), dev)
+        nfull = max(2, min(16, L.T))
+        def full_pass():
+            for t in range(nfull):
+                for layer in range(wl.layers):
+                    S.check(S.selkv_decode_attn(fshape, L.dq[t, layer], L.K[layer], L.V[layer], None, flen,
+                                                None, None, L.out[t, layer], fws.buf, fws.nbytes, sp), "full")
+        with torch.cuda.stream(stream):
+            full_pass()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            full_pass()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        full_tok_s = B * nfull / (e0.elapsed_time(e1) / 1e3)
+
+    # end to end through the public API from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(L, S, api, torch, params, stream, dev, min(args.steps, 2))
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
+                   "rho": wl.rho, "decode_steps": L.T, "q_heads": Hq, "kv_heads": Hkv,
+                   "head_dim": d, "obs_window": wl.obs_window, "parallelism": "replicas",
+                   "l2": "inputs larger than L2: every token streams all layers' compressed "
+                         "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
+                   "cuda_graph": True},
+        "decode_tok_s": decode_tok_s,
+        "decode_gbs": achieved_gbs,
+        "compress_ms_per_layer": comp_ms_avg / wl.layers,
+        "full_cache_decode_tok_s": full_tok_s,
+        "decode_speedup_vs_full_cache": (decode_tok_s / full_tok_s) if full_tok_s else None,
+        "roofline": {"kernel": "selkv decode (split-K, GQA, bias in softmax)", "bound": "hbm",
+                     "achieved": achieved_gbs, "peak": peak_hbm, "unit": "GB/s",
+                     "frac": achieved_gbs / peak_hbm, "peak_source": peak_src,
+                     "bytes_per_launch": dec_bytes_per_layer_step,
+                     "launch_us": dec_launch_us, "traffic": traffic},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+        "wall_s_timed": wall,
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_sample(wl)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int):
+    """The step through the public API with pinned host inputs: copy each layer's K, V, Q_obs
+    to the device, compress, then per token copy q / k_new / v_new in, decode every layer and
+    read the token's outputs back."""
+    wl = L.wl
+    sp = stream.cuda_stream
+    hq = L.dq.cpu().pin_memory()
+    hk = L.dk.cpu().pin_memory()
+    hv = L.dv.cpu().pin_memory()
+    hout = torch.empty(L.out.shape[1:], dtype=L.out.dtype).pin_memory()
+    dq = torch.empty_like(L.dq[0])
+    dk = torch.empty_like(L.dk[0])
+    dv = torch.empty_like(L.dv[0])
+    h2d = sum(t.numel() * t.element_size() for trip in L.host for t in trip) + \
+        L.T * (dq.numel() + dk.numel() + dv.numel()) * dq.element_size()
+    d2h = L.T * hout.numel() * hout.element_size()
+
+    def one():
+        with torch.cuda.stream(stream):
+            for layer in range(wl.layers):
+                hK, hV, hQ = L.host[layer]
+                L.K[layer].copy_(hK, non_blocking=True)
+                L.V[layer].copy_(hV, non_blocking=True)
+                L.Q[layer].copy_(hQ, non_blocking=True)
+                c = L.caches[layer]
+                api.compress(L.shape, L.n_len, wl.rho, L.K[layer], L.V[layer], L.Q[layer], params=params,
+                             out=c, workspace=L.cws, stream=sp)
+            for t in range(L.T):
+                dq.copy_(hq[t], non_blocking=True)
+                dk.copy_(hk[t], non_blocking=True)
+                dv.copy_(hv[t], non_blocking=True)
+                for layer in range(wl.layers):
+                    api.decode(L.caches[layer], dq[layer], dk[layer], dv[layer], out=L.out[0, layer],
+                               workspace=L.dws, stream=sp)
+                hout.copy_(L.out[0], non_blocking=True)
+            stream.synchronize()
+
+    one()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    dt = (time.perf_counter() - t0) / steps
+    return {"value": wl.batch * L.T / dt, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps}
+
+
+def kernel_revision() -> str:
+    """Content hash of the CUDA sources: profiler figures are valid only for this revision."""
+    import hashlib
+    h = hashlib.sha256()
+    cs = os.path.join(ROOT, "paper_2607_16213_gb300", "csrc")
+    for f in sorted(os.listdir(cs)):
+        with open(os.path.join(cs, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1 and rank != 0:
+        return
+    wl = synth.WORKLOADS[args.workload]
+    if args.decode_steps is not None:
+        wl = wl.with_(decode_steps=args.decode_steps)
+    vals = []
+    for _ in range(args.warmup):
+        oracle_sample(wl, layers=1, decode_tokens=1)
+    info = None
+    for _ in range(args.steps):
+        info = oracle_sample(wl, layers=1, decode_tokens=1)
+        vals.append(info["value"])
+    v = statistics.median(vals)
+    tokens = wl.batch * wl.decode_steps
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": tokens / v * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
+                       "rho": wl.rho, "decode_steps": wl.decode_steps},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
+                             "sample": info["sample"]},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="selkv", choices=["selkv", "reference"])
+    ap.add_argument("--workload", default="long_100k", choices=list(synth.WORKLOADS))
+    ap.add_argument("--decode-steps", type=int, default=None)
+    ap.add_argument("--layers", type=int, default=None, help=argparse.SUPPRESS)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-full", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,193 @@
+/*
+ * selkv.h - C ABI of the SelKV GB300 library (sm_103a).
+ *
+ * SelKV compresses a prefilled KV cache once (score -> select -> route -> gate -> merge ->
+ * attention ratio) and then decodes over the compressed cache with the attention-ratio
+ * compensation added to the logits (arxiv 2607.16213, Algorithm 1).  Two calls carry the
+ * whole path:
+ *
+ *   selkv_compress(K, V, Q_obs, budget, params) -> (K_c, V_c, bias, lengths)
+ *   selkv_decode_attn(q, K_c, V_c, bias, lengths) -> out
+ *
+ * Conventions shared by every entry point
+ *   - All tensors are caller-owned DEVICE memory, dense, row-major, in the layouts given
+ *     below; every base pointer is 16-byte aligned.  The library never allocates: scratch
+ *     space is a caller-provided workspace whose size comes from the *_workspace_size call.
+ *   - Work is enqueued asynchronously on `stream`; no call synchronises the stream except
+ *     selkv_workspace_error.  Host-side argument checks happen before any launch: a call
+ *     that returns anything but SELKV_OK has enqueued nothing (SELKV_ERR_CUDA excepted: a
+ *     launch failed).
+ *   - Conditions only the device can see (a length beyond capacity, a timed-out wait) set
+ *     bits in the workspace's error word (SELKV_DEVERR_*); the kernels never trap.  Read and
+ *     clear them with selkv_workspace_error.
+ *   - A workspace must be zeroed once before its first use (selkv_workspace_init).  Calls
+ *     that share a workspace must not overlap on the GPU.
+ *   - Element types: dtype SELKV_BF16 (storage bf16, fp32 arithmetic) or SELKV_FP32.
+ *   - Shapes: B sequences, Hq query heads, Hkv KV heads (Hkv divides Hq, G = Hq / Hkv; query
+ *     head h reads KV head h / G), head dimension d in {64, 128}, observation window W.
+ */
+#ifndef SELKV_H
+#define SELKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SELKV_API __attribute__((visibility("default")))
+#else
+#define SELKV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream (the same handle as cudaStream_t); NULL is the legacy default stream. */
+typedef struct CUstream_st* selkv_stream_t;
+
+typedef enum selkv_status {
+  SELKV_OK = 0,
+  SELKV_ERR_INVALID_ARG = 1, /* a pointer, size, shape or budget violates the contract */
+  SELKV_ERR_UNSUPPORTED = 2, /* a valid request this build does not implement          */
+  SELKV_ERR_WORKSPACE = 3,   /* workspace NULL, misaligned or smaller than required    */
+  SELKV_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed                   */
+  SELKV_ERR_DEVICE = 5       /* selkv_workspace_error found device error bits          */
+} selkv_status;
+
+typedef enum selkv_dtype { SELKV_BF16 = 0, SELKV_FP32 = 1 } selkv_dtype;
+
+/* Eq. 4 gate: COSINE is the method (g = clamp(cos(v_j, v_pi(j)), 0, 1)); OPEN (g = 1) and
+ * CLOSED (g = 0) are the paper's ablation end points "merge all" and "eviction only". */
+typedef enum selkv_gate_mode {
+  SELKV_GATE_COSINE = 0,
+  SELKV_GATE_OPEN = 1,
+  SELKV_GATE_CLOSED = 2
+} selkv_gate_mode;
+
+/* Evicted tokens whose bucket holds no kept token (Eq. 3 leaves this open): EXPAND looks at
+ * buckets b-r and b+r for r = 1, 2, ... and takes the first ring with a kept token; DROP
+ * gives them g = 0 and no target. */
+typedef enum selkv_empty_bucket { SELKV_EMPTY_EXPAND = 0, SELKV_EMPTY_DROP = 1 } selkv_empty_bucket;
+
+/* Device error bits (selkv_workspace_error). */
+#define SELKV_DEVERR_CAPACITY 0x1u /* decode append would pass m_cap: not appended       */
+#define SELKV_DEVERR_TIMEOUT 0x2u  /* a bounded wait gave up; the launch's output is void  */
+#define SELKV_DEVERR_LENGTH 0x4u   /* lengths[b] outside [0, m_cap]; clamped              */
+#define SELKV_DEVERR_COUNT 0x8u    /* compress kept a count other than m_b (internal)     */
+
+typedef struct selkv_shape {
+  int32_t dtype;        /* selkv_dtype of K, V, Q_obs, q, k_new, v_new, K_c, V_c and out  */
+  int32_t batch;        /* B, 1 .. SELKV_MAX_BATCH                                       */
+  int32_t num_q_heads;  /* Hq                                                            */
+  int32_t num_kv_heads; /* Hkv, divides Hq, at most 32                                   */
+  int32_t head_dim;     /* d: 64 or 128                                                  */
+  int32_t obs_window;   /* W: observation-window rows per query head (Sec. 3.1)          */
+  int32_t n_cap;        /* rows per (b, kv) of K and V                                   */
+  int32_t m_cap;        /* rows per (b, kv) of K_c, V_c and bias                         */
+} selkv_shape;
+
+#define SELKV_MAX_BATCH 1024
+
+/* Hyperparameters (Sec. 3, defaults of Sec. 4.1 / App. F in the comments). */
+typedef struct selkv_params {
+  float alpha;          /* compensation strength, 0.5 (Sec. 3.6); 0 disables the bias  */
+  int32_t pool_kernel;  /* average-pooling kernel K, odd, 5 (Sec. 3.2)                  */
+  int32_t bucket;       /* routing bucket size B, 1 .. 32, 32 (Sec. 3.4)                */
+  int32_t recent;       /* recent window m_r always kept, 16 (Sec. 3.1)                 */
+  int32_t gate_mode;    /* selkv_gate_mode                                              */
+  int32_t empty_bucket; /* selkv_empty_bucket                                           */
+} selkv_params;
+
+/* Optional device outputs of selkv_compress, for inspection and testing.  Any field may be
+ * NULL.  Entries for positions >= n_b (or slots >= m_b) are left untouched. */
+typedef struct selkv_compress_debug {
+  float* attn;       /* [B][Hkv][n_cap] a: cumulative window attention, group mean     */
+  float* score;      /* [B][Hkv][n_cap] pooled contribution score; 0 past candidates   */
+  uint8_t* topk;     /* [B][Hkv][n_cap] 1 where KV head kv's own top-m_s chose j       */
+  int32_t* kept_idx; /* [B][m_cap] kept positions, ascending                           */
+  int32_t* target;   /* [B][Hkv][n_cap] merge target of evicted j; -1 for kept j and
+                        for tokens left without a target                              */
+  float* gate;       /* [B][Hkv][n_cap] g of evicted j (0 for kept j)                  */
+  uint8_t* decision; /* [B][Hkv][n_cap] 1 = merge (g > 0), 0 = drop; 2 for kept j      */
+  float* ratio;      /* [B][Hkv][m_cap] attention ratio R per kept slot (Eq. 6)        */
+} selkv_compress_debug;
+
+/* Human-readable name of a status code (static storage). */
+SELKV_API const char* selkv_status_string(selkv_status status);
+
+/* Number of kernels this library has enqueued since it was loaded, over all threads and
+ * devices (a diagnostic counter; a captured CUDA graph counts its kernels once, at capture). */
+SELKV_API uint64_t selkv_kernel_launches(void);
+
+/* Zero a workspace (its error word and the decode counters).  Enqueued on `stream`.
+ * Returns SELKV_ERR_WORKSPACE for a NULL or misaligned workspace. */
+SELKV_API selkv_status selkv_workspace_init(void* workspace, size_t workspace_bytes, selkv_stream_t stream);
+
+/* Synchronise `stream`, copy the workspace's device error bits to *flags and clear them.
+ * Returns SELKV_OK when no bit was set, SELKV_ERR_DEVICE when some were. */
+SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t stream, uint32_t* flags);
+
+/* ---------------------------------------------------------------------------------------
+ * Compression (Algorithm 1, steps 1-6; step 7, RoPE repositioning, off as in Sec. 4.1).
+ *
+ * For every sequence b (prefill length n_b = n_len[b]) and every KV head:
+ *   a  = mean over the G query heads of the column sums of the causal observation-window
+ *        attention softmax(Q_obs K^T / sqrt(d)), row i at position n_b - W + i (Sec. 3.1);
+ *   c  = a * ||v|| (Eq. 1), average-pooled over the candidates [0, n_b - m_r) (Sec. 3.2);
+ *   per-KV-head top-m_s of c (Eq. 2), union over KV heads, trimmed to m_s by the mean score
+ *   (Sec. 3.3), plus the recent window: m_b = floor(rho * n_b) kept positions shared by
+ *   every head, ties to the lower position;
+ *   each evicted j routes to the kept token of its bucket with the largest a (Eq. 3, Sec. 3.4), gets
+ *   g = clamp(cos(v_j, v_pi(j)), 0, 1) (Eq. 4) and is merged into V_c with weight g*a_j
+ *   (Eq. 5); R = (a_i + sum g a_j) / a_i (Eq. 6); bias = alpha * ln(mean over KV heads R)
+ *   (Sec. 3.6, GQA); K_c holds the kept keys unchanged.
+ *
+ * n_len     HOST array [B]: prefill lengths, W <= n_b <= n_cap.
+ * rho       retention ratio in (0, 1]; m_b = floor(rho * n_b) (double), and
+ *           m_b - recent >= 0 and m_b <= m_cap must hold for every b.
+ * K, V      [B][Hkv][n_cap][d]; rows >= n_b are ignored.
+ * Q_obs     [B][Hq][W][d]: the last W query rows of each sequence.
+ * K_c, V_c  [B][Hkv][m_cap][d] outputs; rows >= m_b untouched.
+ * bias      [B][Hkv][m_cap] fp32 output (the same row for every KV head).
+ * lengths   [B] int32 device output: m_b.
+ * Errors: SELKV_ERR_INVALID_ARG for a NULL tensor, a bad shape, a misaligned pointer or a
+ * budget outside the rules above; SELKV_ERR_UNSUPPORTED for d not in {64, 128} or a bucket
+ * above 32; SELKV_ERR_WORKSPACE when workspace_bytes < selkv_compress_workspace_size.
+ * ------------------------------------------------------------------------------------- */
+SELKV_API size_t selkv_compress_workspace_size(const selkv_shape* shape);
+
+SELKV_API selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, double rho,
+                            const selkv_params* params, const void* K, const void* V,
+                            const void* Q_obs, void* K_c, void* V_c, float* bias,
+                            int32_t* lengths, const selkv_compress_debug* debug,
+                            void* workspace, size_t workspace_bytes, selkv_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------
+ * Compensated decode attention (Algorithm 1, "Decode with compressed cache + alpha log R";
+ * Sec. 3.6).  For every sequence b and query head h (KV head kv = h / G):
+ *   out[b][h] = sum_{i < L} softmax_i(q[b][h] . K_c[b][kv][i] / sqrt(d) + bias[b][kv][i])
+ *               * V_c[b][kv][i]
+ * over L = lengths[b] rows, plus, when k_new and v_new are given, the new row
+ * (k_new[b][kv], v_new[b][kv]) with bias 0 (R = 1).  The new row is then written at row
+ * lengths[b] of K_c / V_c (bias 0), and lengths[b] is incremented, all inside the call.
+ *
+ * q, out        [B][Hq][d].
+ * K_c, V_c      [B][Hkv][m_cap][d]; bias [B][Hkv][m_cap] fp32 or NULL (no compensation:
+ *               plain attention, e.g. over an uncompressed cache with m_cap = n_cap).
+ * lengths       [B] int32 device, read (and incremented when appending).
+ * k_new, v_new  [B][Hkv][d] or both NULL.
+ * An empty cache with no new row gives out = 0.  An append that would pass m_cap is skipped
+ * and sets SELKV_DEVERR_CAPACITY.
+ * ------------------------------------------------------------------------------------- */
+SELKV_API size_t selkv_decode_workspace_size(const selkv_shape* shape);
+
+SELKV_API selkv_status selkv_decode_attn(const selkv_shape* shape, const void* q, void* K_c, void* V_c,
+                               float* bias, int32_t* lengths, const void* k_new,
+                               const void* v_new, void* out, void* workspace,
+                               size_t workspace_bytes, selkv_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SELKV_H */

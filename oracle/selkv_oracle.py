@@ -10,9 +10,9 @@ Merge-or-Drop and Attention Compensation"):
   observation re-pass (Sec. 3.1) -> contribution score (Eq. 1) -> average pooling (Sec. 3.2)
   -> budget m = floor(rho n), recent window m_r (Sec. 3.1) -> per-KV-head top-m_s, union over
   KV heads, trim by mean score (Eq. 2, Sec. 3.3 "Union selection") -> bucket-attention routing
-  (Eq. 3) -> soft cosine gate (Eq. 4) -> gated attention-weighted merge (Eq. 5) -> attention
-  ratio (Eq. 6) -> GQA bias alpha*log(mean_kv R) (Sec. 3.5) -> decode with the bias (Alg. 1,
-  last step).  RoPE repositioning (Eq. 7) is off, as in the paper's configuration (Sec. 4.1).
+  (Eq. 3, Sec. 3.4) -> soft cosine gate (Eq. 4, Sec. 3.5) -> gated attention-weighted merge (Eq. 5) -> attention
+  ratio (Eq. 6) -> GQA bias alpha*log(mean_kv R) (Sec. 3.6) -> decode with the bias (Alg. 1,
+  last step).  RoPE repositioning (Eq. 7) is off, as in the paper's configuration (Sec. 4.1; Eq. 7 is Sec. 3.7).
 
 Readings where the paper is silent or garbled (each is a named choice, mirrored by the CUDA
 path):
@@ -314,7 +314,7 @@ def merge(a_kv: np.ndarray, V_kv: np.ndarray, kept_idx: np.ndarray, target: np.n
 
 
 def gqa_bias(R: np.ndarray, alpha: float) -> np.ndarray:
-    """Sec. 3.5 for GQA: bias_i = alpha * ln(mean over KV heads of R_{kv,i}) (R16).
+    """Sec. 3.6 for GQA: bias_i = alpha * ln(mean over KV heads of R_{kv,i}) (R16).
     R: [Hkv][m]."""
     return alpha * np.log(R.mean(axis=0))
 
@@ -385,7 +385,7 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
 
 
 # ----------------------------------------------------------------------------------------
-# Decode with the compensated cache (Alg. 1, last step; Sec. 3.5)
+# Decode with the compensated cache (Alg. 1, last step; Sec. 3.6)
 # ----------------------------------------------------------------------------------------
 def decode(q: np.ndarray, K_c: np.ndarray, V_c: np.ndarray, bias: Optional[np.ndarray],
            length: int) -> np.ndarray:

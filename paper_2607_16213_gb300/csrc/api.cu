@@ -1,0 +1,290 @@
+// C-ABI entry points of the SelKV library: argument validation, workspace planning and
+// kernel launches.  Host code only; every step of the method runs in the kernels.
+#include <atomic>
+#include <cmath>
+#include <cstring>
+
+#include "selkv_internal.cuh"
+
+namespace selkv {
+cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
+cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
+cudaError_t launch_norm_pool(const CompressArgs& a, cudaStream_t s);
+cudaError_t launch_select(const CompressArgs& a, float* tkey, uint8_t* uflag, cudaStream_t s);
+cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s);
+
+namespace {
+
+// Kernels enqueued by each call (diagnostic count, see selkv_kernel_launches).
+std::atomic<uint64_t> g_launches{0};
+constexpr int kCompressKernels = 9;
+constexpr int kDecodeKernels = 1;
+// SM count used for planning the decode split: fixed, so that workspace sizes do not depend
+// on which device answers (GB300: 152 SMs).
+constexpr int kPlanSMs = 152;
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool shape_ok(const selkv_shape* s) {
+  if (s == nullptr) return false;
+  if (s->dtype != SELKV_BF16 && s->dtype != SELKV_FP32) return false;
+  if (s->batch < 1 || s->batch > SELKV_MAX_BATCH) return false;
+  if (s->num_kv_heads < 1 || s->num_kv_heads > 32 || s->num_q_heads < 1) return false;
+  if (s->num_q_heads % s->num_kv_heads != 0) return false;
+  if (s->num_q_heads / s->num_kv_heads > 16) return false;
+  if (s->head_dim < 1 || s->n_cap < 0 || s->m_cap < 0 || s->obs_window < 0) return false;
+  return true;
+}
+
+size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct CompressPlan {
+  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, thr, kflag, slot, tkey, uflag, total;
+  int nchunks, R;
+};
+
+CompressPlan plan_compress(const selkv_shape& s) {
+  CompressPlan p{};
+  size_t off = sizeof(WsHeader);
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += round256(bytes);
+    return o;
+  };
+  const size_t B = s.batch, Hkv = s.num_kv_heads, n = s.n_cap;
+  p.R = (s.num_q_heads / s.num_kv_heads) * s.obs_window;
+  p.nchunks = (int)((n + kRowChunk - 1) / kRowChunk);
+  p.seq_n = take(B * 4);
+  p.seq_m = take(B * 4);
+  p.rowpart = take(B * Hkv * (size_t)p.nchunks * p.R * sizeof(float2));
+  p.rowstat = take(B * Hkv * (size_t)p.R * sizeof(float2));
+  p.attn = take(B * Hkv * n * 4);
+  p.vnorm = take(B * Hkv * n * 4);
+  p.score = take(B * Hkv * n * 4);
+  p.thr = take(B * Hkv * sizeof(uint2));
+  p.kflag = take(B * n);
+  p.slot = take(B * n * 4);
+  p.tkey = take(B * n * 4);
+  p.uflag = take(B * n);
+  p.total = off;
+  return p;
+}
+
+struct DecodePlan {
+  size_t cnt_head, cnt_seq, partial, total;
+  int splits;
+};
+
+DecodePlan plan_decode(const selkv_shape& s) {
+  DecodePlan p{};
+  size_t off = sizeof(WsHeader);
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += round256(bytes);
+    return o;
+  };
+  p.splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs);
+  p.cnt_head = take((size_t)s.batch * s.num_kv_heads * 4);
+  p.cnt_seq = take((size_t)s.batch * 4);
+  p.partial = take((size_t)s.batch * s.num_q_heads * p.splits * (s.head_dim + 2) * 4);
+  p.total = off;
+  return p;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+}  // namespace
+}  // namespace selkv
+
+using namespace selkv;
+
+extern "C" {
+
+const char* selkv_status_string(selkv_status status) {
+  switch (status) {
+    case SELKV_OK: return "ok";
+    case SELKV_ERR_INVALID_ARG: return "invalid argument";
+    case SELKV_ERR_UNSUPPORTED: return "unsupported configuration";
+    case SELKV_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case SELKV_ERR_CUDA: return "CUDA error";
+    case SELKV_ERR_DEVICE: return "device reported an error";
+  }
+  return "unknown status";
+}
+
+uint64_t selkv_kernel_launches(void) { return g_launches.load(); }
+
+selkv_status selkv_workspace_init(void* workspace, size_t workspace_bytes, selkv_stream_t stream) {
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < sizeof(WsHeader))
+    return SELKV_ERR_WORKSPACE;
+  if (cudaMemsetAsync(workspace, 0, workspace_bytes, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return SELKV_ERR_CUDA;
+  return SELKV_OK;
+}
+
+selkv_status selkv_workspace_error(void* workspace, selkv_stream_t stream, uint32_t* flags) {
+  if (workspace == nullptr || flags == nullptr) return SELKV_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t f = 0;
+  if (cudaMemcpyAsync(&f, workspace, sizeof(f), cudaMemcpyDeviceToHost, st) != cudaSuccess) return SELKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return SELKV_ERR_CUDA;
+  *flags = f;
+  if (f != 0) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), st) != cudaSuccess) return SELKV_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return SELKV_ERR_CUDA;
+    return SELKV_ERR_DEVICE;
+  }
+  return SELKV_OK;
+}
+
+size_t selkv_compress_workspace_size(const selkv_shape* shape) {
+  if (!shape_ok(shape)) return 0;
+  return plan_compress(*shape).total;
+}
+
+selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, double rho,
+                            const selkv_params* params, const void* K, const void* V,
+                            const void* Q_obs, void* K_c, void* V_c, float* bias,
+                            int32_t* lengths, const selkv_compress_debug* debug,
+                            void* workspace, size_t workspace_bytes, selkv_stream_t stream) {
+  if (!shape_ok(shape) || params == nullptr || n_len == nullptr) return SELKV_ERR_INVALID_ARG;
+  const selkv_shape& s = *shape;
+  if (s.head_dim != 64 && s.head_dim != 128) return SELKV_ERR_UNSUPPORTED;
+  if (s.obs_window < 1 || s.n_cap < 1) return SELKV_ERR_INVALID_ARG;
+  const selkv_params& p = *params;
+  if (!std::isfinite(p.alpha) || p.pool_kernel < 1 || (p.pool_kernel & 1) == 0 || p.recent < 0 ||
+      p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1)
+    return SELKV_ERR_INVALID_ARG;
+  if (p.bucket > 32) return SELKV_ERR_UNSUPPORTED;
+  if (!(rho > 0.0 && rho <= 1.0)) return SELKV_ERR_INVALID_ARG;
+  const void* tensors[] = {K, V, Q_obs, K_c, V_c, bias, lengths};
+  for (const void* t : tensors)
+    if (t == nullptr || !aligned(t, 16)) return SELKV_ERR_INVALID_ARG;
+  if (debug != nullptr) {
+    const void* dbg[] = {debug->attn, debug->score, debug->topk, debug->kept_idx,
+                         debug->target, debug->gate, debug->decision, debug->ratio};
+    for (const void* t : dbg)
+      if (t != nullptr && !aligned(t, 16)) return SELKV_ERR_INVALID_ARG;
+  }
+  static thread_local SeqTable tab;
+  for (int b = 0; b < s.batch; ++b) {
+    const int n = n_len[b];
+    if (n < s.obs_window || n > s.n_cap) return SELKV_ERR_INVALID_ARG;
+    const double mm = std::floor(rho * (double)n);
+    const int m = (int)mm;
+    if (m - p.recent < 0 || m > s.m_cap || m > n) return SELKV_ERR_INVALID_ARG;
+    tab.n[b] = n;
+    tab.m[b] = m;
+  }
+  const CompressPlan plan = plan_compress(s);
+  if (workspace == nullptr || !aligned(workspace, 256)) return SELKV_ERR_WORKSPACE;
+  if (workspace_bytes < plan.total) return SELKV_ERR_WORKSPACE;
+
+  CompressArgs a{};
+  a.dtype = s.dtype;
+  a.B = s.batch;
+  a.Hq = s.num_q_heads;
+  a.Hkv = s.num_kv_heads;
+  a.G = s.num_q_heads / s.num_kv_heads;
+  a.D = s.head_dim;
+  a.W = s.obs_window;
+  a.n_cap = s.n_cap;
+  a.m_cap = s.m_cap;
+  a.R = plan.R;
+  a.nchunks = plan.nchunks;
+  a.alpha = p.alpha;
+  a.pool_kernel = p.pool_kernel;
+  a.bucket = p.bucket;
+  a.recent = p.recent;
+  a.gate_mode = p.gate_mode;
+  a.empty_bucket = p.empty_bucket;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
+  a.K = K;
+  a.V = V;
+  a.Q = Q_obs;
+  a.Kc = K_c;
+  a.Vc = V_c;
+  a.bias = bias;
+  a.lengths = lengths;
+  a.flags = at<uint32_t>(workspace, 0);
+  a.seq_n = at<int32_t>(workspace, plan.seq_n);
+  a.seq_m = at<int32_t>(workspace, plan.seq_m);
+  a.rowpart = at<float2>(workspace, plan.rowpart);
+  a.rowstat = at<float2>(workspace, plan.rowstat);
+  a.attn = (debug && debug->attn) ? debug->attn : at<float>(workspace, plan.attn);
+  a.vnorm = at<float>(workspace, plan.vnorm);
+  a.score = (debug && debug->score) ? debug->score : at<float>(workspace, plan.score);
+  a.thr = at<uint2>(workspace, plan.thr);
+  a.kflag = at<uint8_t>(workspace, plan.kflag);
+  a.slot_of = at<int32_t>(workspace, plan.slot);
+  if (debug != nullptr) {
+    a.dbg_topk = debug->topk;
+    a.dbg_kept_idx = debug->kept_idx;
+    a.dbg_target = debug->target;
+    a.dbg_gate = debug->gate;
+    a.dbg_decision = debug->decision;
+    a.dbg_ratio = debug->ratio;
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_setup(a, tab, st);
+  if (e == cudaSuccess) e = launch_score_simt(a, st);
+  if (e == cudaSuccess) e = launch_norm_pool(a, st);
+  if (e == cudaSuccess) e = launch_select(a, at<float>(workspace, plan.tkey), at<uint8_t>(workspace, plan.uflag), st);
+  if (e == cudaSuccess) e = launch_merge(a, st);
+  g_launches += kCompressKernels;
+  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+}
+
+size_t selkv_decode_workspace_size(const selkv_shape* shape) {
+  if (!shape_ok(shape)) return 0;
+  return plan_decode(*shape).total;
+}
+
+selkv_status selkv_decode_attn(const selkv_shape* shape, const void* q, void* K_c, void* V_c,
+                               float* bias, int32_t* lengths, const void* k_new,
+                               const void* v_new, void* out, void* workspace,
+                               size_t workspace_bytes, selkv_stream_t stream) {
+  if (!shape_ok(shape)) return SELKV_ERR_INVALID_ARG;
+  const selkv_shape& s = *shape;
+  if (s.head_dim != 64 && s.head_dim != 128) return SELKV_ERR_UNSUPPORTED;
+  if (s.m_cap < 1) return SELKV_ERR_INVALID_ARG;
+  const void* tensors[] = {q, K_c, V_c, lengths, out};
+  for (const void* t : tensors)
+    if (t == nullptr || !aligned(t, 16)) return SELKV_ERR_INVALID_ARG;
+  if ((k_new == nullptr) != (v_new == nullptr)) return SELKV_ERR_INVALID_ARG;
+  if (k_new != nullptr && (!aligned(k_new, 16) || !aligned(v_new, 16))) return SELKV_ERR_INVALID_ARG;
+  if (bias != nullptr && !aligned(bias, 16)) return SELKV_ERR_INVALID_ARG;
+  const DecodePlan plan = plan_decode(s);
+  if (workspace == nullptr || !aligned(workspace, 256)) return SELKV_ERR_WORKSPACE;
+  if (workspace_bytes < plan.total) return SELKV_ERR_WORKSPACE;
+  DecodeArgs a{};
+  a.dtype = s.dtype;
+  a.B = s.batch;
+  a.Hq = s.num_q_heads;
+  a.Hkv = s.num_kv_heads;
+  a.G = s.num_q_heads / s.num_kv_heads;
+  a.D = s.head_dim;
+  a.m_cap = s.m_cap;
+  a.splits = plan.splits;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
+  a.q = q;
+  a.Kc = K_c;
+  a.Vc = V_c;
+  a.bias = bias;
+  a.lengths = lengths;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.out = out;
+  a.flags = at<uint32_t>(workspace, 0);
+  a.cnt_head = at<uint32_t>(workspace, plan.cnt_head);
+  a.cnt_seq = at<uint32_t>(workspace, plan.cnt_seq);
+  a.partial = at<float>(workspace, plan.partial);
+  const cudaError_t e = launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
+  g_launches += kDecodeKernels;
+  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+}
+
+}  // extern "C"

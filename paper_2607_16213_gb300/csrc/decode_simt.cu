@@ -1,0 +1,224 @@
+// Compensated decode attention on CUDA cores (fp32 arithmetic; both storage dtypes).
+//
+//   out[b][h] = sum_i softmax_i(q_h . k_i / sqrt(d) + bias_i) v_i      (Alg. 1 decode,
+//                                                                     Sec. 3.6 compensation)
+// Split-K flash decoding: CTA (split s, KV head kv, sequence b) streams a contiguous slice of
+// the compressed rows once for all G query heads of the group, keeping a running max / sum
+// per head in the base-2 domain (the bias is folded into the logit before the max).  Each CTA
+// leaves (max, sum, unnormalised output) in the workspace; the last CTA of a (b, kv) to
+// arrive (one atomic add, no waiting) folds the splits in split order, so the result does
+// not depend on scheduling.  With k_new / v_new the new row joins the softmax with bias 0 and
+// is then written at row lengths[b]; the last (b, kv) of a sequence bumps lengths[b].
+#include <algorithm>
+
+#include "selkv_internal.cuh"
+
+namespace selkv {
+namespace {
+
+constexpr int kWarps = 4;
+
+template <typename T, int D, int GM>
+__global__ __launch_bounds__(kWarps * 32) void decode_simt_kernel(DecodeArgs a) {
+  constexpr int PER = D / 32;
+  __shared__ __align__(16) float qs[GM][D];
+  __shared__ float wm[kWarps][GM], wl[kWarps][GM];
+  __shared__ float wo[kWarps][GM][D];
+  __shared__ bool s_last;
+  const int s = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int G = a.G, S = a.splits;
+  const size_t bk = (size_t)b * a.Hkv + kv;
+
+  int L = a.lengths[b];
+  if (L < 0 || L > a.m_cap) {
+    if (tid == 0 && s == 0 && kv == 0) raise_flag(a.flags, SELKV_DEVERR_LENGTH);
+    L = L < 0 ? 0 : a.m_cap;
+  }
+  bool app = a.k_new != nullptr;
+  if (app && L + 1 > a.m_cap) {
+    if (tid == 0 && s == 0 && kv == 0) raise_flag(a.flags, SELKV_DEVERR_CAPACITY);
+    app = false;
+  }
+  const int total = L + (app ? 1 : 0);
+  const int chunk = ((total + S - 1) / S + 31) / 32 * 32;
+  const int lo = s * chunk, hi = min(total, lo + chunk);
+
+  for (int i = tid; i < G * D; i += blockDim.x) {
+    const int g = i / D, d = i % D;
+    qs[g][d] = load1(static_cast<const T*>(a.q) + ((size_t)b * a.Hq + kv * G + g) * D + d) * a.scale_log2;
+  }
+  __syncthreads();
+
+  const T* Kb = static_cast<const T*>(a.Kc) + bk * a.m_cap * D;
+  const T* Vb = static_cast<const T*>(a.Vc) + bk * a.m_cap * D;
+  const T* kn = app ? static_cast<const T*>(a.k_new) + bk * D : nullptr;
+  const T* vnw = app ? static_cast<const T*>(a.v_new) + bk * D : nullptr;
+  const float* bias = a.bias != nullptr ? a.bias + bk * a.m_cap : nullptr;
+
+  float m[GM], l[GM], o[GM][PER], pg[GM];
+#pragma unroll
+  for (int g = 0; g < GM; ++g) {
+    m[g] = -INFINITY;
+    l[g] = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) o[g][e] = 0.f;
+  }
+  for (int t0 = lo + warp * 32; t0 < hi; t0 += kWarps * 32) {
+    const int key = t0 + lane;
+    const bool valid = key < hi;
+    float sc[GM];
+#pragma unroll
+    for (int g = 0; g < GM; ++g) sc[g] = 0.f;
+    if (valid) {
+      const T* kr = key < L ? Kb + (size_t)key * D : kn;
+#pragma unroll 4
+      for (int d = 0; d < D; d += 8) {
+        float x[8];
+        load8(kr + d, x);
+#pragma unroll
+        for (int g = 0; g < GM; ++g) {
+          if (g < G) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) sc[g] = fmaf(qs[g][d + e], x[e], sc[g]);
+          }
+        }
+      }
+    }
+    const float bv = (valid && key < L && bias != nullptr) ? bias[key] * kLog2e : 0.f;
+#pragma unroll
+    for (int g = 0; g < GM; ++g) {
+      if (g >= G) break;
+      const float v = valid ? sc[g] + bv : -INFINITY;
+      const float mn = fmaxf(m[g], warp_max(v));
+      const float corr = exp2f(m[g] - mn);
+      const float p = exp2f(v - mn);
+      l[g] = l[g] * corr + warp_sum(p);
+#pragma unroll
+      for (int e = 0; e < PER; ++e) o[g][e] *= corr;
+      m[g] = mn;
+      pg[g] = p;
+    }
+    const int nk = min(32, hi - t0);
+    for (int k = 0; k < nk; ++k) {
+      const int key2 = t0 + k;
+      const T* vr = key2 < L ? Vb + (size_t)key2 * D : vnw;
+      float v[PER];
+      if constexpr (PER == 4) load4(vr + lane * 4, v); else load2(vr + lane * 2, v);
+#pragma unroll
+      for (int g = 0; g < GM; ++g) {
+        if (g >= G) break;
+        const float pk = __shfl_sync(0xffffffffu, pg[g], k);
+#pragma unroll
+        for (int e = 0; e < PER; ++e) o[g][e] = fmaf(pk, v[e], o[g][e]);
+      }
+    }
+  }
+  // fold the warps
+#pragma unroll
+  for (int g = 0; g < GM; ++g) {
+    if (g >= G) break;
+    if (lane == 0) {
+      wm[warp][g] = m[g];
+      wl[warp][g] = l[g];
+    }
+#pragma unroll
+    for (int e = 0; e < PER; ++e) wo[warp][g][lane * PER + e] = o[g][e];
+  }
+  __syncthreads();
+  float* part = a.partial;
+  for (int i = tid; i < G * D; i += blockDim.x) {
+    const int g = i / D, d = i % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, wm[w][g]);
+    float sl = 0.f, so = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        const float f = exp2f(wm[w][g] - M);
+        sl += wl[w][g] * f;
+        so += wo[w][g][d] * f;
+      }
+    }
+    float* pp = part + (((size_t)b * a.Hq + kv * G + g) * S + s) * (D + 2);
+    pp[d] = so;
+    if (d == 0) {
+      pp[D] = M;
+      pp[D + 1] = sl;
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) {
+    const uint32_t prev = atomicAdd(&a.cnt_head[bk], 1u);
+    s_last = (prev == (uint32_t)S - 1u);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int i = tid; i < G * D; i += blockDim.x) {
+    const int g = i / D, d = i % D;
+    const float* pp = part + ((size_t)b * a.Hq + kv * G + g) * S * (D + 2);
+    float M = -INFINITY;
+    for (int t = 0; t < S; ++t) M = fmaxf(M, __ldcg(pp + (size_t)t * (D + 2) + D));
+    float sl = 0.f, so = 0.f;
+    if (M != -INFINITY) {
+      for (int t = 0; t < S; ++t) {
+        const float* q = pp + (size_t)t * (D + 2);
+        const float f = exp2f(__ldcg(q + D) - M);
+        sl += __ldcg(q + D + 1) * f;
+        so += __ldcg(q + d) * f;
+      }
+    }
+    store1(static_cast<T*>(a.out) + ((size_t)b * a.Hq + kv * G + g) * D + d, sl > 0.f ? so / sl : 0.f);
+  }
+  if (app) {
+    T* Kw = static_cast<T*>(a.Kc) + (bk * a.m_cap + L) * D;
+    T* Vw = static_cast<T*>(a.Vc) + (bk * a.m_cap + L) * D;
+    for (int d = tid; d < D; d += blockDim.x) {
+      Kw[d] = kn[d];
+      Vw[d] = vnw[d];
+    }
+    if (a.bias != nullptr && tid == 0) a.bias[bk * a.m_cap + L] = 0.f;
+  }
+  if (tid == 0) {
+    a.cnt_head[bk] = 0u;
+    if (app) {
+      __threadfence();
+      const uint32_t prev = atomicAdd(&a.cnt_seq[b], 1u);
+      if (prev == (uint32_t)a.Hkv - 1u) {
+        a.lengths[b] = L + 1;
+        a.cnt_seq[b] = 0u;
+      }
+    }
+  }
+}
+
+template <typename T, int D>
+cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
+  const dim3 grid(a.splits, a.Hkv, a.B);
+  const int th = kWarps * 32;
+  if (a.G <= 1) decode_simt_kernel<T, D, 1><<<grid, th, 0, st>>>(a);
+  else if (a.G <= 2) decode_simt_kernel<T, D, 2><<<grid, th, 0, st>>>(a);
+  else if (a.G <= 4) decode_simt_kernel<T, D, 4><<<grid, th, 0, st>>>(a);
+  else if (a.G <= 8) decode_simt_kernel<T, D, 8><<<grid, th, 0, st>>>(a);
+  else decode_simt_kernel<T, D, 16><<<grid, th, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
+  const int units = B * Hkv;
+  int S = (2 * num_sms + units - 1) / units;
+  S = std::min(S, std::max(1, (m_cap + 63) / 64));
+  return std::max(1, std::min(S, 64));
+}
+
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
+  if (a.dtype == SELKV_BF16) return a.D == 128 ? launch_t<__nv_bfloat16, 128>(a, st) : launch_t<__nv_bfloat16, 64>(a, st);
+  return a.D == 128 ? launch_t<float, 128>(a, st) : launch_t<float, 64>(a, st);
+}
+
+}  // namespace selkv

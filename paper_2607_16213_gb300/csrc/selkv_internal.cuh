@@ -1,0 +1,153 @@
+// Internal declarations shared by the SelKV kernels and the C-ABI host code.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/selkv.h"
+
+namespace selkv {
+
+// Every workspace starts with this header; the rest is carved by the host planners.
+struct WsHeader {
+  uint32_t flags;  // SELKV_DEVERR_* bits, sticky until selkv_workspace_error
+  uint32_t pad[63];
+};
+static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ void raise_flag(uint32_t* flags, uint32_t bit) { atomicOr(flags, bit); }
+
+// ---- element access: storage dtype -> fp32 ------------------------------------------------
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Load 8 consecutive elements starting at p (16-byte aligned for bf16, 32-byte for fp32).
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&x)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  x[0] = bf16_lo(u.x); x[1] = bf16_hi(u.x);
+  x[2] = bf16_lo(u.y); x[3] = bf16_hi(u.y);
+  x[4] = bf16_lo(u.z); x[5] = bf16_hi(u.z);
+  x[6] = bf16_lo(u.w); x[7] = bf16_hi(u.w);
+}
+__device__ __forceinline__ void load8(const float* p, float (&x)[8]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+  x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+}
+// Load 4 consecutive elements (8-byte aligned for bf16, 16-byte for fp32).
+__device__ __forceinline__ void load4(const __nv_bfloat16* p, float (&x)[4]) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  x[0] = bf16_lo(u.x); x[1] = bf16_hi(u.x);
+  x[2] = bf16_lo(u.y); x[3] = bf16_hi(u.y);
+}
+__device__ __forceinline__ void load4(const float* p, float (&x)[4]) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+}
+__device__ __forceinline__ void load2(const __nv_bfloat16* p, float (&x)[2]) {
+  const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+  x[0] = bf16_lo(u); x[1] = bf16_hi(u);
+}
+__device__ __forceinline__ void load2(const float* p, float (&x)[2]) {
+  const float2 a = *reinterpret_cast<const float2*>(p);
+  x[0] = a.x; x[1] = a.y;
+}
+__device__ __forceinline__ float load1(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ float load1(const float* p) { return *p; }
+
+__device__ __forceinline__ void store1(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+__device__ __forceinline__ void store1(float* p, float v) { *p = v; }
+__device__ __forceinline__ void store4(__nv_bfloat16* p, const float (&x)[4]) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(x[0], x[1]);
+  __nv_bfloat162 b = __floats2bfloat162_rn(x[2], x[3]);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+__device__ __forceinline__ void store4(float* p, const float (&x)[4]) {
+  *reinterpret_cast<float4*>(p) = make_float4(x[0], x[1], x[2], x[3]);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// ---- compress -----------------------------------------------------------------------------
+struct SeqTable {
+  int32_t n[SELKV_MAX_BATCH];  // prefill length n_b
+  int32_t m[SELKV_MAX_BATCH];  // budget m_b = floor(rho * n_b)
+};
+
+struct CompressArgs {
+  int dtype, B, Hq, Hkv, G, D, W, n_cap, m_cap;
+  int R;          // observation rows per KV head: G * W
+  int nchunks;    // column chunks of the row-statistics pass
+  float alpha;
+  int pool_kernel, bucket, recent, gate_mode, empty_bucket;
+  float scale_log2;  // log2(e) / sqrt(d)
+  const void* K;
+  const void* V;
+  const void* Q;
+  void* Kc;
+  void* Vc;
+  float* bias;
+  int32_t* lengths;
+  // debug outputs (nullable)
+  uint8_t* dbg_topk;
+  int32_t* dbg_kept_idx;
+  int32_t* dbg_target;
+  float* dbg_gate;
+  uint8_t* dbg_decision;
+  float* dbg_ratio;
+  // workspace arrays
+  uint32_t* flags;
+  int32_t* seq_n;
+  int32_t* seq_m;
+  float2* rowpart;   // [B][Hkv][nchunks][R] (max, sum) of 2^(s' - max) per column chunk
+  float2* rowstat;   // [B][Hkv][R] (M, 1 / (G * Z))
+  float* attn;       // [B][Hkv][n_cap]
+  float* vnorm;      // [B][Hkv][n_cap]
+  float* score;      // [B][Hkv][n_cap]
+  uint2* thr;        // [B][Hkv] (score bits threshold, last index taken at the threshold)
+  uint8_t* kflag;    // [B][n_cap] 1 = kept
+  int32_t* slot_of;  // [B][n_cap] slot of a kept position, -1 otherwise
+};
+
+constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
+
+cudaError_t launch_compress(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
+
+// ---- decode -------------------------------------------------------------------------------
+struct DecodeArgs {
+  int dtype, B, Hq, Hkv, G, D, m_cap, splits;
+  float scale_log2;  // log2(e) / sqrt(d)
+  const void* q;
+  void* Kc;
+  void* Vc;
+  float* bias;
+  int32_t* lengths;
+  const void* k_new;
+  const void* v_new;
+  void* out;
+  uint32_t* flags;
+  uint32_t* cnt_head;  // [B][Hkv] arrivals per (b, kv) (self-resetting)
+  uint32_t* cnt_seq;   // [B] (b, kv) completions per sequence (self-resetting)
+  float* partial;      // [B][Hq][splits][D + 2]
+};
+
+int decode_splits(int B, int Hkv, int m_cap, int num_sms);
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
+
+}  // namespace selkv

@@ -1,0 +1,204 @@
+"""GPU-vs-oracle comparison helpers for the parity tests.
+
+Discrete decisions (per-KV-head top-k, trim, routing, merge/drop) must agree exactly, except
+where the oracle's own margin at that decision is below the arithmetic noise of the fp32 GPU
+path: there either resolution is correct, the test checks that the GPU's choice is one of the
+near-tied options, and the oracle then continues from the GPU's choice ("follow"), so the
+continuous outputs downstream are still compared element by element.
+
+Margins (derived from the arithmetic):
+  DELTA      relative gap on scores / cumulative attention: the fp32 GPU values carry a
+             relative error of a few 1e-6 (fp32 sums of exponentials whose arguments carry
+             rounding error), so near-ties closer than 1e-4 relative may resolve either way.
+  DELTA_SIM  absolute margin on the cosine around 0 (merge vs drop).
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import synth
+from oracle import selkv_oracle as O
+from paper_2607_16213_gb300 import api
+import paper_2607_16213_gb300 as S
+
+DELTA = 1e-4
+DELTA_SIM = 1e-5
+
+# continuous tolerances
+ATTN_RTOL = 5e-5        # a and pooled scores: relative to the value (plus a tiny floor)
+GATE_ATOL = 2e-6        # g on the same target
+RATIO_RTOL = 2e-5       # R
+BIAS_ATOL = 2e-5        # alpha * ln(mean R)
+VC_FP32_RTOL = 2e-5     # merged values, fp32 storage
+DEC_BF16_MAX, DEC_BF16_MEAN = 2e-2, 2e-3   # decode: bf16 storage, fp32 accumulation
+DEC_FP32_REL = 1e-5     # decode: fp32 storage, relative to max |out|
+
+
+def device():
+    return torch.device("cuda:0")
+
+
+def to_dev(x: np.ndarray, dtype: str) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(x)).to(device())
+    return t.to(torch.bfloat16) if dtype == "bf16" else t
+
+
+def params_of(p: O.Params) -> S.selkv_params:
+    return S.selkv_params(alpha=p.alpha, pool_kernel=p.pool_kernel, bucket=p.bucket,
+                          recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket)
+
+
+def run_compress(wl: synth.Workload, x: dict, p: O.Params, rho=None, extra: int = 0):
+    rho = wl.rho if rho is None else rho
+    n_len = [int(v) for v in x["n_len"]]
+    m_cap = api.capacity(max(n_len), rho, extra=extra)
+    shape = api.make_shape(wl.dtype, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                           wl.obs_window, wl.n, m_cap)
+    K, V, Q = to_dev(x["K"], wl.dtype), to_dev(x["V"], wl.dtype), to_dev(x["Q_obs"], wl.dtype)
+    ws = api.Workspace(S.selkv_compress_workspace_size(shape))
+    cache = api.compress(shape, n_len, rho, K, V, Q, params=params_of(p), debug=True, workspace=ws)
+    torch.cuda.synchronize()
+    flags = ws.errors()
+    assert flags == 0, "device error flags %#x" % flags
+    host = {k: v.cpu().numpy() for k, v in cache.debug.items()}
+    host["K_c"] = cache.K_c.float().cpu().numpy()
+    host["V_c"] = cache.V_c.float().cpu().numpy()
+    host["bias"] = cache.bias.cpu().numpy()
+    host["lengths"] = cache.lengths.cpu().numpy()
+    return cache, host, (K, V, Q)
+
+
+def check_topk_choice(gpu_mask: np.ndarray, values: np.ndarray, k: int, what: str) -> int:
+    """GPU top-k equals the oracle's up to swaps among near-ties of the k-th value."""
+    assert int(gpu_mask.sum()) == k, "%s: %d selected, expected %d" % (what, gpu_mask.sum(), k)
+    own = O.top_k_mask(values, k)
+    diff = np.flatnonzero(gpu_mask != own)
+    if diff.size == 0:
+        return 0
+    thr = np.sort(values)[::-1][k - 1]
+    gap = np.abs(values[diff] - thr) / max(abs(thr), 1e-300)
+    assert gap.max() <= DELTA, "%s: %d positions differ, largest gap %.3g" % (what, diff.size, gap.max())
+    return int(diff.size)
+
+
+class Stats(dict):
+    def add(self, k, v=1):
+        self[k] = self.get(k, 0) + v
+
+
+def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = None,
+                   check_values: bool = True) -> dict:
+    """Compare sequence b of one compressed layer with the oracle, stage by stage."""
+    rho = wl.rho if rho is None else rho
+    stats = stats if stats is not None else Stats()
+    n = int(x["n_len"][b])
+    K = x["K"][b, :, :n].astype(np.float64)
+    V = x["V"][b, :, :n].astype(np.float64)
+    Q = x["Q_obs"][b].astype(np.float64)
+    Hkv = K.shape[0]
+    m, m_s = O.budget(n, rho, p.recent)
+    assert int(host["lengths"][b]) == m
+    n_cand = n - p.recent
+
+    # step 1: cumulative attention and pooled contribution score (continuous)
+    a = O.cumulative_attention(Q, K, n)
+    vn = O.value_norms(V, n)
+    cp = O.pool_scores(a * vn, n_cand, p.pool_kernel)
+    a_g = host["attn"][b, :, :n].astype(np.float64)
+    err_a = np.abs(a_g - a) / (np.abs(a) + 1e-30)
+    stats["attn_rel_max"] = max(stats.get("attn_rel_max", 0.0), float(err_a.max()))
+    assert err_a.max() <= ATTN_RTOL, "attention rel err %.3g" % err_a.max()
+    sc_g = host["score"][b, :, :n_cand].astype(np.float64)
+    err_s = np.abs(sc_g - cp) / (np.abs(cp) + 1e-30)
+    stats["score_rel_max"] = max(stats.get("score_rel_max", 0.0), float(err_s.max()))
+    assert err_s.max() <= ATTN_RTOL, "score rel err %.3g" % err_s.max()
+
+    # step 2a: each KV head's top-m_s (Eq. 2)
+    per_kv = host["topk"][b, :, :n_cand].astype(bool)
+    if m_s > 0:
+        for kv in range(Hkv):
+            stats.add("topk_near_ties", check_topk_choice(per_kv[kv], cp[kv], m_s, "top-k kv%d" % kv))
+    else:
+        assert not per_kv.any()
+    # step 2b: union and trim (Sec. 3.3), continuing from the GPU's per-head choice
+    sel = O.select_shared(cp, n, m_s, p.recent, follow_per_kv=per_kv)
+    kept_idx_g = host["kept_idx"][b, :m].astype(np.int64)
+    assert (np.diff(kept_idx_g) > 0).all() and kept_idx_g.min() >= 0 and kept_idx_g.max() < n
+    kept_g = np.zeros(n, dtype=bool)
+    kept_g[kept_idx_g] = True
+    assert kept_g[n - p.recent:].all()
+    if sel.trimmed:
+        members = np.flatnonzero(sel.union)
+        mean = cp.mean(axis=0)
+        gpu_in = kept_g[:n_cand][members]
+        stats.add("trim_near_ties", check_topk_choice(gpu_in, mean[members], m_s, "trim"))
+        assert not kept_g[:n_cand][~sel.union].any(), "kept a candidate outside the union"
+    else:
+        assert (kept_g[:n_cand] == sel.union).all()
+
+    # steps 3-6 per KV head, continuing from the GPU's kept set
+    tgt_g = host["target"][b, :, :n].astype(np.int64)
+    gate_g = host["gate"][b, :, :n].astype(np.float64)
+    dec_g = host["decision"][b, :, :n]
+    Vc_o = np.empty((Hkv, m, V.shape[2]))
+    R_o = np.empty((Hkv, m))
+    ev = np.flatnonzero(~kept_g)
+    for kv in range(Hkv):
+        assert (tgt_g[kv, kept_g] == -1).all() and (dec_g[kv, kept_g] == 2).all()
+        own = O.route(a[kv], kept_g, p.bucket, p.empty_bucket)
+        diff = ev[tgt_g[kv, ev] != own[ev]]
+        for j in diff:
+            tg, to = int(tgt_g[kv, j]), int(own[j])
+            assert tg >= 0 and to >= 0 and kept_g[tg], "target of %d: gpu %d oracle %d" % (j, tg, to)
+            # same ring distance, a within DELTA of the oracle's choice
+            assert abs(tg // p.bucket - j // p.bucket) == abs(to // p.bucket - j // p.bucket)
+            assert abs(a[kv, tg] - a[kv, to]) <= DELTA * a[kv, to], "routing differs at %d" % j
+        stats.add("route_near_ties", int(diff.size))
+        g_o, sim_o, dec_o = O.gate(V[kv], tgt_g[kv], p.gate_mode)
+        routed = ev[tgt_g[kv, ev] >= 0]
+        err_g = np.abs(gate_g[kv, routed] - g_o[routed])
+        stats["gate_abs_max"] = max(stats.get("gate_abs_max", 0.0), float(err_g.max(initial=0.0)))
+        assert err_g.max(initial=0.0) <= GATE_ATOL, "gate err %.3g" % err_g.max()
+        ddiff = ev[dec_g[kv, ev] != dec_o[ev]]
+        assert (np.abs(sim_o[ddiff]) <= DELTA_SIM).all(), "merge/drop differs away from sim = 0"
+        stats.add("decision_near_ties", int(ddiff.size))
+        stats.add("evicted", int(ev.size))
+        stats.add("merged", int((dec_g[kv, ev] == 1).sum()))
+        Vc_o[kv], R_o[kv] = O.merge(a[kv], V[kv], kept_idx_g, tgt_g[kv], g_o)
+    bias_o = O.gqa_bias(R_o, p.alpha)
+
+    # continuous outputs
+    np.testing.assert_array_equal(host["K_c"][b, :, :m], K[:, kept_idx_g].astype(np.float32))
+    R_g = host["ratio"][b, :, :m].astype(np.float64)
+    err_r = np.abs(R_g - R_o) / R_o
+    stats["ratio_rel_max"] = max(stats.get("ratio_rel_max", 0.0), float(err_r.max()))
+    assert err_r.max() <= RATIO_RTOL, "R rel err %.3g" % err_r.max()
+    bias_g = host["bias"][b, :, :m].astype(np.float64)
+    assert (bias_g == bias_g[:1]).all(), "bias rows differ across KV heads"
+    err_b = np.abs(bias_g[0] - bias_o)
+    stats["bias_abs_max"] = max(stats.get("bias_abs_max", 0.0), float(err_b.max()))
+    assert err_b.max() <= BIAS_ATOL, "bias err %.3g" % err_b.max()
+    Vc_g = host["V_c"][b, :, :m].astype(np.float64)
+    if wl.dtype == "bf16":
+        # the GPU rounds its fp32 result to bf16 once: within one bf16 rounding of the exact
+        # value (half an ulp, 2^-9 relative), plus fp32 noise
+        tol = np.abs(Vc_o) * 2.0 ** -8 + 1e-5
+    else:
+        tol = np.abs(Vc_o) * VC_FP32_RTOL + 1e-6
+    err_v = np.abs(Vc_g - Vc_o) - tol
+    assert err_v.max() <= 0, "V_c error beyond tolerance by %.3g" % err_v.max()
+    return dict(n=n, m=m, K_c=K[:, kept_idx_g], V_c=Vc_o, bias=bias_o, a=a, kept_idx=kept_idx_g)
+
+
+def check_decode(out_gpu: np.ndarray, want: np.ndarray, dtype: str, what: str = "decode"):
+    err = np.abs(out_gpu.astype(np.float64) - want)
+    if dtype == "bf16":
+        assert err.max() <= DEC_BF16_MAX, "%s max-abs %.3g" % (what, err.max())
+        assert err.mean() <= DEC_BF16_MEAN, "%s mean-abs %.3g" % (what, err.mean())
+    else:
+        rel = err.max() / max(np.abs(want).max(), 1e-30)
+        assert rel <= DEC_FP32_REL, "%s rel %.3g" % (what, rel)
+    return float(err.max()), float(err.mean())

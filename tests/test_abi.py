@@ -1,0 +1,116 @@
+"""The C-ABI library on the host: it loads, exports every function include/selkv.h declares,
+sizes workspaces, and rejects invalid arguments with a status code before any CUDA call (so
+these run without a GPU; no call here reaches a kernel launch)."""
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+import paper_2607_16213_gb300 as S
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+FAKE = 1 << 40          # a 256-aligned address that is never dereferenced: every call below
+                        # fails validation first
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_16213_gb300 import build as b
+    b.build()
+    return S.library()
+
+
+def shape(**kw):
+    base = dict(dtype=S.SELKV_BF16, batch=1, num_q_heads=32, num_kv_heads=8, head_dim=128,
+                obs_window=64, n_cap=16384, m_cap=4160)
+    base.update(kw)
+    return S.selkv_shape(**base)
+
+
+def test_exports_every_declared_symbol(lib):
+    names = S.exported_symbols()
+    assert {"selkv_compress", "selkv_decode_attn", "selkv_compress_workspace_size",
+            "selkv_decode_workspace_size", "selkv_workspace_init", "selkv_workspace_error",
+            "selkv_status_string", "selkv_kernel_launches"} <= set(names)
+    out = subprocess.run(["nm", "-D", "--defined-only", S.library_path()], capture_output=True,
+                         text=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    for n in names:
+        assert n in exported, n
+        assert hasattr(lib, n)
+    assert all(e.startswith("selkv_") for e in exported), exported
+
+
+def test_status_strings(lib):
+    assert S.selkv_status_string(S.SELKV_OK) == "ok"
+    assert "workspace" in S.selkv_status_string(S.SELKV_ERR_WORKSPACE)
+    assert S.selkv_status_string(99) == "unknown status"
+
+
+def test_workspace_sizes(lib):
+    s = shape()
+    c = S.selkv_compress_workspace_size(s)
+    d = S.selkv_decode_workspace_size(s)
+    assert c > 256 and d > 256 and c % 256 == 0 and d % 256 == 0
+    assert S.selkv_compress_workspace_size(shape(n_cap=32768)) > c
+    assert S.selkv_compress_workspace_size(shape(num_kv_heads=7)) == 0      # 32 % 7 != 0
+    assert S.selkv_compress_workspace_size(shape(batch=0)) == 0
+    assert S.selkv_decode_workspace_size(shape(dtype=5)) == 0
+
+
+def _compress(s, n_len, rho=0.25, params=None, ptrs=None, ws=FAKE, wsb=1 << 40):
+    p = params or S.selkv_params.defaults()
+    t = dict(K=FAKE, V=FAKE, Q=FAKE, Kc=FAKE, Vc=FAKE, bias=FAKE, lengths=FAKE)
+    t.update(ptrs or {})
+    return S.selkv_compress(s, n_len, rho, p, t["K"], t["V"], t["Q"], t["Kc"], t["Vc"], t["bias"],
+                            t["lengths"], None, ws, wsb, 0)
+
+
+@pytest.mark.parametrize("case", [
+    dict(n_len=[16384], rho=0.0),                 # rho must be in (0, 1]
+    dict(n_len=[16384], rho=1.5),
+    dict(n_len=[40]),                              # W = 64 > n_b
+    dict(n_len=[20000]),                           # n_b > n_cap
+    dict(n_len=[100], rho=0.1),                    # m = 10 < recent window 16
+    dict(n_len=[16384], rho=0.5),                  # m = 8192 > m_cap
+    dict(n_len=[16384], ptrs=dict(K=0)),           # NULL tensor
+    dict(n_len=[16384], ptrs=dict(V=FAKE + 8)),    # misaligned tensor
+    dict(n_len=[16384], params=S.selkv_params.defaults(pool_kernel=4)),   # even kernel
+    dict(n_len=[16384], params=S.selkv_params.defaults(gate_mode=7)),
+    dict(n_len=[16384], params=S.selkv_params.defaults(alpha=float("nan"))),
+])
+def test_compress_rejects_invalid_arguments(lib, case):
+    assert _compress(shape(), **case) == S.SELKV_ERR_INVALID_ARG
+
+
+def test_compress_unsupported_and_workspace(lib):
+    assert _compress(shape(head_dim=96), [16384]) == S.SELKV_ERR_UNSUPPORTED
+    assert _compress(shape(), [16384], params=S.selkv_params.defaults(bucket=64)) == S.SELKV_ERR_UNSUPPORTED
+    assert _compress(shape(), [16384], ws=0) == S.SELKV_ERR_WORKSPACE
+    assert _compress(shape(), [16384], ws=FAKE + 16) == S.SELKV_ERR_WORKSPACE
+    assert _compress(shape(), [16384], wsb=1024) == S.SELKV_ERR_WORKSPACE
+    assert _compress(shape(batch=2), [16384, 16384], ptrs=dict(Q=None)) == S.SELKV_ERR_INVALID_ARG
+
+
+def test_decode_rejects_invalid_arguments(lib):
+    s = shape()
+    dec = lambda **kw: S.selkv_decode_attn(
+        kw.get("shape", s), kw.get("q", FAKE), FAKE, FAKE, kw.get("bias", FAKE), FAKE,
+        kw.get("k_new", None), kw.get("v_new", None), FAKE, kw.get("ws", FAKE),
+        kw.get("wsb", 1 << 40), 0)
+    assert dec(q=0) == S.SELKV_ERR_INVALID_ARG
+    assert dec(k_new=FAKE) == S.SELKV_ERR_INVALID_ARG          # k_new without v_new
+    assert dec(bias=FAKE + 4) == S.SELKV_ERR_INVALID_ARG
+    assert dec(shape=shape(head_dim=80)) == S.SELKV_ERR_UNSUPPORTED
+    assert dec(shape=shape(m_cap=0)) == S.SELKV_ERR_INVALID_ARG
+    assert dec(ws=0) == S.SELKV_ERR_WORKSPACE
+    assert dec(wsb=100) == S.SELKV_ERR_WORKSPACE
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    import paper_2607_16213_gb300._binding as bind
+    monkeypatch.setattr(bind, "_LIB", None)
+    monkeypatch.setattr(bind, "library_path", lambda: str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        bind.library()

@@ -1,0 +1,223 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the same seeded
+inputs.  Selections, routing targets and merge/drop decisions must agree exactly up to the
+near-tie rule of tests/parity.py; continuous outputs within the stated tolerances."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import selkv_oracle as O
+from paper_2607_16213_gb300 import api
+import paper_2607_16213_gb300 as S
+
+from parity import (Stats, check_decode, check_sequence, params_of, run_compress, to_dev)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2607_16213_gb300 import build as b
+    b.build()
+    S.library()
+
+
+# Small workloads that still span several 64-wide tiles, several buckets and ragged tails.
+SMALL = {
+    "tiny": synth.WORKLOADS["tiny"],
+    "bf16_ragged": synth.WORKLOADS["llama_layer"].with_(name="bf16_ragged", batch=3, n=3001,
+                                                        num_q_heads=8, num_kv_heads=2,
+                                                        ragged=(0.5, 1.0), seed=11),
+    "bf16_d64_g4": synth.WORKLOADS["llama_layer"].with_(name="bf16_d64_g4", batch=2, n=2500,
+                                                        head_dim=64, num_q_heads=16,
+                                                        num_kv_heads=4, obs_window=40, seed=12),
+    "fp32_d128": synth.WORKLOADS["tiny"].with_(name="fp32_d128", head_dim=128, n=1500, batch=2,
+                                               ragged=(0.6, 1.0), seed=13),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_compress_parity_small(name):
+    wl = SMALL[name]
+    x = synth.gen_layer(wl, 0)
+    p = O.Params()
+    _, host, _ = run_compress(wl, x, p)
+    st = Stats()
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p, stats=st)
+    print(name, dict(st))
+
+
+@pytest.mark.parametrize("gate_mode", [O.GATE_OPEN, O.GATE_CLOSED])
+def test_compress_gate_end_points(gate_mode):
+    wl = SMALL["bf16_ragged"]
+    x = synth.gen_layer(wl, 1)
+    p = O.Params(gate_mode=gate_mode)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p)
+        m = int(host["lengths"][b])
+        if gate_mode == O.GATE_CLOSED:   # pure eviction: V_c = V[S] exactly, R = 1, bias = 0
+            kept = host["kept_idx"][b, :m]
+            np.testing.assert_array_equal(host["V_c"][b, :, :m], x["V"][b][:, kept])
+            np.testing.assert_array_equal(host["ratio"][b, :, :m], 1.0)
+            np.testing.assert_array_equal(host["bias"][b, :, :m], 0.0)
+
+
+@pytest.mark.parametrize("case", [
+    dict(rho=1.0),                                   # nothing evicted
+    dict(rho=16 / 3001 + 1e-9),                      # m_s = 0: only the recent window
+    dict(p=dict(empty_bucket=O.EMPTY_DROP), rho=0.1),
+    dict(p=dict(bucket=16, pool_kernel=3, recent=0)),
+    dict(p=dict(bucket=7, pool_kernel=1, recent=5, alpha=1.0)),
+    dict(p=dict(alpha=0.0)),
+])
+def test_compress_edge_cases(case):
+    wl = SMALL["bf16_ragged"].with_(batch=1, ragged=None)
+    x = synth.gen_layer(wl, 2)
+    p = O.Params(**case.get("p", {}))
+    rho = case.get("rho", wl.rho)
+    _, host, _ = run_compress(wl, x, p, rho=rho)
+    check_sequence(wl, x, host, 0, p, rho=rho)
+    m = int(host["lengths"][0])
+    if rho == 1.0:
+        np.testing.assert_array_equal(host["kept_idx"][0, :m], np.arange(wl.n))
+        np.testing.assert_array_equal(host["V_c"][0, :, :m], x["V"][0])
+        np.testing.assert_array_equal(host["bias"][0, :, :m], 0.0)
+    if p.alpha == 0.0:
+        np.testing.assert_array_equal(host["bias"][0, :, :m], 0.0)
+
+
+def test_window_equals_sequence():
+    wl = SMALL["tiny"].with_(n=96, obs_window=96, rho=0.5)
+    x = synth.gen_layer(wl, 0)
+    p = O.Params()
+    _, host, _ = run_compress(wl, x, p)
+    check_sequence(wl, x, host, 0, p)
+
+
+def test_compress_parity_llama_layer():
+    """One Llama-3-8B-shaped layer at 16k (32 q / 8 KV heads, d = 128, bf16, W = 64)."""
+    wl = synth.WORKLOADS["llama_layer"]
+    x = synth.gen_layer(wl, 0, threads=8)
+    p = O.Params()
+    _, host, _ = run_compress(wl, x, p)
+    st = Stats()
+    check_sequence(wl, x, host, 0, p, stats=st)
+    print("llama_layer", dict(st))
+
+
+def _decode_case(wl, layer, steps, use_bias=True):
+    x = synth.gen_layer(wl, layer, threads=8)
+    p = O.Params()
+    cache, host, _ = run_compress(wl, x, p, extra=steps)
+    dec = synth.gen_decode(wl, layer, steps)
+    Kc0 = cache.K_c.double().cpu().numpy()
+    Vc0 = cache.V_c.double().cpu().numpy()
+    bias0 = cache.bias.double().cpu().numpy()
+    lens0 = cache.lengths.cpu().numpy().copy()
+    ws = api.Workspace(S.selkv_decode_workspace_size(cache.shape))
+    worst = (0.0, 0.0)
+    for t in range(steps):
+        q = to_dev(dec["q"][t], wl.dtype)
+        kn, vn = to_dev(dec["k_new"][t], wl.dtype), to_dev(dec["v_new"][t], wl.dtype)
+        out = api.decode(cache, q, kn, vn, use_bias=use_bias, workspace=ws).float().cpu().numpy()
+        for b in range(wl.batch):
+            L0 = int(lens0[b])
+            Kc = np.concatenate([Kc0[b, :, :L0], dec["k_new"][:t + 1, b].transpose(1, 0, 2)], axis=1)
+            Vc = np.concatenate([Vc0[b, :, :L0], dec["v_new"][:t + 1, b].transpose(1, 0, 2)], axis=1)
+            bs = np.concatenate([bias0[b, 0, :L0], np.zeros(t + 1)]) if use_bias else None
+            want = O.decode(dec["q"][t, b], Kc, Vc, bs, L0 + t + 1)
+            e = check_decode(out[b], want, wl.dtype, "step %d seq %d" % (t, b))
+            worst = (max(worst[0], e[0]), max(worst[1], e[1]))
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    lens = cache.lengths.cpu().numpy()
+    np.testing.assert_array_equal(lens, lens0 + steps)
+    Kc = cache.K_c.float().cpu().numpy()
+    Vc = cache.V_c.float().cpu().numpy()
+    bias = cache.bias.cpu().numpy()
+    for b in range(wl.batch):
+        L0 = int(lens0[b])
+        np.testing.assert_array_equal(Kc[b, :, L0:L0 + steps], dec["k_new"][:, b].transpose(1, 0, 2))
+        np.testing.assert_array_equal(Vc[b, :, L0:L0 + steps], dec["v_new"][:, b].transpose(1, 0, 2))
+        if use_bias:
+            np.testing.assert_array_equal(bias[b, :, L0:L0 + steps], 0.0)
+    return worst
+
+
+@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4", "fp32_d128"])
+def test_decode_parity_small(name):
+    worst = _decode_case(SMALL[name], 0, steps=4)
+    print(name, "decode worst max/mean abs", worst)
+
+
+def test_decode_parity_tiny_16_steps():
+    """The tiny workload's 16 decode steps with fresh N(0, 1) queries and appended rows."""
+    worst = _decode_case(synth.WORKLOADS["tiny"], 0, steps=16)
+    print("tiny 16 steps", worst)
+
+
+def test_decode_parity_llama_layer():
+    worst = _decode_case(synth.WORKLOADS["llama_layer"], 0, steps=3)
+    print("llama_layer decode", worst)
+
+
+def test_decode_without_bias_is_plain_attention():
+    worst = _decode_case(SMALL["bf16_ragged"], 3, steps=2, use_bias=False)
+    print("no bias", worst)
+
+
+def test_decode_full_cache_uncompressed():
+    """bias = NULL over an uncompressed cache (m_cap = n_cap, lengths = n): exact attention."""
+    wl = SMALL["bf16_ragged"]
+    x = synth.gen_layer(wl, 4)
+    shape = api.make_shape(wl.dtype, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                           wl.obs_window, wl.n, wl.n)
+    cache = api.CompressedCache(shape=shape, K_c=to_dev(x["K"], wl.dtype), V_c=to_dev(x["V"], wl.dtype),
+                                bias=torch.zeros((wl.batch, wl.num_kv_heads, wl.n), device="cuda"),
+                                lengths=torch.from_numpy(x["n_len"].astype(np.int32)).cuda())
+    dec = synth.gen_decode(wl, 4, 1)
+    out = api.decode(cache, to_dev(dec["q"][0], wl.dtype), use_bias=False).float().cpu().numpy()
+    for b in range(wl.batch):
+        n = int(x["n_len"][b])
+        want = O.decode(dec["q"][0, b], x["K"][b], x["V"][b], None, n)
+        check_decode(out[b], want, wl.dtype)
+
+
+def test_decode_edge_lengths():
+    """Empty cache: without a new row out = 0; with one, out = v_new.  A full cache with an
+    append sets the capacity flag and attends over the existing rows only."""
+    wl = SMALL["tiny"]
+    shape = api.make_shape("fp32", 2, 4, 2, 64, 32, 64, 64)
+    cache = api.alloc_compressed(shape)
+    g = torch.Generator().manual_seed(0)
+    cache.K_c.copy_(torch.randn(cache.K_c.shape, generator=g))
+    cache.V_c.copy_(torch.randn(cache.V_c.shape, generator=g))
+    cache.lengths.copy_(torch.tensor([0, 64], dtype=torch.int32))
+    q = torch.randn((2, 4, 64), generator=g).cuda()
+    kn = torch.randn((2, 2, 64), generator=g).cuda()
+    vn = torch.randn((2, 2, 64), generator=g).cuda()
+    ws = api.Workspace(S.selkv_decode_workspace_size(shape))
+    out = api.decode(cache, q, workspace=ws).cpu().numpy()
+    np.testing.assert_array_equal(out[0], 0.0)
+    assert ws.errors() == 0
+    out = api.decode(cache, q, kn, vn, workspace=ws).cpu().numpy()
+    for h in range(4):
+        np.testing.assert_allclose(out[0, h], vn[0, h // 2].cpu().numpy(), rtol=1e-6)
+    assert ws.errors() == S.SELKV_DEVERR_CAPACITY
+    lens = cache.lengths.cpu().numpy()
+    np.testing.assert_array_equal(lens, [1, 64])
+    want = O.decode(q[1].cpu().double().numpy(), cache.K_c[1].cpu().double().numpy(),
+                    cache.V_c[1].cpu().double().numpy(), cache.bias[1].cpu().double().numpy(), 64)
+    check_decode(out[1], want, "fp32")
+
+
+def test_repeat_runs_are_bitwise_identical():
+    wl = SMALL["bf16_ragged"]
+    x = synth.gen_layer(wl, 5)
+    p = O.Params()
+    _, h1, _ = run_compress(wl, x, p)
+    _, h2, _ = run_compress(wl, x, p)
+    for k in ("attn", "score", "kept_idx", "target", "gate", "V_c", "bias"):
+        np.testing.assert_array_equal(h1[k], h2[k], err_msg=k)

@@ -195,7 +195,7 @@ def test_routing_brute_force():
             assert t[j] == best
 
 
-# ---------------------------------------------------------------- Eq. 4-6, Sec. 3.5
+# ---------------------------------------------------------------- Eq. 4-6, Sec. 3.5-3.6
 def test_gate_merge_ratio_worked_example():
     gd = golden("gate_merge.json")
     V = np.array([gd["v_target"]] + gd["contributors"], dtype=float)
@@ -233,7 +233,7 @@ def _tiny(seed=0, **kw):
 
 
 def test_gate_closed_is_pure_eviction():
-    """g = 0 everywhere reduces Eq. 5 to dropping (Sec. 3.4; ablation 'eviction only')."""
+    """g = 0 everywhere reduces Eq. 5 to dropping (Sec. 3.5; ablation 'eviction only')."""
     wl, K, V, Q, n = _tiny()
     r = O.compress(K, V, Q, n, wl.rho, O.Params(gate_mode=O.GATE_CLOSED))
     # (a_i v_i) / a_i is v_i up to one rounding of fp64
@@ -246,7 +246,7 @@ def test_gate_closed_is_pure_eviction():
 
 def test_gate_open_is_attention_weighted_merge():
     """g = 1 reduces Eq. 5 to the attention-weighted average of each kept token and the
-    tokens routed to it (Sec. 3.4; ablation 'merge all'), computed here by explicit scans."""
+    tokens routed to it (Sec. 3.5; ablation 'merge all'), computed here by explicit scans."""
     wl, K, V, Q, n = _tiny(seed=1)
     r = O.compress(K, V, Q, n, wl.rho, O.Params(gate_mode=O.GATE_OPEN))
     for kv in range(K.shape[0]):
@@ -293,7 +293,7 @@ def test_decode_bias_matches_sdpa_additive_mask():
 def test_merged_duplicates_recover_softmax_mass():
     """m identical tokens merged into one kept copy with g = 1 and equal attention give
     R = m; with alpha = 1 the bias is ln m and decode over the compressed cache equals decode
-    over the full cache exactly (the attention-sag correction of Sec. 3.5)."""
+    over the full cache exactly (the attention-sag correction of Sec. 3.6)."""
     r = rng(8)
     Hq, Hkv, W, d, n, B = 2, 1, 4, 8, 64, 32
     K = r.standard_normal((Hkv, n, d))
