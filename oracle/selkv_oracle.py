@@ -144,16 +144,6 @@ def top_k_mask(values: np.ndarray, k: int) -> np.ndarray:
     return mask
 
 
-def kth_gap(values: np.ndarray, k: int) -> float:
-    """Relative gap between the k-th and (k+1)-th best values (0 if either is missing):
-    how far the top-k boundary is from a tie."""
-    if k <= 0 or k >= values.shape[0]:
-        return math.inf
-    s = np.sort(values)[::-1]
-    hi, lo = s[k - 1], s[k]
-    return float((hi - lo) / max(abs(hi), 1e-300))
-
-
 @dataclass
 class Selection:
     per_kv: np.ndarray        # [Hkv][n_cand] bool: each KV head's top-m_s (Eq. 2)
@@ -239,25 +229,6 @@ def route(a_kv: np.ndarray, kept: np.ndarray, bucket: int, empty_policy: int) ->
         for j in evicted:
             target[j] = t
     return target
-
-
-def routing_gap(a_kv: np.ndarray, kept: np.ndarray, target: np.ndarray, bucket: int,
-                j: int) -> float:
-    """Relative gap between the chosen target's a and the best other candidate of the same
-    candidate set (used to tell near-ties from real disagreements)."""
-    t = int(target[j])
-    if t < 0:
-        return math.inf
-    b, bt = j // bucket, t // bucket
-    # candidate set: the ring that contains t, at t's bucket distance from j's bucket
-    r = abs(bt - b)
-    n = kept.shape[0]
-    cands = [i for bb in {b - r, b + r} if 0 <= bb * bucket < n
-             for i in range(bb * bucket, min(n, (bb + 1) * bucket)) if kept[i] and i != t]
-    if not cands:
-        return math.inf
-    other = max(a_kv[i] for i in cands)
-    return float((a_kv[t] - other) / max(abs(a_kv[t]), 1e-300))
 
 
 # ----------------------------------------------------------------------------------------
