@@ -186,6 +186,35 @@ SELKV_API selkv_status selkv_decode_attn(const selkv_shape* shape, const void* q
                                const void* v_new, void* out, void* workspace,
                                size_t workspace_bytes, selkv_stream_t stream);
 
+/* ---------------------------------------------------------------------------------------
+ * Decode without a workspace.  The paper has no counterpart: this is a deployment variant of
+ * selkv_decode_attn for callers that cannot allocate device memory, such as code running
+ * inside a host framework that owns every device buffer and passes a kernel only its inputs
+ * and outputs, or a serving loop that must not call cudaMalloc / cudaFree (cudaFree
+ * synchronises the device) and has no workspace planned for this call.
+ *
+ * It computes exactly what selkv_decode_attn computes, with the same arguments except the
+ * workspace; the scratch it needs (split partials, arrival counters) lives in one static
+ * device array of SELKV_STATIC_SCRATCH_BYTES inside the library, reserved on every GPU that
+ * loads the library until the process exits.  The call allocates nothing.
+ *   - Shapes whose scratch exceeds SELKV_STATIC_SCRATCH_BYTES return SELKV_ERR_WORKSPACE
+ *     before any launch (about B * Hq * splits * (d + 2) * 4 bytes plus counters).
+ *   - Every call shares the array and it keeps the last call's contents; each call clears the
+ *     part that must start at zero before its kernel.  Calls that overlap on the GPU (on
+ *     different streams or from different host threads) race on the array: serialise them.
+ *   - The first call on a device looks up the array's device address with that device
+ *     current; make that first call before any stream capture.
+ *   - flags_out: optional device uint32 that receives the SELKV_DEVERR_* bits (OR-ed in,
+ *     never cleared); NULL drops them.
+ * ------------------------------------------------------------------------------------- */
+#define SELKV_STATIC_SCRATCH_BYTES (4u << 20)
+
+SELKV_API selkv_status selkv_decode_attn_static(const selkv_shape* shape, const void* q,
+                                                void* K_c, void* V_c, float* bias,
+                                                int32_t* lengths, const void* k_new,
+                                                const void* v_new, void* out,
+                                                uint32_t* flags_out, selkv_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -14,5 +14,6 @@ from ._binding import (  # noqa: F401
     SelKVError, selkv_shape, selkv_params, selkv_compress_debug, library, library_path,
     exported_symbols, check, selkv_status_string, selkv_kernel_launches, selkv_workspace_init,
     selkv_workspace_error, selkv_compress_workspace_size, selkv_compress,
-    selkv_decode_workspace_size, selkv_decode_attn,
+    selkv_decode_workspace_size, selkv_decode_attn, selkv_decode_attn_static,
+    SELKV_STATIC_SCRATCH_BYTES,
 )

@@ -16,6 +16,7 @@ SELKV_GATE_COSINE, SELKV_GATE_OPEN, SELKV_GATE_CLOSED = 0, 1, 2
 SELKV_EMPTY_EXPAND, SELKV_EMPTY_DROP = 0, 1
 SELKV_DEVERR_CAPACITY, SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT = 1, 2, 4, 8
 SELKV_MAX_BATCH = 1024
+SELKV_STATIC_SCRATCH_BYTES = 4 << 20
 
 c_i32, c_u32, c_u64, c_sz, c_vp, c_f32, c_f64 = (ctypes.c_int32, ctypes.c_uint32, ctypes.c_uint64,
                                                  ctypes.c_size_t, ctypes.c_void_p, ctypes.c_float,
@@ -80,6 +81,8 @@ def library() -> ctypes.CDLL:
         "selkv_decode_workspace_size": (c_sz, [ctypes.POINTER(selkv_shape)]),
         "selkv_decode_attn": (c_i32, [ctypes.POINTER(selkv_shape), c_vp, c_vp, c_vp, c_vp, c_vp,
                                       c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]),
+        "selkv_decode_attn_static": (c_i32, [ctypes.POINTER(selkv_shape), c_vp, c_vp, c_vp, c_vp,
+                                             c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -168,3 +171,11 @@ def selkv_decode_attn(shape: selkv_shape, q, K_c, V_c, bias, lengths, k_new, v_n
     return library().selkv_decode_attn(ctypes.byref(shape), _ptr(q), _ptr(K_c), _ptr(V_c), _ptr(bias),
                                        _ptr(lengths), _ptr(k_new), _ptr(v_new), _ptr(out),
                                        _ptr(workspace), int(workspace_bytes), _stream(stream))
+
+
+def selkv_decode_attn_static(shape: selkv_shape, q, K_c, V_c, bias, lengths, k_new, v_new, out,
+                             flags_out=None, stream=None) -> int:
+    """See include/selkv.h: the decode for callers that cannot allocate (no workspace)."""
+    return library().selkv_decode_attn_static(ctypes.byref(shape), _ptr(q), _ptr(K_c), _ptr(V_c),
+                                              _ptr(bias), _ptr(lengths), _ptr(k_new), _ptr(v_new),
+                                              _ptr(out), _ptr(flags_out), _stream(stream))
