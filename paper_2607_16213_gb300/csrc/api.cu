@@ -8,7 +8,6 @@
 
 namespace selkv {
 cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
-cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_norm_pool(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_select(const CompressArgs& a, float* tkey, uint8_t* uflag, cudaStream_t s);
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s);
@@ -53,7 +52,8 @@ CompressPlan plan_compress(const selkv_shape& s) {
   };
   const size_t B = s.batch, Hkv = s.num_kv_heads, n = s.n_cap;
   p.R = (s.num_q_heads / s.num_kv_heads) * s.obs_window;
-  p.nchunks = (int)((n + kRowChunk - 1) / kRowChunk);
+  p.nchunks = score_uses_tc(s.dtype, s.head_dim, p.R) ? score_tc_splits(s.batch, s.num_kv_heads, s.n_cap, kPlanSMs)
+                                                       : (int)((n + kRowChunk - 1) / kRowChunk);
   p.seq_n = take(B * 4);
   p.seq_m = take(B * 4);
   p.rowpart = take(B * Hkv * (size_t)p.nchunks * p.R * sizeof(float2));
@@ -233,7 +233,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = launch_setup(a, tab, st);
-  if (e == cudaSuccess) e = launch_score_simt(a, st);
+  if (e == cudaSuccess) e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st) : launch_score_simt(a, st);
   if (e == cudaSuccess) e = launch_norm_pool(a, st);
   if (e == cudaSuccess) e = launch_select(a, at<float>(workspace, plan.tkey), at<uint8_t>(workspace, plan.uflag), st);
   if (e == cudaSuccess) e = launch_merge(a, st);

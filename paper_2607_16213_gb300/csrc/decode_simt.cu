@@ -1,4 +1,4 @@
-// Compensated decode attention on CUDA cores (fp32 arithmetic; both storage dtypes).
+// Compensated decode attention on CUDA cores for fp32 caches (bf16 caches use decode_tc.cu).
 //
 //   out[b][h] = sum_i softmax_i(q_h . k_i / sqrt(d) + bias_i) v_i      (Alg. 1 decode,
 //                                                                     Sec. 3.6 compensation)
@@ -11,6 +11,7 @@
 // is then written at row lengths[b]; the last (b, kv) of a sequence bumps lengths[b].
 #include <algorithm>
 
+#include "decode_common.cuh"
 #include "selkv_internal.cuh"
 
 namespace selkv {
@@ -126,73 +127,10 @@ __global__ __launch_bounds__(kWarps * 32) void decode_simt_kernel(DecodeArgs a) 
     for (int e = 0; e < PER; ++e) wo[warp][g][lane * PER + e] = o[g][e];
   }
   __syncthreads();
-  float* part = a.partial;
-  for (int i = tid; i < G * D; i += blockDim.x) {
-    const int g = i / D, d = i % D;
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, wm[w][g]);
-    float sl = 0.f, so = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const float f = exp2f(wm[w][g] - M);
-        sl += wl[w][g] * f;
-        so += wo[w][g][d] * f;
-      }
-    }
-    float* pp = part + (((size_t)b * a.Hq + kv * G + g) * S + s) * (D + 2);
-    pp[d] = so;
-    if (d == 0) {
-      pp[D] = M;
-      pp[D + 1] = sl;
-    }
-  }
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    const uint32_t prev = atomicAdd(&a.cnt_head[bk], 1u);
-    s_last = (prev == (uint32_t)S - 1u);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  for (int i = tid; i < G * D; i += blockDim.x) {
-    const int g = i / D, d = i % D;
-    const float* pp = part + ((size_t)b * a.Hq + kv * G + g) * S * (D + 2);
-    float M = -INFINITY;
-    for (int t = 0; t < S; ++t) M = fmaxf(M, __ldcg(pp + (size_t)t * (D + 2) + D));
-    float sl = 0.f, so = 0.f;
-    if (M != -INFINITY) {
-      for (int t = 0; t < S; ++t) {
-        const float* q = pp + (size_t)t * (D + 2);
-        const float f = exp2f(__ldcg(q + D) - M);
-        sl += __ldcg(q + D + 1) * f;
-        so += __ldcg(q + d) * f;
-      }
-    }
-    store1(static_cast<T*>(a.out) + ((size_t)b * a.Hq + kv * G + g) * D + d, sl > 0.f ? so / sl : 0.f);
-  }
-  if (app) {
-    T* Kw = static_cast<T*>(a.Kc) + (bk * a.m_cap + L) * D;
-    T* Vw = static_cast<T*>(a.Vc) + (bk * a.m_cap + L) * D;
-    for (int d = tid; d < D; d += blockDim.x) {
-      Kw[d] = kn[d];
-      Vw[d] = vnw[d];
-    }
-    if (a.bias != nullptr && tid == 0) a.bias[bk * a.m_cap + L] = 0.f;
-  }
-  if (tid == 0) {
-    a.cnt_head[bk] = 0u;
-    if (app) {
-      __threadfence();
-      const uint32_t prev = atomicAdd(&a.cnt_seq[b], 1u);
-      if (prev == (uint32_t)a.Hkv - 1u) {
-        a.lengths[b] = L + 1;
-        a.cnt_seq[b] = 0u;
-      }
-    }
-  }
+  write_split_partial<kWarps>(a, b, kv, s, &wo[0][0][0], &wm[0][0], &wl[0][0], GM, false);
+  if (!arrive_last(a, bk, &s_last)) return;
+  combine_splits<T>(a, b, kv, &wo[0][0][0]);
+  finish_append<T>(a, b, bk, L, app);
 }
 
 template <typename T, int D>
@@ -209,15 +147,19 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 
 }  // namespace
 
+#ifndef SELKV_DEC_CTAS_PER_SM
+#define SELKV_DEC_CTAS_PER_SM 1  // decode CTAs planned per SM when splitting the rows
+#endif
+
 int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
   const int units = B * Hkv;
-  int S = (2 * num_sms + units - 1) / units;
+  int S = (SELKV_DEC_CTAS_PER_SM * num_sms + units - 1) / units;
   S = std::min(S, std::max(1, (m_cap + 63) / 64));
   return std::max(1, std::min(S, 64));
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
-  if (a.dtype == SELKV_BF16) return a.D == 128 ? launch_t<__nv_bfloat16, 128>(a, st) : launch_t<__nv_bfloat16, 64>(a, st);
+  if (a.dtype == SELKV_BF16) return launch_decode_tc(a, st);
   return a.D == 128 ? launch_t<float, 128>(a, st) : launch_t<float, 64>(a, st);
 }
 

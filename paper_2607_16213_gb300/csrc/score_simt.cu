@@ -12,6 +12,9 @@
 #include "selkv_internal.cuh"
 
 namespace selkv {
+
+cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
+
 namespace {
 
 constexpr int kTile = 64;   // rows and columns per tile
@@ -133,9 +136,8 @@ __global__ __launch_bounds__(256) void rowstats_kernel(CompressArgs a) {
 __global__ void rowstat_reduce_kernel(CompressArgs a) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= a.B * a.Hkv * a.R) return;
-  const int r = idx % a.R, bk = idx / a.R, b = bk / a.Hkv;
-  const int n = a.seq_n[b];
-  const int nch = (n + kRowChunk - 1) / kRowChunk;
+  const int r = idx % a.R, bk = idx / a.R;
+  const int nch = a.nchunks;  // chunks without visible columns hold (-inf, 0)
   const float2* part = a.rowpart + (size_t)bk * a.nchunks * a.R + r;
   float M = -INFINITY;
   for (int c = 0; c < nch; ++c) M = fmaxf(M, part[(size_t)c * a.R].x);
@@ -191,13 +193,18 @@ template <typename T, int D>
 cudaError_t launch_score_t(const CompressArgs& a, cudaStream_t s) {
   const int row_tiles = (a.R + kTile - 1) / kTile;
   rowstats_kernel<T, D><<<dim3(a.nchunks, row_tiles, a.B * a.Hkv), 256, 0, s>>>(a);
-  const int nrows = a.B * a.Hkv * a.R;
-  rowstat_reduce_kernel<<<(nrows + 255) / 256, 256, 0, s>>>(a);
+  launch_rowstat_reduce(a, s);
   colsum_kernel<T, D><<<dim3((a.n_cap + kTile - 1) / kTile, a.B * a.Hkv), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 
 }  // namespace
+
+cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s) {
+  const int nrows = a.B * a.Hkv * a.R;
+  rowstat_reduce_kernel<<<(nrows + 255) / 256, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s) {
   if (a.dtype == SELKV_BF16)

@@ -127,7 +127,12 @@ struct CompressArgs {
 
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
 
-cudaError_t launch_compress(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
+// Scoring: tensor-core path for bf16 with G W <= 256 rows, CUDA-core path otherwise.
+bool score_uses_tc(int dtype, int D, int R);
+int score_tc_splits(int B, int Hkv, int n_cap, int num_sms);
+cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s);
+cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
+cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
 
 // ---- decode -------------------------------------------------------------------------------
 struct DecodeArgs {
@@ -148,6 +153,7 @@ struct DecodeArgs {
 };
 
 int decode_splits(int B, int Hkv, int m_cap, int num_sms);
-cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);     // dispatch by dtype
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);  // bf16: TMA + tensor cores
 
 }  // namespace selkv
