@@ -8,15 +8,14 @@
 
 namespace selkv {
 cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
-cudaError_t launch_norm_pool(const CompressArgs& a, cudaStream_t s);
-cudaError_t launch_select(const CompressArgs& a, float* tkey, uint8_t* uflag, cudaStream_t s);
+cudaError_t launch_vnorm(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s);
 
 namespace {
 
 // Kernels enqueued by each call (diagnostic count, see selkv_kernel_launches).
 std::atomic<uint64_t> g_launches{0};
-constexpr int kCompressKernels = 9;
+constexpr int kCompressKernels = 15;  // with the tensor-core scoring (17 with the CUDA-core one)
 constexpr int kDecodeKernels = 1;
 // SM count used for planning the decode split: fixed, so that workspace sizes do not depend
 // on which device answers (GB300: 152 SMs).
@@ -38,7 +37,7 @@ bool shape_ok(const selkv_shape* s) {
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, thr, kflag, slot, tkey, uflag, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, kflag, slot, select, total;
   int nchunks, R;
 };
 
@@ -61,11 +60,9 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.attn = take(B * Hkv * n * 4);
   p.vnorm = take(B * Hkv * n * 4);
   p.score = take(B * Hkv * n * 4);
-  p.thr = take(B * Hkv * sizeof(uint2));
   p.kflag = take(B * n);
   p.slot = take(B * n * 4);
-  p.tkey = take(B * n * 4);
-  p.uflag = take(B * n);
+  p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
   p.total = off;
   return p;
 }
@@ -220,7 +217,6 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.attn = (debug && debug->attn) ? debug->attn : at<float>(workspace, plan.attn);
   a.vnorm = at<float>(workspace, plan.vnorm);
   a.score = (debug && debug->score) ? debug->score : at<float>(workspace, plan.score);
-  a.thr = at<uint2>(workspace, plan.thr);
   a.kflag = at<uint8_t>(workspace, plan.kflag);
   a.slot_of = at<int32_t>(workspace, plan.slot);
   if (debug != nullptr) {
@@ -234,10 +230,11 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = launch_setup(a, tab, st);
   if (e == cudaSuccess) e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st) : launch_score_simt(a, st);
-  if (e == cudaSuccess) e = launch_norm_pool(a, st);
-  if (e == cudaSuccess) e = launch_select(a, at<float>(workspace, plan.tkey), at<uint8_t>(workspace, plan.uflag), st);
+  if (e == cudaSuccess) e = launch_vnorm(a, st);
+  if (e == cudaSuccess)
+    e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
-  g_launches += kCompressKernels;
+  g_launches += score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2;
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

@@ -195,19 +195,26 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
           for (int c = 0; c < kKeys; c += 32) {
             float v[32];
             tmem_ld32(tmem + lane_base + buf * 256 + wg * 128 + c, v);
-            float cm = -INFINITY;
+            float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (full_tile && row_ok) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const bool vis = full_tile || key0 + c + i <= p;
-              v[i] = (row_ok && vis) ? v[i] * sc : -INFINITY;
-              cm = fmaxf(cm, v[i]);
+              for (int i = 0; i < 32; ++i) {
+                v[i] *= sc;
+                cm[i & 3] = fmaxf(cm[i & 3], v[i]);
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                v[i] = (row_ok && key0 + c + i <= p) ? v[i] * sc : -INFINITY;
+                cm[i & 3] = fmaxf(cm[i & 3], v[i]);
+              }
             }
-            const float mn = fmaxf(m_run, cm);
+            const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
             if (mn != -INFINITY) {
-              float s = 0.f;
+              float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int i = 0; i < 32; ++i) s += exp2f(v[i] - mn);
-              l_run = l_run * exp2f(m_run - mn) + s;
+              for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_approx(v[i] - mn);
+              l_run = l_run * ex2_approx(m_run - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
               m_run = mn;
             }
           }
@@ -233,19 +240,21 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
             float v[32];
             tmem_ld32(tmem + lane_base + buf * 256 + c, v);
             const int cnt = min(32, r_hi - c);
-            if (jrel <= 0) {
+            if (jrel <= 0 && cnt == 32) {
+              float a4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (i < cnt) {
-                  const float2 st = rstat[c + i];
-                  acc = fmaf(exp2f(fmaf(v[i], sc, -st.x)), st.y, acc);
-                }
+              for (int i = 0; i < 32; i += 2) {
+                const float4 st = *reinterpret_cast<const float4*>(&rstat[c + i]);  // rows c+i, c+i+1
+                a4[i & 3] = fmaf(ex2_approx(fmaf(v[i], sc, -st.x)), st.y, a4[i & 3]);
+                a4[(i + 1) & 3] = fmaf(ex2_approx(fmaf(v[i + 1], sc, -st.z)), st.w, a4[(i + 1) & 3]);
+              }
+              acc += (a4[0] + a4[1]) + (a4[2] + a4[3]);
             } else {
 #pragma unroll
               for (int i = 0; i < 32; ++i)
-                if (i < cnt && (c + i) % a.W >= jrel) {
+                if (i < cnt && (jrel <= 0 || (c + i) % a.W >= jrel)) {
                   const float2 st = rstat[c + i];
-                  acc = fmaf(exp2f(fmaf(v[i], sc, -st.x)), st.y, acc);
+                  acc = fmaf(ex2_approx(fmaf(v[i], sc, -st.x)), st.y, acc);
                 }
             }
           }

@@ -120,12 +120,36 @@ struct CompressArgs {
   float* attn;       // [B][Hkv][n_cap]
   float* vnorm;      // [B][Hkv][n_cap]
   float* score;      // [B][Hkv][n_cap]
-  uint2* thr;        // [B][Hkv] (score bits threshold, last index taken at the threshold)
   uint8_t* kflag;    // [B][n_cap] 1 = kept
   int32_t* slot_of;  // [B][n_cap] slot of a kept position, -1 otherwise
 };
 
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
+
+// Grid-wide exact radix selection (select_grid.cu).
+struct RadixState {
+  uint32_t prefix;    // threshold bits fixed so far (the threshold T after the last pass)
+  uint32_t krem;      // entries still to take among those matching `prefix`
+  uint32_t count_eq;  // after the last pass: entries equal to T
+  int32_t jcut;       // last position taken among the entries equal to T
+  uint32_t active;    // a selection is still being narrowed
+  uint32_t arrive;    // CTAs of the current pass that have finished (self-resetting)
+  uint32_t ucount;    // trim only: size of the union
+  uint32_t pad;
+};
+struct SelectWs {
+  RadixState* topk;     // [B * Hkv]
+  RadixState* trim;     // [B]
+  uint32_t* topk_hist;  // [B * Hkv][3][2048]
+  uint32_t* trim_hist;  // [B][3][2048]
+  size_t hist_bytes;    // both histogram arrays (contiguous)
+  uint32_t* blkcnt;     // [B][position blocks]
+  float* tkey;          // [B][n_cap] score summed over KV heads
+  uint8_t* uflag;       // [B][n_cap] member of the union
+};
+size_t select_ws_bytes(int B, int Hkv, int n_cap);
+SelectWs carve_select_ws(void* base, int B, int Hkv, int n_cap);
+cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStream_t s);
 
 // Scoring: tensor-core path for bf16 with G W <= 256 rows, CUDA-core path otherwise.
 bool score_uses_tc(int dtype, int D, int R);
