@@ -1,5 +1,6 @@
 // Split-K bookkeeping shared by the decode kernels: the per-split partial layout, the fold of
-// a CTA's warp states into one partial, the last-CTA combine of the splits, and the append.
+// a CTA's warp states into one partial, the last-CTA combine of the splits, the append and the
+// length update.
 //
 // Partial layout in the workspace (B * Hq * S * (D + 2) floats in total):
 //   o  [B][Hq][S][D]   unnormalised output of each split (fp32)
@@ -66,76 +67,63 @@ __device__ __forceinline__ bool arrive_last(const DecodeArgs& a, size_t bk, bool
   return *s_flag;
 }
 
-// Fold the S split partials of (b, kv) in split order and write out[b][kv*G + g].  `scratch`
-// holds at least 3 * G * S + G floats of shared memory.
+// Fold the S split partials of (b, kv) in split order and write out[b][kv*G + g].  Each
+// thread owns an output quad: one pass takes the max over the splits, a second sums the
+// splits' outputs and sums with weights 2^(max_t - max); the loads of both passes are
+// independent of each other, so a pass costs about one memory round trip.
 template <typename T>
-__device__ __forceinline__ void combine_splits(const DecodeArgs& a, int b, int kv, float* scratch) {
+__device__ __forceinline__ void combine_splits(const DecodeArgs& a, int b, int kv, float* /*scratch*/) {
   const int G = a.G, D = a.D, S = a.splits;
   const PartialView pv = partial_view(a);
   const size_t bh0 = (size_t)b * a.Hq + (size_t)kv * G;
-  float* sm = scratch;            // [G][S] split max
-  float* sl = sm + G * S;         // [G][S] split sum
-  float* f = sl + G * S;          // [G][S] weight of each split
-  float* Lt = f + G * S;          // [G]   total sum
-  for (int i = threadIdx.x; i < G * S; i += blockDim.x) {
-    const float2 v = __ldcg(&pv.ml[bh0 * S + i]);
-    sm[i] = v.x;
-    sl[i] = v.y;
-  }
-  __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (int g = warp; g < G; g += nw) {
-    float M = -INFINITY;
-    for (int t = lane; t < S; t += 32) M = fmaxf(M, sm[g * S + t]);
-    M = warp_max(M);
-    float L = 0.f;
-    for (int t = lane; t < S; t += 32) {
-      const float w = M == -INFINITY ? 0.f : exp2f(sm[g * S + t] - M);
-      f[g * S + t] = w;
-      L += sl[g * S + t] * w;
-    }
-    L = warp_sum(L);
-    if (lane == 0) Lt[g] = L;
-  }
-  __syncthreads();
   const int D4 = D / 4;
   for (int i = threadIdx.x; i < G * D4; i += blockDim.x) {
     const int g = i / D4, d4 = i % D4;
     const float4* op = reinterpret_cast<const float4*>(pv.o + (bh0 + g) * S * D) + d4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float2* mp = pv.ml + (bh0 + g) * S;
+    float M = -INFINITY;
 #pragma unroll 8
-    for (int t = 0; t < S; ++t) {
-      const float4 v = __ldcg(op + (size_t)t * D4);
-      const float w = f[g * S + t];
-      acc.x = fmaf(v.x, w, acc.x);
-      acc.y = fmaf(v.y, w, acc.y);
-      acc.z = fmaf(v.z, w, acc.z);
-      acc.w = fmaf(v.w, w, acc.w);
+    for (int t = 0; t < S; ++t) M = fmaxf(M, __ldcg(mp + t).x);
+    float L = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (M != -INFINITY) {
+#pragma unroll 8
+      for (int t = 0; t < S; ++t) {
+        const float2 ml = __ldcg(mp + t);
+        const float4 v = __ldcg(op + (size_t)t * D4);
+        const float w = exp2f(ml.x - M);
+        L = fmaf(ml.y, w, L);
+        acc.x = fmaf(v.x, w, acc.x);
+        acc.y = fmaf(v.y, w, acc.y);
+        acc.z = fmaf(v.z, w, acc.z);
+        acc.w = fmaf(v.w, w, acc.w);
+      }
     }
-    const float L = Lt[g];
     const float inv = L > 0.f ? 1.f / L : 0.f;
     const float r[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
     store4(static_cast<T*>(a.out) + (bh0 + g) * D + d4 * 4, r);
   }
 }
 
-// Write the appended row at row L of K_c / V_c (bias 0), reset the (b, kv) counter, and let the
-// last (b, kv) of the sequence advance lengths[b].  Called by the last CTA of (b, kv).
+// Write the appended row (k_new, v_new) at row L of K_c / V_c with bias 0.  No CTA of this
+// launch reads row L (they read rows below L), so any one CTA may do it.
 template <typename T>
-__device__ __forceinline__ void finish_append(const DecodeArgs& a, int b, size_t bk, int L, bool app) {
+__device__ __forceinline__ void write_append_row(const DecodeArgs& a, size_t bk, int L, int tid, int nthreads) {
   const int D = a.D;
-  if (app) {
-    const uint4* kn = reinterpret_cast<const uint4*>(static_cast<const T*>(a.k_new) + bk * D);
-    const uint4* vn = reinterpret_cast<const uint4*>(static_cast<const T*>(a.v_new) + bk * D);
-    uint4* Kw = reinterpret_cast<uint4*>(static_cast<T*>(a.Kc) + (bk * a.m_cap + L) * D);
-    uint4* Vw = reinterpret_cast<uint4*>(static_cast<T*>(a.Vc) + (bk * a.m_cap + L) * D);
-    const int n16 = D * (int)sizeof(T) / 16;
-    for (int i = threadIdx.x; i < n16; i += blockDim.x) {
-      Kw[i] = kn[i];
-      Vw[i] = vn[i];
-    }
-    if (a.bias != nullptr && threadIdx.x == 0) a.bias[bk * a.m_cap + L] = 0.f;
+  const uint4* kn = reinterpret_cast<const uint4*>(static_cast<const T*>(a.k_new) + bk * D);
+  const uint4* vn = reinterpret_cast<const uint4*>(static_cast<const T*>(a.v_new) + bk * D);
+  uint4* Kw = reinterpret_cast<uint4*>(static_cast<T*>(a.Kc) + (bk * a.m_cap + L) * D);
+  uint4* Vw = reinterpret_cast<uint4*>(static_cast<T*>(a.Vc) + (bk * a.m_cap + L) * D);
+  const int n16 = D * (int)sizeof(T) / 16;
+  for (int i = tid; i < n16; i += nthreads) {
+    Kw[i] = kn[i];
+    Vw[i] = vn[i];
   }
+  if (a.bias != nullptr && tid == 0) a.bias[bk * a.m_cap + L] = 0.f;
+}
+
+// Reset the (b, kv) counter and let the last (b, kv) of the sequence advance lengths[b].
+__device__ __forceinline__ void finish_lengths(const DecodeArgs& a, int b, size_t bk, int L, bool app) {
   if (threadIdx.x == 0) {
     a.cnt_head[bk] = 0u;
     if (app) {

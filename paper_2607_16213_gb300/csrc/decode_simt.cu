@@ -130,7 +130,8 @@ __global__ __launch_bounds__(kWarps * 32) void decode_simt_kernel(DecodeArgs a) 
   write_split_partial<kWarps>(a, b, kv, s, &wo[0][0][0], &wm[0][0], &wl[0][0], GM, false);
   if (!arrive_last(a, bk, &s_last)) return;
   combine_splits<T>(a, b, kv, &wo[0][0][0]);
-  finish_append<T>(a, b, bk, L, app);
+  if (app) write_append_row<T>(a, bk, L, threadIdx.x, blockDim.x);
+  finish_lengths(a, b, bk, L, app);
 }
 
 template <typename T, int D>
@@ -150,12 +151,15 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 #ifndef SELKV_DEC_CTAS_PER_SM
 #define SELKV_DEC_CTAS_PER_SM 1  // decode CTAs planned per SM when splitting the rows
 #endif
+#ifndef SELKV_DEC_MAX_SPLITS
+#define SELKV_DEC_MAX_SPLITS 64  // most splits of one (sequence, KV head)
+#endif
 
 int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
   const int units = B * Hkv;
   int S = (SELKV_DEC_CTAS_PER_SM * num_sms + units - 1) / units;
   S = std::min(S, std::max(1, (m_cap + 63) / 64));
-  return std::max(1, std::min(S, 64));
+  return std::max(1, std::min(S, SELKV_DEC_MAX_SPLITS));
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {

@@ -32,6 +32,9 @@ namespace {
 #ifndef SELKV_DEC_STAGES
 #define SELKV_DEC_STAGES 2     // tiles in flight per CTA
 #endif
+#ifndef SELKV_DEC_PDL
+#define SELKV_DEC_PDL 1        // launch with programmatic dependent launch
+#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif
@@ -84,13 +87,12 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
     prefetch_tensormap(&tmK);
     prefetch_tensormap(&tmV);
   }
-  __syncthreads();
   // Everything above touches only this CTA's shared memory; everything below may read what
   // the previous kernel in the stream wrote (lengths, the cache, the workspace).
   pdl_wait();
   pdl_launch_dependents();
-
-  int L = a.lengths[b];
+  int L = a.lengths[b];  // in flight across the barrier below
+  __syncthreads();
   if (L < 0 || L > a.m_cap) {
     if (tid == 0 && s == 0 && kv == 0) raise_flag(a.flags, SELKV_DEVERR_LENGTH);
     L = L < 0 ? 0 : a.m_cap;
@@ -295,6 +297,7 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
         }
         mrow[r] = mn;
       }
+      write_append_row<__nv_bfloat16>(a, bk, L, lane, 32);
     }
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
@@ -327,7 +330,7 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
   write_split_partial<kConsumers>(a, b, kv, s, wo, wm, wl, 16, *s_abort != 0);
   if (!arrive_last(a, bk, &s_last)) return;
   combine_splits<__nv_bfloat16>(a, b, kv, wo);
-  finish_append<__nv_bfloat16>(a, b, bk, L, app);
+  finish_lengths(a, b, bk, L, app);
 }
 
 template <int D, bool R16>
@@ -348,7 +351,7 @@ cudaError_t launch_tc_t(const DecodeArgs& a, cudaStream_t st) {
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = SELKV_DEC_PDL ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, tk, tv, a);
 }
 

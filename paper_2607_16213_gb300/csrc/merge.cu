@@ -18,8 +18,8 @@
 namespace selkv {
 namespace {
 
-template <typename T, int D>
-__global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
+template <typename T, int D, int MAXT>
+__global__ __launch_bounds__(MAXT) void merge_kernel(CompressArgs a) {
   constexpr int PER = D / 32;  // elements of a row per lane
   __shared__ float Rs[32][33];
   const int X = blockIdx.x, b = blockIdx.y;
@@ -36,14 +36,20 @@ __global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
   };
   const size_t bk = (size_t)b * a.Hkv + kv;
   const float* A = a.attn + bk * a.n_cap;
+  const float* vn = a.vnorm + bk * a.n_cap;
+  const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
+  const int base = X * Bs;
+  const int cntX = min(Bs, n - base);
+  // this lane's position of bucket X: a and ||v||, fetched together with the kept flags
+  const float A_l = lane < cntX ? A[base + lane] : -INFINITY;
+  const float vn_l = lane < cntX ? vn[base + lane] : 0.f;
   const uint32_t mX = bucket_mask(X);
   if (mX == 0u) {
     // Empty bucket: under EXPAND a neighbour's CTA owns these tokens; under DROP (or with
     // nothing kept at all) they stay without target.
     if (a.empty_bucket == SELKV_EMPTY_DROP || a.seq_m[b] == 0) {
-      const int p = X * Bs + lane;
-      if (lane < Bs && p < n) {
-        const size_t o = bk * a.n_cap + p;
+      if (lane < cntX) {
+        const size_t o = bk * a.n_cap + base + lane;
         if (a.dbg_target) a.dbg_target[o] = -1;
         if (a.dbg_gate) a.dbg_gate[o] = 0.f;
         if (a.dbg_decision) a.dbg_decision[o] = 0;
@@ -51,11 +57,8 @@ __global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
     }
     return;
   }
-  // argmax of a over the kept tokens of bucket e (larger a, then lower position).
-  auto best_in = [&](int e, uint32_t mask) -> int {
-    const bool in = (mask >> lane) & 1u;
-    float v = in ? A[e * Bs + lane] : -INFINITY;
-    int idx = in ? e * Bs + lane : INT_MAX;
+  // argmax of a over the kept tokens of a bucket (larger a, then lower position).
+  auto best_of = [&](float v, int idx) -> int {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float v2 = __shfl_xor_sync(0xffffffffu, v, o);
@@ -64,8 +67,14 @@ __global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
     }
     return idx;
   };
-  const int tau = best_in(X, mX);
-  const float a_tau = A[tau];
+  auto best_in = [&](int e, uint32_t mask) -> int {
+    const bool in = (mask >> lane) & 1u;
+    return best_of(in ? A[e * Bs + lane] : -INFINITY, in ? e * Bs + lane : INT_MAX);
+  };
+  const bool inX = (mX >> lane) & 1u;
+  const int tau = best_of(inX ? A_l : -INFINITY, inX ? base + lane : INT_MAX);
+  const float a_tau = __shfl_sync(0xffffffffu, A_l, tau - base);
+  const float vn_tau = __shfl_sync(0xffffffffu, vn_l, tau - base);
   int lo_b = X, hi_b = X;  // buckets whose evicted tokens route to tau
   if (a.empty_bucket == SELKV_EMPTY_EXPAND) {
     int L = X - 1;
@@ -89,45 +98,83 @@ __global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
       if (((X + Rb) & 1) == 0 && a_tau >= A[best_in(Rb, mR)]) hi_b = (X + Rb) / 2;
     }
   }
-  const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
-  const float* vn = a.vnorm + bk * a.n_cap;
   float vt[PER];
   if constexpr (PER == 4) load4(Vb + (size_t)tau * D + lane * 4, vt); else load2(Vb + (size_t)tau * D + lane * 2, vt);
-  const float vn_tau = vn[tau];
+
   float num[PER];
 #pragma unroll
   for (int e = 0; e < PER; ++e) num[e] = 0.f;
   float den = 0.f;
+  // Contributors in ascending position order, a batch at a time: their loads are independent
+  // and their dot-product reductions interleave (the sums stay in position order).
+  constexpr int kBatch = MAXT <= 256 ? 8 : 4;
   for (int e = lo_b; e <= hi_b; ++e) {
-    const uint32_t me = (e == X) ? mX : 0u;
-    const int pend = min(n, (e + 1) * Bs);
-    for (int p = e * Bs; p < pend; ++p) {
-      if ((me >> (p - e * Bs)) & 1u) continue;
-      float vj[PER];
-      if constexpr (PER == 4) load4(Vb + (size_t)p * D + lane * 4, vj); else load2(Vb + (size_t)p * D + lane * 2, vj);
-      float g;
-      if (a.gate_mode == SELKV_GATE_OPEN) {
-        g = 1.f;
-      } else if (a.gate_mode == SELKV_GATE_CLOSED) {
-        g = 0.f;
-      } else {
-        float dot = 0.f;
+    const int eb = e * Bs;
+    const int cnt_e = min(Bs, n - eb);
+    const uint32_t valid = cnt_e >= 32 ? 0xffffffffu : ((1u << cnt_e) - 1u);
+    const bool own = e == X;
+    uint32_t rem = valid & ~(own ? mX : 0u);
+    // a and ||v|| of bucket e, one position per lane
+    const float Ae = own ? A_l : (lane < cnt_e ? A[eb + lane] : 0.f);
+    const float Ne = own ? vn_l : (lane < cnt_e ? vn[eb + lane] : 0.f);
+    while (rem) {
+      int pos[kBatch];
+      int nb_ = 0;
 #pragma unroll
-        for (int t = 0; t < PER; ++t) dot = fmaf(vj[t], vt[t], dot);
-        dot = warp_sum(dot);
-        const float nj = vn[p];
-        const float sim = (nj == 0.f || vn_tau == 0.f) ? 0.f : dot / (nj * vn_tau);
-        g = fminf(fmaxf(sim, 0.f), 1.f);
+      for (int k = 0; k < kBatch; ++k) {
+        pos[k] = -1;
+        if (rem) {
+          pos[k] = eb + __ffs(rem) - 1;
+          rem &= rem - 1u;
+          ++nb_;
+        }
       }
-      const float w = g * A[p];
+      float vj[kBatch][PER];
+      float dot[kBatch];
 #pragma unroll
-      for (int t = 0; t < PER; ++t) num[t] = fmaf(w, vj[t], num[t]);
-      den += w;
-      if (lane == 0) {
-        const size_t o = bk * a.n_cap + p;
-        if (a.dbg_target) a.dbg_target[o] = tau;
-        if (a.dbg_gate) a.dbg_gate[o] = g;
-        if (a.dbg_decision) a.dbg_decision[o] = g > 0.f ? 1 : 0;
+      for (int k = 0; k < kBatch; ++k) {
+        if (pos[k] >= 0) {
+          if constexpr (PER == 4) load4(Vb + (size_t)pos[k] * D + lane * 4, vj[k]);
+          else load2(Vb + (size_t)pos[k] * D + lane * 2, vj[k]);
+        } else {
+#pragma unroll
+          for (int t = 0; t < PER; ++t) vj[k][t] = 0.f;
+        }
+        dot[k] = 0.f;
+#pragma unroll
+        for (int t = 0; t < PER; ++t) dot[k] = fmaf(vj[k][t], vt[t], dot[k]);
+      }
+      if (a.gate_mode == SELKV_GATE_COSINE) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+          for (int k = 0; k < kBatch; ++k) dot[k] += __shfl_xor_sync(0xffffffffu, dot[k], o);
+      }
+#pragma unroll
+      for (int k = 0; k < kBatch; ++k) {
+        if (k >= nb_) break;
+        const int src = pos[k] - eb;
+        const float ak = __shfl_sync(0xffffffffu, Ae, src);
+        const float nk = __shfl_sync(0xffffffffu, Ne, src);
+        float g;
+        if (a.gate_mode == SELKV_GATE_OPEN) {
+          g = 1.f;
+        } else if (a.gate_mode == SELKV_GATE_CLOSED) {
+          g = 0.f;
+        } else {
+          const float sim = (nk == 0.f || vn_tau == 0.f) ? 0.f : dot[k] / (nk * vn_tau);
+          g = fminf(fmaxf(sim, 0.f), 1.f);
+        }
+        const float w = g * ak;
+#pragma unroll
+        for (int t = 0; t < PER; ++t) num[t] = fmaf(w, vj[k][t], num[t]);
+        den += w;
+        if (lane == k) {
+          const size_t o = bk * a.n_cap + pos[k];
+          if (a.dbg_target) a.dbg_target[o] = tau;
+          if (a.dbg_gate) a.dbg_gate[o] = g;
+          if (a.dbg_decision) a.dbg_decision[o] = g > 0.f ? 1 : 0;
+        }
       }
     }
   }
@@ -137,63 +184,87 @@ __global__ __launch_bounds__(1024) void merge_kernel(CompressArgs a) {
   for (int t = 0; t < PER; ++t) vm[t] = tot > 0.f ? (a_tau * vt[t] + num[t]) / tot : vt[t];
   const float R_tau = a_tau > 0.f ? tot / a_tau : 1.f;
 
-  // Copy the kept tokens of X to their slots.
+  // Kept tokens of X, four at a time (loads first, then stores).
   const T* Kb = static_cast<const T*>(a.K) + bk * a.n_cap * D;
   T* Kc = static_cast<T*>(a.Kc) + bk * a.m_cap * D;
   T* Vc = static_cast<T*>(a.Vc) + bk * a.m_cap * D;
   const int32_t* so = a.slot_of + (size_t)b * a.n_cap;
   uint32_t rem = mX;
   while (rem) {
-    const int t = __ffs(rem) - 1;
-    rem &= rem - 1u;
-    const int p = X * Bs + t;
-    const int slot = so[p];
-    if (slot < 0 || slot >= a.m_cap) {
-      if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
-      continue;
-    }
-    float x[PER];
-    if constexpr (PER == 4) {
-      load4(Kb + (size_t)p * D + lane * 4, x);
-      store4(Kc + (size_t)slot * D + lane * 4, x);
-    } else {
-      load2(Kb + (size_t)p * D + lane * 2, x);
-      store1(Kc + (size_t)slot * D + lane * 2, x[0]);
-      store1(Kc + (size_t)slot * D + lane * 2 + 1, x[1]);
-    }
-    if (p == tau) {
+    constexpr int kCopy = 4;
+    int tk[kCopy], sl[kCopy];
 #pragma unroll
-      for (int e = 0; e < PER; ++e) x[e] = vm[e];
-    } else {
-      if constexpr (PER == 4) load4(Vb + (size_t)p * D + lane * 4, x); else load2(Vb + (size_t)p * D + lane * 2, x);
+    for (int k = 0; k < kCopy; ++k) {
+      tk[k] = -1;
+      sl[k] = -1;
+      if (rem) {
+        tk[k] = __ffs(rem) - 1;
+        rem &= rem - 1u;
+        sl[k] = so[base + tk[k]];
+        if (sl[k] < 0 || sl[k] >= a.m_cap) {
+          if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
+          sl[k] = -1;
+        }
+      }
     }
-    if constexpr (PER == 4) {
-      store4(Vc + (size_t)slot * D + lane * 4, x);
-    } else {
-      store1(Vc + (size_t)slot * D + lane * 2, x[0]);
-      store1(Vc + (size_t)slot * D + lane * 2 + 1, x[1]);
+    float kx[kCopy][PER], vx[kCopy][PER];
+#pragma unroll
+    for (int k = 0; k < kCopy; ++k) {
+      if (sl[k] < 0) continue;
+      const int p = base + tk[k];
+      if constexpr (PER == 4) {
+        load4(Kb + (size_t)p * D + lane * 4, kx[k]);
+        if (p != tau) load4(Vb + (size_t)p * D + lane * 4, vx[k]);
+      } else {
+        load2(Kb + (size_t)p * D + lane * 2, kx[k]);
+        if (p != tau) load2(Vb + (size_t)p * D + lane * 2, vx[k]);
+      }
+      if (p == tau) {
+#pragma unroll
+        for (int e = 0; e < PER; ++e) vx[k][e] = vm[e];
+      }
     }
-    if (lane == 0) {
-      const float Rv = (p == tau) ? R_tau : 1.f;
-      Rs[kv][t] = Rv;
-      const size_t o = bk * a.n_cap + p;
-      if (a.dbg_target) a.dbg_target[o] = -1;
-      if (a.dbg_gate) a.dbg_gate[o] = 0.f;
-      if (a.dbg_decision) a.dbg_decision[o] = 2;
-      if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = Rv;
+#pragma unroll
+    for (int k = 0; k < kCopy; ++k) {
+      if (sl[k] < 0) continue;
+      const int p = base + tk[k];
+      const int slot = sl[k];
+      if constexpr (PER == 4) {
+        store4(Kc + (size_t)slot * D + lane * 4, kx[k]);
+        store4(Vc + (size_t)slot * D + lane * 4, vx[k]);
+      } else {
+        store1(Kc + (size_t)slot * D + lane * 2, kx[k][0]);
+        store1(Kc + (size_t)slot * D + lane * 2 + 1, kx[k][1]);
+        store1(Vc + (size_t)slot * D + lane * 2, vx[k][0]);
+        store1(Vc + (size_t)slot * D + lane * 2 + 1, vx[k][1]);
+      }
+      if (lane == 0) {
+        const float Rv = (p == tau) ? R_tau : 1.f;
+        Rs[kv][tk[k]] = Rv;
+        const size_t o = bk * a.n_cap + p;
+        if (a.dbg_target) a.dbg_target[o] = -1;
+        if (a.dbg_gate) a.dbg_gate[o] = 0.f;
+        if (a.dbg_decision) a.dbg_decision[o] = 2;
+        if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = Rv;
+      }
     }
   }
   __syncthreads();
   // bias = alpha * ln(mean over KV heads of R) (Sec. 3.6, GQA), the same row for every head.
-  if (((mX >> lane) & 1u) != 0u) {
-    const int p = X * Bs + lane;
-    const int slot = so[p];
+  if (inX) {
+    const int slot = so[base + lane];
     if (slot >= 0 && slot < a.m_cap) {
       float s = 0.f;
       for (int h = 0; h < a.Hkv; ++h) s += Rs[h][lane];
       a.bias[bk * a.m_cap + slot] = a.alpha * logf(s / (float)a.Hkv);
     }
   }
+}
+
+template <typename T, int D>
+void launch_merge_t(const CompressArgs& a, dim3 grid, int threads, cudaStream_t s) {
+  if (threads <= 256) merge_kernel<T, D, 256><<<grid, threads, 0, s>>>(a);
+  else merge_kernel<T, D, 1024><<<grid, threads, 0, s>>>(a);
 }
 
 }  // namespace
@@ -203,11 +274,11 @@ cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s) {
   const dim3 grid(nb, a.B);
   const int threads = 32 * a.Hkv;
   if (a.dtype == SELKV_BF16) {
-    if (a.D == 128) merge_kernel<__nv_bfloat16, 128><<<grid, threads, 0, s>>>(a);
-    else merge_kernel<__nv_bfloat16, 64><<<grid, threads, 0, s>>>(a);
+    if (a.D == 128) launch_merge_t<__nv_bfloat16, 128>(a, grid, threads, s);
+    else launch_merge_t<__nv_bfloat16, 64>(a, grid, threads, s);
   } else {
-    if (a.D == 128) merge_kernel<float, 128><<<grid, threads, 0, s>>>(a);
-    else merge_kernel<float, 64><<<grid, threads, 0, s>>>(a);
+    if (a.D == 128) launch_merge_t<float, 128>(a, grid, threads, s);
+    else launch_merge_t<float, 64>(a, grid, threads, s);
   }
   return cudaGetLastError();
 }
