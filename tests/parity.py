@@ -202,3 +202,46 @@ def check_decode(out_gpu: np.ndarray, want: np.ndarray, dtype: str, what: str = 
         rel = err.max() / max(np.abs(want).max(), 1e-30)
         assert rel <= DEC_FP32_REL, "%s rel %.3g" % (what, rel)
     return float(err.max()), float(err.mean())
+
+
+def check_properties(wl, x, host, p: O.Params, rho=None):
+    """Structural checks of every sequence of a compressed layer that hold at any size:
+    exactly m_b kept positions in ascending order including the recent window, every evicted
+    token routed to a kept token of its own bucket when that bucket keeps one (Eq. 3), merge
+    decisions consistent with g (Eq. 4), R >= 1 and R = 1 for kept tokens that are nobody's
+    target, bias = alpha ln(mean over KV heads of R) (Sec. 3.6), keys copied unchanged, and
+    the values of kept tokens that absorbed nothing copied unchanged."""
+    rho = wl.rho if rho is None else rho
+    for b in range(wl.batch):
+        n = int(x["n_len"][b])
+        m, m_s = O.budget(n, rho, p.recent)
+        assert int(host["lengths"][b]) == m
+        kept_idx = host["kept_idx"][b, :m].astype(np.int64)
+        assert (np.diff(kept_idx) > 0).all() and kept_idx[0] >= 0 and kept_idx[-1] < n
+        kept = np.zeros(n, dtype=bool)
+        kept[kept_idx] = True
+        assert kept[n - p.recent:].all()
+        bucket_has = np.add.reduceat(kept.astype(np.int64), np.arange(0, n, p.bucket)) > 0
+        ev = np.flatnonzero(~kept)
+        tgt = host["target"][b, :, :n].astype(np.int64)
+        dec = host["decision"][b, :, :n]
+        g = host["gate"][b, :, :n]
+        R = host["ratio"][b, :, :m].astype(np.float64)
+        for kv in range(wl.num_kv_heads):
+            t = tgt[kv, ev]
+            assert (t >= 0).all() and kept[t].all(), "evicted token without a kept target"
+            own = bucket_has[ev // p.bucket]
+            assert (t[own] // p.bucket == ev[own] // p.bucket).all(), "target outside the bucket"
+            assert ((g[kv, ev] > 0) == (dec[kv, ev] == 1)).all() and (dec[kv, kept] == 2).all()
+            assert (g[kv, ev] >= 0).all() and (g[kv, ev] <= 1).all()
+            assert (R[kv] >= 1.0).all()
+            absorbed = np.zeros(n, dtype=bool)
+            absorbed[t[g[kv, ev] > 0]] = True
+            slot_abs = absorbed[kept_idx]
+            assert (R[kv][~slot_abs] == 1.0).all()
+            np.testing.assert_array_equal(host["K_c"][b, kv, :m], x["K"][b, kv, kept_idx])
+            np.testing.assert_array_equal(host["V_c"][b, kv, :m][~slot_abs], x["V"][b, kv, kept_idx][~slot_abs])
+        want_bias = p.alpha * np.log(R.mean(axis=0))
+        bias = host["bias"][b, :, :m].astype(np.float64)
+        assert (bias == bias[:1]).all()
+        np.testing.assert_allclose(bias[0], want_bias, rtol=1e-6, atol=1e-6)
