@@ -410,12 +410,17 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int):
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps}
 
 
+DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "decode_simt.cu", "ptx.cuh", "selkv_internal.cuh",
+                  "tma_host.cu")
+
+
 def kernel_revision() -> str:
-    """Content hash of the CUDA sources: profiler figures are valid only for this revision."""
+    """Content hash of the decode kernel's sources: profiler figures recorded for the decode
+    kernel are valid only for this revision."""
     import hashlib
     h = hashlib.sha256()
     cs = os.path.join(ROOT, "paper_2607_16213_gb300", "csrc")
-    for f in sorted(os.listdir(cs)):
+    for f in DECODE_SOURCES:
         with open(os.path.join(cs, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
