@@ -7,6 +7,7 @@
 //   ml [B][Hq][S]      (running max in base 2, running sum) of each split
 #pragma once
 
+#include "ptx.cuh"
 #include "selkv_internal.cuh"
 
 namespace selkv {
@@ -57,13 +58,19 @@ __device__ __forceinline__ void write_split_partial(const DecodeArgs& a, int b, 
   }
 }
 
-// One atomic arrival per CTA on the (b, kv) counter; true for the last of the S splits.
+// One atomic arrival per CTA on the (b, kv) counter; true for the last of the S splits.  The
+// CTA barrier orders every thread's partial stores before thread 0's gpu-scope fence, which
+// publishes them before the arrival (fences are cumulative); the last CTA fences again before
+// the barrier that lets its threads read the other splits' partials.
 __device__ __forceinline__ bool arrive_last(const DecodeArgs& a, size_t bk, bool* s_flag) {
-  __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) *s_flag = atomicAdd(&a.cnt_head[bk], 1u) == (uint32_t)a.splits - 1u;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const bool last = atomicAdd(&a.cnt_head[bk], 1u) == (uint32_t)a.splits - 1u;
+    if (last) __threadfence();
+    *s_flag = last;
+  }
   __syncthreads();
-  if (*s_flag) __threadfence();
   return *s_flag;
 }
 
@@ -105,6 +112,65 @@ __device__ __forceinline__ void combine_splits(const DecodeArgs& a, int b, int k
   }
 }
 
+// combine_splits with one memory round trip: the partials of (b, kv) are copied into shared
+// memory (`scratch`, 16-byte aligned, `scratch_bytes` long) with every copy in flight at
+// once, then folded there in the same order and arithmetic as combine_splits.  Heads are
+// taken in groups that fit; when not even one head's S partials fit, combine_splits runs.
+template <typename T>
+__device__ __forceinline__ void combine_splits_staged(const DecodeArgs& a, int b, int kv, unsigned char* scratch,
+                                                      int scratch_bytes) {
+  const int G = a.G, D = a.D, S = a.splits;
+  const PartialView pv = partial_view(a);
+  const size_t bh0 = (size_t)b * a.Hq + (size_t)kv * G;
+  const int ml_bytes = (G * S * 8 + 15) & ~15;
+  const int head_bytes = S * D * 4;
+  const int gc = min(G, (scratch_bytes - ml_bytes) / head_bytes);
+  if (gc < 1) {
+    combine_splits<T>(a, b, kv, nullptr);
+    return;
+  }
+  float2* mls = reinterpret_cast<float2*>(scratch);            // [G][S]
+  float* os = reinterpret_cast<float*>(scratch + ml_bytes);     // [gc][S][D]
+  const int D4 = D / 4;
+  for (int gb = 0; gb < G; gb += gc) {
+    const int ng = min(gc, G - gb);
+    const float4* src = reinterpret_cast<const float4*>(pv.o + (bh0 + gb) * S * D);  // ng heads, contiguous
+    const uint32_t dst = smem_u32(os);
+    const int n16 = ng * S * D4;
+    for (int i = threadIdx.x; i < n16; i += blockDim.x) cp_async16_cg(dst + i * 16, src + i);
+    if (gb == 0)
+      for (int i = threadIdx.x; i < G * S; i += blockDim.x) mls[i] = __ldcg(pv.ml + bh0 * S + i);
+    cp_async_wait_all();
+    __syncthreads();
+    for (int i = threadIdx.x; i < ng * D4; i += blockDim.x) {
+      const int g = i / D4, d4 = i % D4;
+      const float2* mp = mls + (gb + g) * S;
+      const float4* op = reinterpret_cast<const float4*>(os + (size_t)g * S * D) + d4;
+      float M = -INFINITY;
+      for (int t = 0; t < S; ++t) M = fmaxf(M, mp[t].x);
+      float L = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (M != -INFINITY) {
+#pragma unroll 4
+        for (int t = 0; t < S; ++t) {
+          const float2 ml = mp[t];
+          const float4 v = op[t * D4];
+          const float w = exp2f(ml.x - M);
+          L = fmaf(ml.y, w, L);
+          acc.x = fmaf(v.x, w, acc.x);
+          acc.y = fmaf(v.y, w, acc.y);
+          acc.z = fmaf(v.z, w, acc.z);
+          acc.w = fmaf(v.w, w, acc.w);
+        }
+      }
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      const float r[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+      store4(static_cast<T*>(a.out) + (bh0 + gb + g) * D + d4 * 4, r);
+    }
+    if (gb + gc < G) __syncthreads();
+  }
+}
+
 // Write the appended row (k_new, v_new) at row L of K_c / V_c with bias 0.  No CTA of this
 // launch reads row L (they read rows below L), so any one CTA may do it.
 template <typename T>
@@ -122,18 +188,27 @@ __device__ __forceinline__ void write_append_row(const DecodeArgs& a, size_t bk,
   if (a.bias != nullptr && tid == 0) a.bias[bk * a.m_cap + L] = 0.f;
 }
 
-// Reset the (b, kv) counter and let the last (b, kv) of the sequence advance lengths[b].
-__device__ __forceinline__ void finish_lengths(const DecodeArgs& a, int b, size_t bk, int L, bool app) {
+// Length bookkeeping of the last CTA of (b, kv), split in two so the atomic's round trip
+// overlaps the combine.  begin: reset the (b, kv) counter and count this head on the
+// sequence's counter; every CTA of the sequence has read lengths[b] before its own arrival,
+// so the last head to count may advance it.  end: that head writes lengths[b] = L + 1 (the
+// acquire on the counter keeps the write after the count).
+__device__ __forceinline__ uint32_t finish_lengths_begin(const DecodeArgs& a, int b, size_t bk, bool app) {
+  uint32_t old = 0u;
   if (threadIdx.x == 0) {
     a.cnt_head[bk] = 0u;
-    if (app) {
-      __threadfence();
-      if (atomicAdd(&a.cnt_seq[b], 1u) == (uint32_t)a.Hkv - 1u) {
-        a.lengths[b] = L + 1;
-        a.cnt_seq[b] = 0u;
-      }
-    }
+    if (app) old = atom_add_acquire_gpu(&a.cnt_seq[b], 1u);
   }
+  return old;
+}
+__device__ __forceinline__ void finish_lengths_end(const DecodeArgs& a, int b, int L, bool app, uint32_t old) {
+  if (threadIdx.x == 0 && app && old == (uint32_t)a.Hkv - 1u) {
+    a.lengths[b] = L + 1;
+    a.cnt_seq[b] = 0u;
+  }
+}
+__device__ __forceinline__ void finish_lengths(const DecodeArgs& a, int b, size_t bk, int L, bool app) {
+  finish_lengths_end(a, b, L, app, finish_lengths_begin(a, b, bk, app));
 }
 
 }  // namespace selkv

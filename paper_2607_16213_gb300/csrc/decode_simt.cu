@@ -155,11 +155,27 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 #define SELKV_DEC_MAX_SPLITS 64  // most splits of one (sequence, KV head)
 #endif
 
+// Split count of each (sequence, KV head).  The B * Hkv * S CTAs run in waves of
+// CTAS_PER_SM * num_sms; a wave lasts about as long as streaming one CTA's rows plus a fixed
+// fill-and-fold cost worth kFillRows rows (about 2 us at one SM's share of HBM bandwidth).
+// S minimises waves * (rows per CTA + kFillRows) over the capacity m_cap, fewest splits on ties.
 int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
-  const int units = B * Hkv;
-  int S = (SELKV_DEC_CTAS_PER_SM * num_sms + units - 1) / units;
-  S = std::min(S, std::max(1, (m_cap + 63) / 64));
-  return std::max(1, std::min(S, SELKV_DEC_MAX_SPLITS));
+  constexpr long kFillRows = 192;
+  const long units = (long)B * Hkv;
+  const long slots = std::max(1L, (long)SELKV_DEC_CTAS_PER_SM * num_sms);
+  const int smax = std::max(1, std::min(SELKV_DEC_MAX_SPLITS, (m_cap + 63) / 64));
+  int best = 1;
+  long best_cost = -1;
+  for (int S = 1; S <= smax; ++S) {
+    const long waves = (units * S + slots - 1) / slots;
+    const long rows = ((long)(m_cap + S - 1) / S + 63) / 64 * 64;
+    const long cost = waves * (rows + kFillRows);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = S;
+    }
+  }
+  return best;
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {

@@ -2,16 +2,18 @@
 //
 //   out[b][h] = sum_i softmax_i(q_h . k_i / sqrt(d) + bias_i) v_i     (Alg. 1 decode, Sec. 3.6)
 //
-// CTA (split s, KV head kv, sequence b) owns a contiguous slice of the compressed rows.  A
-// producer warp streams 64-row K and V tiles into a STAGES-deep ring of shared-memory buffers
-// with 2D TMA loads (128-byte swizzle, completion on an mbarrier per stage).  Four consumer
+// CTA (split s, KV head kv, sequence b) owns a contiguous slice of the compressed rows, cut
+// at multiples of 64 rows.  A producer warp streams 128-row K and V tiles into a STAGES-deep
+// ring of shared-memory buffers with 2D TMA loads (64-row boxes, 128-byte swizzle, completion
+// on an mbarrier per stage; a slice's last tile may be a single box high).  Eight consumer
 // warps each take 16 rows of a tile: S = Q K^T for all G query heads of the group at once
 // (mma.sync m16n8k16, bf16 in, fp32 accumulate; the G heads are the M rows, so one K tile
 // serves the whole group), the scale and the fp32 bias are applied to S before the running
 // max, then O += P V on the tensor cores.  The rows of one warp stream form one flash-decoding
-// state; the four states and then the splits are folded in a fixed order, the splits by the
-// last CTA of (b, kv) to arrive (one atomic add, no waiting).  The appended row (k_new, v_new)
-// joins the last split with bias 0 and is then written at row lengths[b].
+// state; the warp states and then the splits are folded in a fixed order, the splits by the
+// last CTA of (b, kv) to arrive (one atomic add, no waiting), which stages every split's
+// partial in the idle ring with one round of asynchronous copies.  The appended row
+// (k_new, v_new) joins the last split with bias 0 and is then written at row lengths[b].
 //
 // Every mbarrier wait is bounded: on timeout the CTA raises SELKV_DEVERR_TIMEOUT, stops, and
 // waits (bounded again) for the copies it has issued before leaving.  Launched with
@@ -43,11 +45,15 @@ constexpr int kTile = SELKV_DEC_TILE;
 constexpr int kConsumers = kTile / 16;  // consumer warps, 16 rows of a tile each
 constexpr int kThreads = (kConsumers + 1) * 32;
 constexpr int kStages = SELKV_DEC_STAGES;
+constexpr int kBoxRows = 64;   // TMA box height; split boundaries fall on multiples of it
+constexpr int kHalves = kTile / kBoxRows;
+static_assert(kTile % kBoxRows == 0, "tile is whole boxes");
 
 template <int D>
 struct Cfg {
   static constexpr int kBoxes = D / 64;                // 128-byte-wide boxes per row
-  static constexpr int kBoxBytes = kTile * 128;        // one box: kTile rows x 128 bytes
+  static constexpr int kBoxBytes = kTile * 128;        // one 128-byte column of a tile
+  static constexpr int kPieceBytes = kBoxRows * 128;   // one TMA box: kBoxRows rows x 128 bytes
   static constexpr int kTileBytes = kTile * D * 2;     // K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
@@ -102,7 +108,7 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
     if (tid == 0 && s == 0 && kv == 0) raise_flag(a.flags, SELKV_DEVERR_CAPACITY);
     app = false;
   }
-  const int chunk = ((L + S - 1) / S + kTile - 1) / kTile * kTile;
+  const int chunk = ((L + S - 1) / S + kBoxRows - 1) / kBoxRows * kBoxRows;
   const int lo = min(L, s * chunk), hi = min(L, lo + chunk);
   const int ntiles = (hi - lo + kTile - 1) / kTile;
   const int row0 = (int)(bk * a.m_cap) + lo;
@@ -128,13 +134,18 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
         }
         if (*s_abort) break;
         unsigned char* base = smem + st * C::kStageBytes;
-        mbar_arrive_expect_tx(&full[st], C::kStageBytes);
+        // a split's last tile may be cut at a box boundary: load only the boxes it covers
+        const int nh = min(kHalves, (hi - lo - t * kTile + kBoxRows - 1) / kBoxRows);
+        mbar_arrive_expect_tx(&full[st], 2 * nh * C::kBoxes * C::kPieceBytes);
+        for (int h = 0; h < nh; ++h) {
+          const int y = row0 + t * kTile + h * kBoxRows;
 #pragma unroll
-        for (int bx = 0; bx < C::kBoxes; ++bx)
-          tma_load_2d(base + bx * C::kBoxBytes, &tmK, bx * 64, row0 + t * kTile, &full[st]);
+          for (int bx = 0; bx < C::kBoxes; ++bx)
+            tma_load_2d(base + bx * C::kBoxBytes + h * C::kPieceBytes, &tmK, bx * 64, y, &full[st]);
 #pragma unroll
-        for (int bx = 0; bx < C::kBoxes; ++bx)
-          tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes, &tmV, bx * 64, row0 + t * kTile, &full[st]);
+          for (int bx = 0; bx < C::kBoxes; ++bx)
+            tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &full[st]);
+        }
         issued = t + 1;
       }
       // every issued copy must have landed before the ring is reused or the CTA exits
@@ -329,15 +340,16 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
   __syncthreads();
   write_split_partial<kConsumers>(a, b, kv, s, wo, wm, wl, 16, *s_abort != 0);
   if (!arrive_last(a, bk, &s_last)) return;
-  combine_splits<__nv_bfloat16>(a, b, kv, wo);
-  finish_lengths(a, b, bk, L, app);
+  const uint32_t seq_old = finish_lengths_begin(a, b, bk, app);
+  combine_splits_staged<__nv_bfloat16>(a, b, kv, smem, C::kRingBytes);
+  finish_lengths_end(a, b, L, app, seq_old);
 }
 
 template <int D, bool R16>
 cudaError_t launch_tc_t(const DecodeArgs& a, cudaStream_t st) {
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)a.B * a.Hkv * a.m_cap;
-  if (!encode_rows_bf16(&tk, a.Kc, rows, D, kTile) || !encode_rows_bf16(&tv, a.Vc, rows, D, kTile))
+  if (!encode_rows_bf16(&tk, a.Kc, rows, D, kBoxRows) || !encode_rows_bf16(&tv, a.Vc, rows, D, kBoxRows))
     return cudaErrorInvalidValue;
   auto kern = decode_tc_kernel<D, R16>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::kSmemBytes);
