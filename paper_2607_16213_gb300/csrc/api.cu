@@ -83,7 +83,8 @@ DecodePlan plan_decode(const selkv_shape& s) {
   p.splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs);
   p.cnt_head = take((size_t)s.batch * s.num_kv_heads * 4);
   p.cnt_seq = take((size_t)s.batch * 4);
-  p.partial = take((size_t)s.batch * s.num_q_heads * p.splits * (s.head_dim + 2) * 4);
+  p.partial = take((size_t)s.batch * s.num_kv_heads *
+                   decode_record_floats(s.num_q_heads / s.num_kv_heads, p.splits, s.head_dim) * 4);
   p.total = off;
   return p;
 }

@@ -2,9 +2,10 @@
 // a CTA's warp states into one partial, the last-CTA combine of the splits, the append and the
 // length update.
 //
-// Partial layout in the workspace (B * Hq * S * (D + 2) floats in total):
-//   o  [B][Hq][S][D]   unnormalised output of each split (fp32)
-//   ml [B][Hq][S]      (running max in base 2, running sum) of each split
+// Partial layout in the workspace: one record per (b, kv) of decode_record_floats(G, S, D)
+// floats, 16-byte aligned:
+//   o  [G][S][D]   unnormalised output of each split (fp32)
+//   ml [G][S]      (running max in base 2, running sum) of each split, padded to 16 bytes
 #pragma once
 
 #include "ptx.cuh"
@@ -13,13 +14,20 @@
 namespace selkv {
 
 struct PartialView {
-  float* o;
-  float2* ml;
+  float* base;
+  size_t rec;  // floats per (b, kv) record
+  int G, S, D;
+  __device__ __forceinline__ float* record(size_t bk) const { return base + bk * rec; }
+  __device__ __forceinline__ float* o(size_t bk, int g, int s) const {
+    return record(bk) + ((size_t)g * S + s) * D;
+  }
+  __device__ __forceinline__ float2* ml(size_t bk, int g, int s) const {
+    return reinterpret_cast<float2*>(record(bk) + (size_t)G * S * D) + g * S + s;
+  }
 };
 
 __device__ __forceinline__ PartialView partial_view(const DecodeArgs& a) {
-  float* o = a.partial;
-  return {o, reinterpret_cast<float2*>(o + (size_t)a.B * a.Hq * a.splits * a.D)};
+  return {a.partial, decode_record_floats(a.G, a.splits, a.D), a.G, a.splits, a.D};
 }
 
 // Griddepcontrol (programmatic dependent launch): a no-op for kernels launched without it.
@@ -28,15 +36,15 @@ __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// Fold NW warp states (max wm[w*rs+g], sum wl[w*rs+g], output wo[(w*rs+g)*D+d]) of heads
+// Fold NW warp states (max wm[w*rs+g], sum wl[w*rs+g], output wo[(w*rs+g)*ld+d]) of heads
 // g < G into this split's partial.  An aborted CTA leaves an empty partial.
 template <int NW>
 __device__ __forceinline__ void write_split_partial(const DecodeArgs& a, int b, int kv, int s,
                                                     const float* wo, const float* wm, const float* wl,
-                                                    int rs, bool aborted) {
-  const int G = a.G, D = a.D, S = a.splits;
+                                                    int rs, int ld, bool aborted) {
+  const int G = a.G, D = a.D;
   const PartialView pv = partial_view(a);
-  const size_t bh0 = (size_t)b * a.Hq + (size_t)kv * G;
+  const size_t bk = (size_t)b * a.Hkv + kv;
   for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
     const int g = i / D, d = i % D;
     float M = -INFINITY;
@@ -48,28 +56,23 @@ __device__ __forceinline__ void write_split_partial(const DecodeArgs& a, int b, 
       for (int w = 0; w < NW; ++w) {
         const float f = exp2f(wm[w * rs + g] - M);
         sl += wl[w * rs + g] * f;
-        so += wo[(w * rs + g) * D + d] * f;
+        so += wo[(w * rs + g) * ld + d] * f;
       }
     } else {
       M = -INFINITY;
     }
-    pv.o[((bh0 + g) * S + s) * D + d] = so;
-    if (d == 0) pv.ml[(bh0 + g) * S + s] = make_float2(M, sl);
+    pv.o(bk, g, s)[d] = so;
+    if (d == 0) *pv.ml(bk, g, s) = make_float2(M, sl);
   }
 }
 
 // One atomic arrival per CTA on the (b, kv) counter; true for the last of the S splits.  The
-// CTA barrier orders every thread's partial stores before thread 0's gpu-scope fence, which
-// publishes them before the arrival (fences are cumulative); the last CTA fences again before
-// the barrier that lets its threads read the other splits' partials.
+// CTA barrier orders every thread's partial stores before thread 0's acquire-release bump,
+// which publishes them (release is cumulative) and, in the last CTA, acquires the other
+// splits' partials before the barrier that lets its threads read them.
 __device__ __forceinline__ bool arrive_last(const DecodeArgs& a, size_t bk, bool* s_flag) {
   __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    const bool last = atomicAdd(&a.cnt_head[bk], 1u) == (uint32_t)a.splits - 1u;
-    if (last) __threadfence();
-    *s_flag = last;
-  }
+  if (threadIdx.x == 0) *s_flag = atom_add_acq_rel_gpu(&a.cnt_head[bk], 1u) == (uint32_t)a.splits - 1u;
   __syncthreads();
   return *s_flag;
 }
@@ -82,12 +85,13 @@ template <typename T>
 __device__ __forceinline__ void combine_splits(const DecodeArgs& a, int b, int kv, float* /*scratch*/) {
   const int G = a.G, D = a.D, S = a.splits;
   const PartialView pv = partial_view(a);
-  const size_t bh0 = (size_t)b * a.Hq + (size_t)kv * G;
+  const size_t bk = (size_t)b * a.Hkv + kv;
+  const size_t bh0 = bk * G;
   const int D4 = D / 4;
   for (int i = threadIdx.x; i < G * D4; i += blockDim.x) {
     const int g = i / D4, d4 = i % D4;
-    const float4* op = reinterpret_cast<const float4*>(pv.o + (bh0 + g) * S * D) + d4;
-    const float2* mp = pv.ml + (bh0 + g) * S;
+    const float4* op = reinterpret_cast<const float4*>(pv.o(bk, g, 0)) + d4;
+    const float2* mp = pv.ml(bk, g, 0);
     float M = -INFINITY;
 #pragma unroll 8
     for (int t = 0; t < S; ++t) M = fmaxf(M, __ldcg(mp + t).x);
@@ -112,65 +116,6 @@ __device__ __forceinline__ void combine_splits(const DecodeArgs& a, int b, int k
   }
 }
 
-// combine_splits with one memory round trip: the partials of (b, kv) are copied into shared
-// memory (`scratch`, 16-byte aligned, `scratch_bytes` long) with every copy in flight at
-// once, then folded there in the same order and arithmetic as combine_splits.  Heads are
-// taken in groups that fit; when not even one head's S partials fit, combine_splits runs.
-template <typename T>
-__device__ __forceinline__ void combine_splits_staged(const DecodeArgs& a, int b, int kv, unsigned char* scratch,
-                                                      int scratch_bytes) {
-  const int G = a.G, D = a.D, S = a.splits;
-  const PartialView pv = partial_view(a);
-  const size_t bh0 = (size_t)b * a.Hq + (size_t)kv * G;
-  const int ml_bytes = (G * S * 8 + 15) & ~15;
-  const int head_bytes = S * D * 4;
-  const int gc = min(G, (scratch_bytes - ml_bytes) / head_bytes);
-  if (gc < 1) {
-    combine_splits<T>(a, b, kv, nullptr);
-    return;
-  }
-  float2* mls = reinterpret_cast<float2*>(scratch);            // [G][S]
-  float* os = reinterpret_cast<float*>(scratch + ml_bytes);     // [gc][S][D]
-  const int D4 = D / 4;
-  for (int gb = 0; gb < G; gb += gc) {
-    const int ng = min(gc, G - gb);
-    const float4* src = reinterpret_cast<const float4*>(pv.o + (bh0 + gb) * S * D);  // ng heads, contiguous
-    const uint32_t dst = smem_u32(os);
-    const int n16 = ng * S * D4;
-    for (int i = threadIdx.x; i < n16; i += blockDim.x) cp_async16_cg(dst + i * 16, src + i);
-    if (gb == 0)
-      for (int i = threadIdx.x; i < G * S; i += blockDim.x) mls[i] = __ldcg(pv.ml + bh0 * S + i);
-    cp_async_wait_all();
-    __syncthreads();
-    for (int i = threadIdx.x; i < ng * D4; i += blockDim.x) {
-      const int g = i / D4, d4 = i % D4;
-      const float2* mp = mls + (gb + g) * S;
-      const float4* op = reinterpret_cast<const float4*>(os + (size_t)g * S * D) + d4;
-      float M = -INFINITY;
-      for (int t = 0; t < S; ++t) M = fmaxf(M, mp[t].x);
-      float L = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (M != -INFINITY) {
-#pragma unroll 4
-        for (int t = 0; t < S; ++t) {
-          const float2 ml = mp[t];
-          const float4 v = op[t * D4];
-          const float w = exp2f(ml.x - M);
-          L = fmaf(ml.y, w, L);
-          acc.x = fmaf(v.x, w, acc.x);
-          acc.y = fmaf(v.y, w, acc.y);
-          acc.z = fmaf(v.z, w, acc.z);
-          acc.w = fmaf(v.w, w, acc.w);
-        }
-      }
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      const float r[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
-      store4(static_cast<T*>(a.out) + (bh0 + gb + g) * D + d4 * 4, r);
-    }
-    if (gb + gc < G) __syncthreads();
-  }
-}
-
 // Write the appended row (k_new, v_new) at row L of K_c / V_c with bias 0.  No CTA of this
 // launch reads row L (they read rows below L), so any one CTA may do it.
 template <typename T>
@@ -189,20 +134,22 @@ __device__ __forceinline__ void write_append_row(const DecodeArgs& a, size_t bk,
 }
 
 // Length bookkeeping of the last CTA of (b, kv), split in two so the atomic's round trip
-// overlaps the combine.  begin: reset the (b, kv) counter and count this head on the
-// sequence's counter; every CTA of the sequence has read lengths[b] before its own arrival,
-// so the last head to count may advance it.  end: that head writes lengths[b] = L + 1 (the
-// acquire on the counter keeps the write after the count).
-__device__ __forceinline__ uint32_t finish_lengths_begin(const DecodeArgs& a, int b, size_t bk, bool app) {
+// overlaps the combine; thread `owner` does both halves.  begin: reset the (b, kv) counter
+// and count this head on the sequence's counter; every CTA of the sequence has read
+// lengths[b] before its own arrival, so the last head to count may advance it.  end: that
+// head writes lengths[b] = L + 1 (the acquire on the counter keeps the write after the count).
+__device__ __forceinline__ uint32_t finish_lengths_begin(const DecodeArgs& a, int b, size_t bk, bool app,
+                                                         int owner = 0) {
   uint32_t old = 0u;
-  if (threadIdx.x == 0) {
+  if ((int)threadIdx.x == owner) {
     a.cnt_head[bk] = 0u;
     if (app) old = atom_add_acquire_gpu(&a.cnt_seq[b], 1u);
   }
   return old;
 }
-__device__ __forceinline__ void finish_lengths_end(const DecodeArgs& a, int b, int L, bool app, uint32_t old) {
-  if (threadIdx.x == 0 && app && old == (uint32_t)a.Hkv - 1u) {
+__device__ __forceinline__ void finish_lengths_end(const DecodeArgs& a, int b, int L, bool app, uint32_t old,
+                                                   int owner = 0) {
+  if ((int)threadIdx.x == owner && app && old == (uint32_t)a.Hkv - 1u) {
     a.lengths[b] = L + 1;
     a.cnt_seq[b] = 0u;
   }

@@ -127,7 +127,7 @@ __global__ __launch_bounds__(kWarps * 32) void decode_simt_kernel(DecodeArgs a) 
     for (int e = 0; e < PER; ++e) wo[warp][g][lane * PER + e] = o[g][e];
   }
   __syncthreads();
-  write_split_partial<kWarps>(a, b, kv, s, &wo[0][0][0], &wm[0][0], &wl[0][0], GM, false);
+  write_split_partial<kWarps>(a, b, kv, s, &wo[0][0][0], &wm[0][0], &wl[0][0], GM, D, false);
   if (!arrive_last(a, bk, &s_last)) return;
   combine_splits<T>(a, b, kv, &wo[0][0][0]);
   if (app) write_append_row<T>(a, bk, L, threadIdx.x, blockDim.x);

@@ -84,7 +84,8 @@ extern "C" SELKV_API selkv_status selkv_decode_attn_static(
   const size_t off_head = 256;
   const size_t off_seq = off_head + round256((size_t)s.batch * s.num_kv_heads * 4);
   const size_t off_part = off_seq + round256((size_t)s.batch * 4);
-  const size_t need = off_part + (size_t)s.batch * s.num_q_heads * splits * (s.head_dim + 2) * 4;
+  const size_t need = off_part + (size_t)s.batch * s.num_kv_heads *
+                                     decode_record_floats(s.num_q_heads / s.num_kv_heads, splits, s.head_dim) * 4;
   if (need > (size_t)SELKV_STATIC_SCRATCH_BYTES) return SELKV_ERR_WORKSPACE;
 
   void* base = nullptr;

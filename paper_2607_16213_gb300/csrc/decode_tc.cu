@@ -11,8 +11,8 @@
 // serves the whole group), the scale and the fp32 bias are applied to S before the running
 // max, then O += P V on the tensor cores.  The rows of one warp stream form one flash-decoding
 // state; the warp states and then the splits are folded in a fixed order, the splits by the
-// last CTA of (b, kv) to arrive (one atomic add, no waiting), which stages every split's
-// partial in the idle ring with one round of asynchronous copies.  The appended row
+// last CTA of (b, kv) to arrive (one atomic add, no waiting), which brings every split's
+// partial into the idle ring with one bulk copy.  The appended row
 // (k_new, v_new) joins the last split with bias 0 and is then written at row lengths[b].
 //
 // Every mbarrier wait is bounded: on timeout the CTA raises SELKV_DEVERR_TIMEOUT, stops, and
@@ -57,9 +57,166 @@ struct Cfg {
   static constexpr int kTileBytes = kTile * D * 2;     // K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + 2 * kStages * 8 + 64;
-  static_assert(kConsumers * 16 * D * 4 + kConsumers * 16 * 8 <= kRingBytes, "fold scratch fits");
+  // after the ring: full[kStages], empty[kStages], comb, abort flag (8 bytes), warp states
+  static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + (2 * kStages + 2) * 8 + 2 * kConsumers * 16 * 4;
+  static constexpr int kFoldLd = D + 8;                // fold row stride (floats): conflict-free float2 stores
+  static_assert(kConsumers * 16 * kFoldLd * 4 <= kRingBytes, "fold scratch fits");
 };
+
+// Combine of (b, kv) by its last CTA when S <= 32, with no shared memory and no barrier.
+// Two lanes own each output float4 (lanes l and l ^ 16: the first and the second half of the
+// splits); every partial they need is loaded into registers at once, next to the (max, sum)
+// of split `lane` of the item's head, so the whole combine costs one L2 round trip.  The
+// weights 2^(max_t - max) and the normaliser come from warp reductions and shuffles; each
+// lane sums its splits in split order and the two halves are added.  The producer warp's
+// lane 0 does the length bookkeeping.
+constexpr int kRegSplits = 32;
+template <int D>
+__device__ __forceinline__ void combine_registers(const DecodeArgs& a, int b, int kv, size_t bk, int L, bool app) {
+  constexpr int D4 = D / 4;
+  constexpr int kHalf = kRegSplits / 2;
+  static_assert(D4 % 16 == 0, "a warp's 16 items share one head");
+  const int G = a.G, S = a.splits;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nwarps = blockDim.x >> 5;
+  const int owner = blockDim.x - 32;
+  const PartialView pv = partial_view(a);
+  const uint32_t seq_old = finish_lengths_begin(a, b, bk, app, owner);
+  const int Sh = (S + 1) / 2;
+  const int half = lane >> 4;
+  const int t0 = half * Sh, cnt = min(S, t0 + Sh) - t0;
+  const int items = G * D4, per_pass = nwarps * 16;
+  for (int base = 0; base < items; base += per_pass) {
+    const int wbase = base + warp * 16;  // first item of this warp (uniform)
+    if (wbase >= items) break;
+    const int g = wbase / D4, d4 = wbase % D4 + (lane & 15);
+    const float4* op = reinterpret_cast<const float4*>(pv.o(bk, g, 0)) + d4;
+    float4 v[kHalf];
+#pragma unroll
+    for (int j = 0; j < kHalf; ++j)
+      v[j] = j < cnt ? __ldcg(op + (size_t)(t0 + j) * D4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float2 ml = lane < S ? __ldcg(pv.ml(bk, g, lane)) : make_float2(-INFINITY, 0.f);
+    const float M = warp_max(ml.x);
+    const float w = (lane < S && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
+    const float Ls = warp_sum(ml.y * w);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < kHalf; ++j) {
+      const float wj = __shfl_sync(0xffffffffu, w, (t0 + j) & 31);
+      if (j < cnt) {
+        acc.x = fmaf(v[j].x, wj, acc.x);
+        acc.y = fmaf(v[j].y, wj, acc.y);
+        acc.z = fmaf(v[j].z, wj, acc.z);
+        acc.w = fmaf(v[j].w, wj, acc.w);
+      }
+    }
+    const float ox = __shfl_xor_sync(0xffffffffu, acc.x, 16);
+    const float oy = __shfl_xor_sync(0xffffffffu, acc.y, 16);
+    const float oz = __shfl_xor_sync(0xffffffffu, acc.z, 16);
+    const float ow = __shfl_xor_sync(0xffffffffu, acc.w, 16);
+    if (half == 0) {
+      const float iv = Ls > 0.f ? 1.f / Ls : 0.f;
+      const float r[4] = {(acc.x + ox) * iv, (acc.y + oy) * iv, (acc.z + oz) * iv, (acc.w + ow) * iv};
+      store4(static_cast<__nv_bfloat16*>(a.out) + (bk * G + g) * D + d4 * 4, r);
+    }
+  }
+  finish_lengths_end(a, b, L, app, seq_old, owner);
+}
+
+// Combine of (b, kv) by its last CTA: one bulk copy brings the whole partial record (every
+// split's output and (max, sum)) into the idle ring; a warp per head turns the maxima into
+// weights 2^(max_t - max) and the normaliser; each output float4 is then summed over the
+// splits by two lanes (first and second half of the splits, in split order) and the halves
+// added.  The producer warp's lane 0, which issues no loads here, does the length
+// bookkeeping.  A record too large for the ring falls back to combine_splits.
+template <int D>
+__device__ __forceinline__ void combine_record(const DecodeArgs& a, int b, int kv, size_t bk, unsigned char* smem,
+                                               int smem_bytes, uint64_t* bar, int L, bool app) {
+  constexpr int D4 = D / 4;
+  const int G = a.G, S = a.splits;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nwarps = blockDim.x >> 5;
+  const int owner = blockDim.x - 32;
+  const PartialView pv = partial_view(a);
+  const uint32_t rec_bytes = (uint32_t)(pv.rec * 4);
+  if ((size_t)rec_bytes + (size_t)G * (S + 1) * 4 > (size_t)smem_bytes) {
+    const uint32_t old = finish_lengths_begin(a, b, bk, app, owner);
+    combine_splits<__nv_bfloat16>(a, b, kv, nullptr);
+    finish_lengths_end(a, b, L, app, old, owner);
+    return;
+  }
+  // the ring was last touched through the generic proxy; the bulk copy writes it through the
+  // async proxy, and reads the other splits' generic-proxy stores acquired by arrive_last
+  fence_proxy_async_all();
+  __syncthreads();
+  if (tid == 0) {
+    mbar_arrive_expect_tx(bar, rec_bytes);
+    bulk_load(smem, pv.record(bk), rec_bytes, bar);
+  }
+  const uint32_t seq_old = finish_lengths_begin(a, b, bk, app, owner);
+  const float* os = reinterpret_cast<const float*>(smem);                              // [G][S][D]
+  const float2* mls = reinterpret_cast<const float2*>(smem + (size_t)G * S * D * 4);   // [G][S]
+  float* wts = reinterpret_cast<float*>(smem + rec_bytes);                              // [G][S]
+  float* inv = wts + G * S;                                                             // [G]
+  if (!mbar_wait(bar, 0)) {
+    if (tid == 0) raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+    mbar_wait(bar, 0);  // the copy must land before the CTA leaves
+    return;
+  }
+  for (int g = warp; g < G; g += nwarps) {
+    float M = -INFINITY;
+    for (int t = lane; t < S; t += 32) M = fmaxf(M, mls[g * S + t].x);
+    M = warp_max(M);
+    float Ls = 0.f;
+    for (int t = lane; t < S; t += 32) {
+      const float2 ml = mls[g * S + t];
+      const float w = M == -INFINITY ? 0.f : exp2f(ml.x - M);
+      wts[g * S + t] = w;
+      Ls = fmaf(ml.y, w, Ls);
+    }
+    Ls = warp_sum(Ls);
+    if (lane == 0) inv[g] = Ls > 0.f ? 1.f / Ls : 0.f;
+  }
+  __syncthreads();
+  const int Sh = (S + 1) / 2;
+  const int items = G * D4, per_pass = nwarps * 16;
+  for (int base = 0; base < items; base += per_pass) {
+    const int item = base + warp * 16 + (lane & 15);
+    const int half = lane >> 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    const int g = item / D4, d4 = item % D4;
+    if (item < items) {
+      const int t0 = half * Sh, t1 = min(S, t0 + Sh);
+      const float4* op = reinterpret_cast<const float4*>(os + (size_t)g * S * D) + d4;
+      const float* wp = wts + g * S;
+      for (int t = t0; t < t1; t += 8) {
+        float4 v[8];
+        float w[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const bool ok = t + j < t1;
+          v[j] = ok ? op[(t + j) * D4] : make_float4(0.f, 0.f, 0.f, 0.f);
+          w[j] = ok ? wp[t + j] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          acc.x = fmaf(v[j].x, w[j], acc.x);
+          acc.y = fmaf(v[j].y, w[j], acc.y);
+          acc.z = fmaf(v[j].z, w[j], acc.z);
+          acc.w = fmaf(v[j].w, w[j], acc.w);
+        }
+      }
+    }
+    const float ox = __shfl_xor_sync(0xffffffffu, acc.x, 16);
+    const float oy = __shfl_xor_sync(0xffffffffu, acc.y, 16);
+    const float oz = __shfl_xor_sync(0xffffffffu, acc.z, 16);
+    const float ow = __shfl_xor_sync(0xffffffffu, acc.w, 16);
+    if (item < items && half == 0) {
+      const float iv = inv[g];
+      const float r[4] = {(acc.x + ox) * iv, (acc.y + oy) * iv, (acc.z + oz) * iv, (acc.w + ow) * iv};
+      store4(static_cast<__nv_bfloat16*>(a.out) + (bk * G + g) * D + d4 * 4, r);
+    }
+  }
+  finish_lengths_end(a, b, L, app, seq_old, owner);
+}
 
 template <int D, bool ROWS16>
 __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -73,7 +230,10 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kRingBytes);
   uint64_t* empty = full + kStages;
-  volatile int* s_abort = reinterpret_cast<volatile int*>(empty + kStages);
+  uint64_t* comb = empty + kStages;  // completion of the combine's bulk copy
+  volatile int* s_abort = reinterpret_cast<volatile int*>(comb + 1);
+  float* wm = reinterpret_cast<float*>(comb + 2);  // [kConsumers][16] warp maxima (base 2)
+  float* wl = wm + kConsumers * 16;                // [kConsumers][16] warp sums
   __shared__ bool s_last;
 
   const int s = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
@@ -86,6 +246,7 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], kConsumers);
     }
+    mbar_init(comb, 1);
     *s_abort = 0;
     fence_mbar_init();
   }
@@ -316,33 +477,69 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
     }
   }
+  // Fold the warp states into this split's partial.  The warps' (max, sum) live outside the
+  // ring, so one barrier both drains the ring and publishes them; each warp then scales its
+  // own output by 2^(m_w - max) while storing it, and the partial output is the sum over
+  // the warps in warp order.  An aborted CTA leaves an empty partial.
+  if (warp < kConsumers && (lane & 3) == 0) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int g = g0 + r * 8;
+      if (g >= G) continue;
+      wm[warp * 16 + g] = mrow[r];
+      wl[warp * 16 + g] = lrow[r];
+    }
+  }
   __syncthreads();  // the ring is idle (drained) from here on: reuse it for the fold
-
-  float* wo = reinterpret_cast<float*>(smem);                  // [kConsumers][16][D]
-  float* wm = wo + kConsumers * 16 * D;                         // [kConsumers][16]
-  float* wl = wm + kConsumers * 16;                             // [kConsumers][16]
+  const bool aborted = *s_abort != 0;
+  const PartialView pv = partial_view(a);
+  float* wo = reinterpret_cast<float*>(smem);  // [kConsumers][16][kFoldLd], scaled outputs
   if (warp < kConsumers) {
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int g = g0 + r * 8;
       if (g >= G) continue;
+      float M = -INFINITY;
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        wo[(warp * 16 + g) * D + nt * 8 + c2] = o[nt][r * 2];
-        wo[(warp * 16 + g) * D + nt * 8 + c2 + 1] = o[nt][r * 2 + 1];
-      }
-      if ((lane & 3) == 0) {
-        wm[warp * 16 + g] = mrow[r];
-        wl[warp * 16 + g] = lrow[r];
+      for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, wm[w * 16 + g]);
+      const float f = M == -INFINITY ? 0.f : exp2f(mrow[r] - M);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+        *reinterpret_cast<float2*>(wo + (warp * 16 + g) * C::kFoldLd + nt * 8 + c2) =
+            make_float2(o[nt][r * 2] * f, o[nt][r * 2 + 1] * f);
+      if (warp == 0 && (lane & 3) == 0) {
+        float Ls = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+          for (int w = 0; w < kConsumers; ++w) Ls = fmaf(wl[w * 16 + g], exp2f(wm[w * 16 + g] - M), Ls);
+        }
+        *pv.ml(bk, g, s) = aborted ? make_float2(-INFINITY, 0.f) : make_float2(M, Ls);
       }
     }
   }
   __syncthreads();
-  write_split_partial<kConsumers>(a, b, kv, s, wo, wm, wl, 16, *s_abort != 0);
+  {
+    constexpr int D4 = D / 4;
+    for (int i = tid; i < G * D4; i += blockDim.x) {
+      const int g = i / D4, d4 = i % D4;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int w = 0; w < kConsumers; ++w) {
+        const float4 v = *reinterpret_cast<const float4*>(wo + (w * 16 + g) * C::kFoldLd + d4 * 4);
+        acc.x += v.x;
+        acc.y += v.y;
+        acc.z += v.z;
+        acc.w += v.w;
+      }
+      if (aborted) acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      reinterpret_cast<float4*>(pv.o(bk, g, s))[d4] = acc;
+    }
+  }
   if (!arrive_last(a, bk, &s_last)) return;
-  const uint32_t seq_old = finish_lengths_begin(a, b, bk, app);
-  combine_splits_staged<__nv_bfloat16>(a, b, kv, smem, C::kRingBytes);
-  finish_lengths_end(a, b, L, app, seq_old);
+  if (S <= kRegSplits)
+    combine_registers<D>(a, b, kv, bk, L, app);
+  else
+    combine_record<D>(a, b, kv, bk, smem, C::kRingBytes, comb, L, app);
 }
 
 template <int D, bool R16>

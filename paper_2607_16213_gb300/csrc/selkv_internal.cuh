@@ -173,8 +173,15 @@ struct DecodeArgs {
   uint32_t* flags;
   uint32_t* cnt_head;  // [B][Hkv] arrivals per (b, kv) (self-resetting)
   uint32_t* cnt_seq;   // [B] (b, kv) completions per sequence (self-resetting)
-  float* partial;      // [B][Hq][splits][D + 2]
+  float* partial;      // [B][Hkv] records of decode_record_floats(G, splits, D) floats
 };
+
+// Floats of one (sequence, KV head) record of split partials: the unnormalised outputs
+// o [G][S][D], then the (max in base 2, sum) pairs [G][S] padded to a 16-byte multiple, so
+// every record starts 16-byte aligned and can be moved with one bulk copy.
+__host__ __device__ constexpr size_t decode_record_floats(int G, int S, int D) {
+  return (size_t)G * S * D + (((size_t)G * S * 2 + 3) & ~(size_t)3);
+}
 
 int decode_splits(int B, int Hkv, int m_cap, int num_sms);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);     // dispatch by dtype
