@@ -15,7 +15,7 @@ namespace {
 
 // Kernels enqueued by each call (diagnostic count, see selkv_kernel_launches).
 std::atomic<uint64_t> g_launches{0};
-constexpr int kCompressKernels = 15;  // with the tensor-core scoring (17 with the CUDA-core one)
+constexpr int kCompressKernels = 18;  // with the tensor-core scoring (20 with the CUDA-core one)
 constexpr int kDecodeKernels = 1;
 // SM count used for planning the decode split: fixed, so that workspace sizes do not depend
 // on which device answers (GB300: 152 SMs).
@@ -37,7 +37,7 @@ bool shape_ok(const selkv_shape* s) {
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, kflag, slot, select, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
   int nchunks, R;
 };
 
@@ -62,6 +62,11 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.score = take(B * Hkv * n * 4);
   p.kflag = take(B * n);
   p.slot = take(B * n * 4);
+  p.kept_pos = take(B * (size_t)s.m_cap * 4);
+  // merge targets per bucket, sized for the smallest bucket (the size is a call parameter)
+  p.tau = take(B * Hkv * n * 4);
+  p.atau = take(B * Hkv * n * 4);
+  p.ratio = take(B * Hkv * (size_t)s.m_cap * 4);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
   p.total = off;
   return p;
@@ -220,6 +225,11 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.score = (debug && debug->score) ? debug->score : at<float>(workspace, plan.score);
   a.kflag = at<uint8_t>(workspace, plan.kflag);
   a.slot_of = at<int32_t>(workspace, plan.slot);
+  a.kept_pos = at<int32_t>(workspace, plan.kept_pos);
+  a.nbk = (s.n_cap + p.bucket - 1) / p.bucket;
+  a.tau = at<int32_t>(workspace, plan.tau);
+  a.atau = at<float>(workspace, plan.atau);
+  a.ratio = at<float>(workspace, plan.ratio);
   if (debug != nullptr) {
     a.dbg_topk = debug->topk;
     a.dbg_kept_idx = debug->kept_idx;

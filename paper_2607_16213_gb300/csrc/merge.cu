@@ -1,16 +1,22 @@
 // Bucket-attention routing, soft cosine gate, gated merge, attention ratio and the
 // compressed-cache write-out of SelKV (Eq. 3-6, Sec. 3.6 GQA bias).
 //
-// One CTA per (bucket X, sequence b) with one warp per KV head.  Under Eq. 3 (argmax over the
-// kept tokens of the bucket of the cumulative attention a) every evicted token of a bucket
-// routes to the same kept token tau_X, so the merge is a gather: the CTA of a non-empty bucket
-// X collects, in ascending position order, the evicted tokens of X and of the empty buckets
-// whose nearest non-empty ring resolves to X, accumulates
-//     num = sum g_j a_j v_j,   den = sum g_j a_j,   g_j = clamp(cos(v_j, v_tau), 0, 1),
-// and writes v~_tau = (a_tau v_tau + num) / (a_tau + den), R_tau = (a_tau + den) / a_tau.
-// Every kept token of X is copied to its slot of K_c / V_c (keys unchanged), and
-// bias = alpha * ln(mean over KV heads of R) is written once all warps have their R.
-// No floating-point atomics: the summation order is fixed, so results are reproducible.
+// Under Eq. 3 (argmax over the kept tokens of a bucket of the cumulative attention a) every
+// evicted token of a bucket routes to the same kept token tau_X, so the merge is a gather.
+// Four kernels, in stream order:
+//   route  warp per (bucket X, sequence b): tau_X and a(tau_X) for every KV head (-1 / -inf
+//          for a bucket with no kept token);
+//   copy   every kept token's key and value row to its slot of K_c / V_c (keys unchanged) and
+//          ratio 1 for the slot; a thread per 16 bytes, coalesced;
+//   merge  warp per (non-empty bucket X, KV head, sequence b): the evicted tokens of X and of
+//          the empty buckets that the nearest-ring rule gives to X, in ascending position
+//          order, 16 at a time: g_j = clamp(cos(v_j, v_tau), 0, 1) and
+//              v~_tau = (a_tau v_tau + sum g_j a_j v_j) / (a_tau + sum g_j a_j),
+//              R_tau  = (a_tau + sum g_j a_j) / a_tau,
+//          written over tau's slot;
+//   bias   bias = alpha * ln(mean over KV heads of R) for every slot (the same row for every
+//          KV head).
+// No floating-point atomics: every sum has a fixed order, so results are reproducible.
 #include <climits>
 
 #include "selkv_internal.cuh"
@@ -18,37 +24,176 @@
 namespace selkv {
 namespace {
 
-template <typename T, int D, int MAXT>
-__global__ __launch_bounds__(MAXT) void merge_kernel(CompressArgs a) {
-  constexpr int PER = D / 32;  // elements of a row per lane
-  __shared__ float Rs[32][33];
-  const int X = blockIdx.x, b = blockIdx.y;
-  const int kv = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = a.seq_n[b];
-  const int Bs = a.bucket;
+constexpr int kWarpsPerCta = 8;
+constexpr int kBatch = 16;  // contributors per merge batch
+
+// argmax over the lanes of (value, position): larger value, then lower position
+__device__ __forceinline__ void argmax_lanes(float& v, int& idx) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float v2 = __shfl_xor_sync(0xffffffffu, v, o);
+    const int i2 = __shfl_xor_sync(0xffffffffu, idx, o);
+    if (v2 > v || (v2 == v && i2 < idx)) {
+      v = v2;
+      idx = i2;
+    }
+  }
+}
+
+__global__ __launch_bounds__(kWarpsPerCta * 32) void route_kernel(CompressArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int X = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5), b = blockIdx.y;
+  const int n = a.seq_n[b], Bs = a.bucket;
   const int nb = (n + Bs - 1) / Bs;
   if (X >= nb) return;
-  const uint8_t* kf = a.kflag + (size_t)b * a.n_cap;
-  auto bucket_mask = [&](int e) -> uint32_t {
-    const int p = e * Bs + lane;
-    const bool k = lane < Bs && p < n && kf[p] != 0;
-    return __ballot_sync(0xffffffffu, k);
-  };
+  const int p = X * Bs + lane;
+  const bool kept = lane < Bs && p < n && a.kflag[(size_t)b * a.n_cap + p] != 0;
+  for (int kv = 0; kv < a.Hkv; ++kv) {
+    const size_t bk = (size_t)b * a.Hkv + kv;
+    float v = kept ? a.attn[bk * a.n_cap + p] : -INFINITY;
+    int idx = kept ? p : INT_MAX;
+    argmax_lanes(v, idx);
+    if (lane == 0) {
+      a.tau[bk * a.nbk + X] = idx == INT_MAX ? -1 : idx;
+      a.atau[bk * a.nbk + X] = v;
+    }
+  }
+}
+
+// One thread per 16 bytes of a kept row: the K and V rows of slot s of (b, kv).
+template <typename T, int D>
+__global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
+  constexpr int kPieces = D * (int)sizeof(T) / 16;  // 16-byte pieces per row
+  const int b = blockIdx.y;
+  const int m = a.seq_m[b];
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int piece = (int)(i % kPieces);
+  const size_t row = i / kPieces;  // over (kv, slot, tensor)
+  const int tensor = (int)(row & 1);
+  const size_t ks = row >> 1;
+  const int slot = (int)(ks % a.m_cap);
+  const int kv = (int)(ks / a.m_cap);
+  if (kv >= a.Hkv || slot >= m) return;
+  const int pos = a.kept_pos[(size_t)b * a.m_cap + slot];
   const size_t bk = (size_t)b * a.Hkv + kv;
-  const float* A = a.attn + bk * a.n_cap;
-  const float* vn = a.vnorm + bk * a.n_cap;
-  const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
+  if (pos < 0 || pos >= a.n_cap) {
+    if (piece == 0 && tensor == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
+    return;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(static_cast<const T*>(tensor ? a.V : a.K) + (bk * a.n_cap + pos) * D);
+  uint4* dst = reinterpret_cast<uint4*>(static_cast<T*>(tensor ? a.Vc : a.Kc) + (bk * a.m_cap + slot) * D);
+  dst[piece] = src[piece];
+  if (piece == 0 && tensor == 0) {
+    a.ratio[bk * a.m_cap + slot] = 1.f;
+    if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = 1.f;
+    const size_t o = bk * a.n_cap + pos;
+    if (a.dbg_target) a.dbg_target[o] = -1;
+    if (a.dbg_gate) a.dbg_gate[o] = 0.f;
+    if (a.dbg_decision) a.dbg_decision[o] = 2;
+  }
+}
+
+// One lane's PER consecutive elements of a row, kept in the storage type.
+template <typename T, int PER>
+struct RowSlice;
+template <>
+struct RowSlice<__nv_bfloat16, 4> {
+  uint2 w;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint2*>(p); }
+  __device__ __forceinline__ void zero() { w = make_uint2(0u, 0u); }
+  __device__ __forceinline__ float operator[](int e) const {
+    const uint32_t x = e < 2 ? w.x : w.y;
+    return (e & 1) ? bf16_hi(x) : bf16_lo(x);
+  }
+};
+template <>
+struct RowSlice<__nv_bfloat16, 2> {
+  uint32_t w;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint32_t*>(p); }
+  __device__ __forceinline__ void zero() { w = 0u; }
+  __device__ __forceinline__ float operator[](int e) const { return (e & 1) ? bf16_hi(w) : bf16_lo(w); }
+};
+template <int PER>
+struct RowSlice<float, PER> {
+  float x[PER];
+  __device__ __forceinline__ void load(const float* p) {
+    if constexpr (PER == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(p);
+      x[0] = v.x;
+      x[1] = v.y;
+      x[2] = v.z;
+      x[3] = v.w;
+    } else {
+      const float2 v = *reinterpret_cast<const float2*>(p);
+      x[0] = v.x;
+      x[1] = v.y;
+    }
+  }
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int e = 0; e < PER; ++e) x[e] = 0.f;
+  }
+  __device__ __forceinline__ float operator[](int e) const { return x[e]; }
+};
+
+// Sum kBatch per-lane partials p[k] over the 32 lanes with the batch spread over the lanes:
+// each butterfly level keeps half of the values and adds the partner's copy of them, so lanes
+// 2k and 2k + 1 end with the full sum of value k.  The pairs added at each level are those
+// of a plain xor butterfly over all 32 lanes, so every sum is bitwise that of a per-value
+// all-reduce.
+__device__ __forceinline__ float transpose_reduce16(const float (&p)[kBatch], int lane) {
+  float q[8];
+  {
+    const bool up = lane & 16;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float mine = up ? p[8 + i] : p[i], other = up ? p[i] : p[8 + i];
+      q[i] = mine + __shfl_xor_sync(0xffffffffu, other, 16);
+    }
+  }
+  float r[4];
+  {
+    const bool up = lane & 8;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float mine = up ? q[4 + i] : q[i], other = up ? q[i] : q[4 + i];
+      r[i] = mine + __shfl_xor_sync(0xffffffffu, other, 8);
+    }
+  }
+  float s[2];
+  {
+    const bool up = lane & 4;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const float mine = up ? r[2 + i] : r[i], other = up ? r[i] : r[2 + i];
+      s[i] = mine + __shfl_xor_sync(0xffffffffu, other, 4);
+    }
+  }
+  const bool up = lane & 2;
+  const float mine = up ? s[1] : s[0], other = up ? s[0] : s[1];
+  const float t = mine + __shfl_xor_sync(0xffffffffu, other, 2);
+  return t + __shfl_xor_sync(0xffffffffu, t, 1);
+}
+
+template <typename T, int D>
+__global__ __launch_bounds__(kWarpsPerCta * 32) void merge_kernel(CompressArgs a) {
+  constexpr int PER = D / 32;  // elements of a row per lane
+  const int lane = threadIdx.x & 31;
+  const int X = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+  const int kv = blockIdx.y % a.Hkv, b = blockIdx.y / a.Hkv;
+  const int n = a.seq_n[b], Bs = a.bucket;
+  const int nb = (n + Bs - 1) / Bs;
+  if (X >= nb) return;
+  const size_t bk = (size_t)b * a.Hkv + kv;
+  const int32_t* tau_of = a.tau + bk * a.nbk;
+  const int tau = tau_of[X];
   const int base = X * Bs;
-  const int cntX = min(Bs, n - base);
-  // this lane's position of bucket X: a and ||v||, fetched together with the kept flags
-  const float A_l = lane < cntX ? A[base + lane] : -INFINITY;
-  const float vn_l = lane < cntX ? vn[base + lane] : 0.f;
-  const uint32_t mX = bucket_mask(X);
-  if (mX == 0u) {
-    // Empty bucket: under EXPAND a neighbour's CTA owns these tokens; under DROP (or with
+  const uint8_t* kf = a.kflag + (size_t)b * a.n_cap;
+  if (tau < 0) {
+    // Empty bucket: under EXPAND a neighbour's warp owns these tokens; under DROP (or with
     // nothing kept at all) they stay without target.
     if (a.empty_bucket == SELKV_EMPTY_DROP || a.seq_m[b] == 0) {
-      if (lane < cntX) {
+      if (lane < min(Bs, n - base)) {
         const size_t o = bk * a.n_cap + base + lane;
         if (a.dbg_target) a.dbg_target[o] = -1;
         if (a.dbg_gate) a.dbg_gate[o] = 0.f;
@@ -57,124 +202,114 @@ __global__ __launch_bounds__(MAXT) void merge_kernel(CompressArgs a) {
     }
     return;
   }
-  // argmax of a over the kept tokens of a bucket (larger a, then lower position).
-  auto best_of = [&](float v, int idx) -> int {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float v2 = __shfl_xor_sync(0xffffffffu, v, o);
-      const int i2 = __shfl_xor_sync(0xffffffffu, idx, o);
-      if (v2 > v || (v2 == v && i2 < idx)) { v = v2; idx = i2; }
-    }
-    return idx;
-  };
-  auto best_in = [&](int e, uint32_t mask) -> int {
-    const bool in = (mask >> lane) & 1u;
-    return best_of(in ? A[e * Bs + lane] : -INFINITY, in ? e * Bs + lane : INT_MAX);
-  };
-  const bool inX = (mX >> lane) & 1u;
-  const int tau = best_of(inX ? A_l : -INFINITY, inX ? base + lane : INT_MAX);
-  const float a_tau = __shfl_sync(0xffffffffu, A_l, tau - base);
-  const float vn_tau = __shfl_sync(0xffffffffu, vn_l, tau - base);
+  const float* A = a.attn + bk * a.n_cap;
+  const float* vn = a.vnorm + bk * a.n_cap;
+  const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
+  const float a_tau = a.atau[bk * a.nbk + X];
+  const float vn_tau = vn[tau];
+  RowSlice<T, PER> vt;
+  vt.load(Vb + (size_t)tau * D + lane * PER);
+
   int lo_b = X, hi_b = X;  // buckets whose evicted tokens route to tau
   if (a.empty_bucket == SELKV_EMPTY_EXPAND) {
-    int L = X - 1;
-    uint32_t mL = 0u;
-    while (L >= 0 && (mL = bucket_mask(L)) == 0u) --L;
+    // nearest non-empty buckets L < X and R > X, probing 32 buckets at a time
+    int L = -1;
+    for (int e0 = X - 1; e0 >= 0 && L < 0; e0 -= 32) {
+      const int e = e0 - lane;
+      const uint32_t m = __ballot_sync(0xffffffffu, e >= 0 && tau_of[e] >= 0);
+      if (m) L = e0 - (__ffs(m) - 1);
+    }
+    int R = -1;
+    for (int e0 = X + 1; e0 < nb && R < 0; e0 += 32) {
+      const int e = e0 + lane;
+      const uint32_t m = __ballot_sync(0xffffffffu, e < nb && tau_of[e] >= 0);
+      if (m) R = e0 + (__ffs(m) - 1);
+    }
+    // An empty e between L and X goes to the nearer one; at equal distance both are in the
+    // ring and X wins only with a strictly larger a (tau_L has the lower index).  Towards R,
+    // X wins ties at equal distance (tau_X has the lower index).
     if (L < 0) {
       lo_b = 0;
     } else if (L < X - 1) {
-      // empty e in (L, X): X is nearer iff X - e < e - L; at equal distance the ring holds
-      // both buckets and X wins only with a strictly larger a (tau_L has the lower index).
       lo_b = (X + L) / 2 + 1;
-      if (((X + L) & 1) == 0 && a_tau > A[best_in(L, mL)]) lo_b = (X + L) / 2;
+      if (((X + L) & 1) == 0 && a_tau > a.atau[bk * a.nbk + L]) lo_b = (X + L) / 2;
     }
-    int Rb = X + 1;
-    uint32_t mR = 0u;
-    while (Rb < nb && (mR = bucket_mask(Rb)) == 0u) ++Rb;
-    if (Rb >= nb) {
+    if (R < 0) {
       hi_b = nb - 1;
-    } else if (Rb > X + 1) {
-      hi_b = (X + Rb - 1) / 2;
-      if (((X + Rb) & 1) == 0 && a_tau >= A[best_in(Rb, mR)]) hi_b = (X + Rb) / 2;
+    } else if (R > X + 1) {
+      hi_b = (X + R - 1) / 2;
+      if (((X + R) & 1) == 0 && a_tau >= a.atau[bk * a.nbk + R]) hi_b = (X + R) / 2;
     }
   }
-  float vt[PER];
-  if constexpr (PER == 4) load4(Vb + (size_t)tau * D + lane * 4, vt); else load2(Vb + (size_t)tau * D + lane * 2, vt);
 
   float num[PER];
 #pragma unroll
   for (int e = 0; e < PER; ++e) num[e] = 0.f;
   float den = 0.f;
-  // Contributors in ascending position order, a batch at a time: their loads are independent
-  // and their dot-product reductions interleave (the sums stay in position order).
-  constexpr int kBatch = MAXT <= 256 ? 8 : 4;
+  const int own = lane >> 1;  // contributor owned by this lane pair within a batch
   for (int e = lo_b; e <= hi_b; ++e) {
     const int eb = e * Bs;
-    const int cnt_e = min(Bs, n - eb);
-    const uint32_t valid = cnt_e >= 32 ? 0xffffffffu : ((1u << cnt_e) - 1u);
-    const bool own = e == X;
-    uint32_t rem = valid & ~(own ? mX : 0u);
+    const bool in_e = lane < min(Bs, n - eb);
+    uint32_t rem = __ballot_sync(0xffffffffu, in_e && kf[eb + lane] == 0);
     // a and ||v|| of bucket e, one position per lane
-    const float Ae = own ? A_l : (lane < cnt_e ? A[eb + lane] : 0.f);
-    const float Ne = own ? vn_l : (lane < cnt_e ? vn[eb + lane] : 0.f);
+    const float Ae = in_e ? A[eb + lane] : 0.f;
+    const float Ne = in_e ? vn[eb + lane] : 0.f;
     while (rem) {
-      int pos[kBatch];
-      int nb_ = 0;
+      // the next (up to) kBatch contributors, in position order
+      int bit[kBatch];
+      int cnt = 0;
 #pragma unroll
       for (int k = 0; k < kBatch; ++k) {
-        pos[k] = -1;
+        bit[k] = -1;
         if (rem) {
-          pos[k] = eb + __ffs(rem) - 1;
+          bit[k] = __ffs(rem) - 1;
           rem &= rem - 1u;
-          ++nb_;
+          ++cnt;
         }
       }
-      float vj[kBatch][PER];
-      float dot[kBatch];
+      RowSlice<T, PER> vj[kBatch];
 #pragma unroll
       for (int k = 0; k < kBatch; ++k) {
-        if (pos[k] >= 0) {
-          if constexpr (PER == 4) load4(Vb + (size_t)pos[k] * D + lane * 4, vj[k]);
-          else load2(Vb + (size_t)pos[k] * D + lane * 2, vj[k]);
-        } else {
-#pragma unroll
-          for (int t = 0; t < PER; ++t) vj[k][t] = 0.f;
-        }
-        dot[k] = 0.f;
-#pragma unroll
-        for (int t = 0; t < PER; ++t) dot[k] = fmaf(vj[k][t], vt[t], dot[k]);
+        if (bit[k] >= 0) vj[k].load(Vb + (size_t)(eb + bit[k]) * D + lane * PER);
+        else vj[k].zero();
       }
-      if (a.gate_mode == SELKV_GATE_COSINE) {
+      int ob = -1;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
+      for (int k = 0; k < kBatch; ++k)
+        if (k == own) ob = bit[k];
+      const float ak = __shfl_sync(0xffffffffu, Ae, ob < 0 ? 0 : ob);
+      const float nk = __shfl_sync(0xffffffffu, Ne, ob < 0 ? 0 : ob);
+      float g;
+      if (a.gate_mode == SELKV_GATE_OPEN) {
+        g = 1.f;
+      } else if (a.gate_mode == SELKV_GATE_CLOSED) {
+        g = 0.f;
+      } else {
+        float part[kBatch];
 #pragma unroll
-          for (int k = 0; k < kBatch; ++k) dot[k] += __shfl_xor_sync(0xffffffffu, dot[k], o);
+        for (int k = 0; k < kBatch; ++k) {
+          part[k] = 0.f;
+#pragma unroll
+          for (int t = 0; t < PER; ++t) part[k] = fmaf(vj[k][t], vt[t], part[k]);
+        }
+        const float dot = transpose_reduce16(part, lane);
+        const float sim = (nk == 0.f || vn_tau == 0.f) ? 0.f : dot / (nk * vn_tau);
+        g = fminf(fmaxf(sim, 0.f), 1.f);
+      }
+      const float w = ob >= 0 ? g * ak : 0.f;
+      if (ob >= 0 && (lane & 1) == 0) {
+        const size_t o = bk * a.n_cap + eb + ob;
+        if (a.dbg_target) a.dbg_target[o] = tau;
+        if (a.dbg_gate) a.dbg_gate[o] = g;
+        if (a.dbg_decision) a.dbg_decision[o] = g > 0.f ? 1 : 0;
       }
 #pragma unroll
       for (int k = 0; k < kBatch; ++k) {
-        if (k >= nb_) break;
-        const int src = pos[k] - eb;
-        const float ak = __shfl_sync(0xffffffffu, Ae, src);
-        const float nk = __shfl_sync(0xffffffffu, Ne, src);
-        float g;
-        if (a.gate_mode == SELKV_GATE_OPEN) {
-          g = 1.f;
-        } else if (a.gate_mode == SELKV_GATE_CLOSED) {
-          g = 0.f;
-        } else {
-          const float sim = (nk == 0.f || vn_tau == 0.f) ? 0.f : dot[k] / (nk * vn_tau);
-          g = fminf(fmaxf(sim, 0.f), 1.f);
-        }
-        const float w = g * ak;
+        if (k >= cnt) break;
+        const float wk = __shfl_sync(0xffffffffu, w, 2 * k);
 #pragma unroll
-        for (int t = 0; t < PER; ++t) num[t] = fmaf(w, vj[k][t], num[t]);
-        den += w;
-        if (lane == k) {
-          const size_t o = bk * a.n_cap + pos[k];
-          if (a.dbg_target) a.dbg_target[o] = tau;
-          if (a.dbg_gate) a.dbg_gate[o] = g;
-          if (a.dbg_decision) a.dbg_decision[o] = g > 0.f ? 1 : 0;
-        }
+        for (int t = 0; t < PER; ++t) num[t] = fmaf(wk, vj[k][t], num[t]);
+        den += wk;
       }
     }
   }
@@ -183,103 +318,55 @@ __global__ __launch_bounds__(MAXT) void merge_kernel(CompressArgs a) {
 #pragma unroll
   for (int t = 0; t < PER; ++t) vm[t] = tot > 0.f ? (a_tau * vt[t] + num[t]) / tot : vt[t];
   const float R_tau = a_tau > 0.f ? tot / a_tau : 1.f;
-
-  // Kept tokens of X, four at a time (loads first, then stores).
-  const T* Kb = static_cast<const T*>(a.K) + bk * a.n_cap * D;
-  T* Kc = static_cast<T*>(a.Kc) + bk * a.m_cap * D;
-  T* Vc = static_cast<T*>(a.Vc) + bk * a.m_cap * D;
-  const int32_t* so = a.slot_of + (size_t)b * a.n_cap;
-  uint32_t rem = mX;
-  while (rem) {
-    constexpr int kCopy = 4;
-    int tk[kCopy], sl[kCopy];
-#pragma unroll
-    for (int k = 0; k < kCopy; ++k) {
-      tk[k] = -1;
-      sl[k] = -1;
-      if (rem) {
-        tk[k] = __ffs(rem) - 1;
-        rem &= rem - 1u;
-        sl[k] = so[base + tk[k]];
-        if (sl[k] < 0 || sl[k] >= a.m_cap) {
-          if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
-          sl[k] = -1;
-        }
-      }
-    }
-    float kx[kCopy][PER], vx[kCopy][PER];
-#pragma unroll
-    for (int k = 0; k < kCopy; ++k) {
-      if (sl[k] < 0) continue;
-      const int p = base + tk[k];
-      if constexpr (PER == 4) {
-        load4(Kb + (size_t)p * D + lane * 4, kx[k]);
-        if (p != tau) load4(Vb + (size_t)p * D + lane * 4, vx[k]);
-      } else {
-        load2(Kb + (size_t)p * D + lane * 2, kx[k]);
-        if (p != tau) load2(Vb + (size_t)p * D + lane * 2, vx[k]);
-      }
-      if (p == tau) {
-#pragma unroll
-        for (int e = 0; e < PER; ++e) vx[k][e] = vm[e];
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < kCopy; ++k) {
-      if (sl[k] < 0) continue;
-      const int p = base + tk[k];
-      const int slot = sl[k];
-      if constexpr (PER == 4) {
-        store4(Kc + (size_t)slot * D + lane * 4, kx[k]);
-        store4(Vc + (size_t)slot * D + lane * 4, vx[k]);
-      } else {
-        store1(Kc + (size_t)slot * D + lane * 2, kx[k][0]);
-        store1(Kc + (size_t)slot * D + lane * 2 + 1, kx[k][1]);
-        store1(Vc + (size_t)slot * D + lane * 2, vx[k][0]);
-        store1(Vc + (size_t)slot * D + lane * 2 + 1, vx[k][1]);
-      }
-      if (lane == 0) {
-        const float Rv = (p == tau) ? R_tau : 1.f;
-        Rs[kv][tk[k]] = Rv;
-        const size_t o = bk * a.n_cap + p;
-        if (a.dbg_target) a.dbg_target[o] = -1;
-        if (a.dbg_gate) a.dbg_gate[o] = 0.f;
-        if (a.dbg_decision) a.dbg_decision[o] = 2;
-        if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = Rv;
-      }
-    }
+  const int slot = a.slot_of[(size_t)b * a.n_cap + tau];
+  if (slot < 0 || slot >= a.m_cap) {
+    if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
+    return;
   }
-  __syncthreads();
-  // bias = alpha * ln(mean over KV heads of R) (Sec. 3.6, GQA), the same row for every head.
-  if (inX) {
-    const int slot = so[base + lane];
-    if (slot >= 0 && slot < a.m_cap) {
-      float s = 0.f;
-      for (int h = 0; h < a.Hkv; ++h) s += Rs[h][lane];
-      a.bias[bk * a.m_cap + slot] = a.alpha * logf(s / (float)a.Hkv);
-    }
+  T* Vc = static_cast<T*>(a.Vc) + (bk * a.m_cap + slot) * D + lane * PER;
+  if constexpr (PER == 4) {
+    store4(Vc, vm);
+  } else {
+    store1(Vc, vm[0]);
+    store1(Vc + 1, vm[1]);
+  }
+  if (lane == 0) {
+    a.ratio[bk * a.m_cap + slot] = R_tau;
+    if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = R_tau;
   }
 }
 
+// bias[b][kv][slot] = alpha * ln(mean over KV heads of R[b][kv][slot])   (Sec. 3.6, GQA)
+__global__ __launch_bounds__(256) void bias_kernel(CompressArgs a) {
+  const int b = blockIdx.y;
+  const int slot = blockIdx.x * blockDim.x + threadIdx.x;
+  if (slot >= a.seq_m[b]) return;
+  float s = 0.f;
+  for (int kv = 0; kv < a.Hkv; ++kv) s += a.ratio[((size_t)b * a.Hkv + kv) * a.m_cap + slot];
+  const float bias = a.alpha * logf(s / (float)a.Hkv);
+  for (int kv = 0; kv < a.Hkv; ++kv) a.bias[((size_t)b * a.Hkv + kv) * a.m_cap + slot] = bias;
+}
+
 template <typename T, int D>
-void launch_merge_t(const CompressArgs& a, dim3 grid, int threads, cudaStream_t s) {
-  if (threads <= 256) merge_kernel<T, D, 256><<<grid, threads, 0, s>>>(a);
-  else merge_kernel<T, D, 1024><<<grid, threads, 0, s>>>(a);
+void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
+  constexpr int kPieces = D * (int)sizeof(T) / 16;
+  const size_t copy_threads = (size_t)a.Hkv * a.m_cap * 2 * kPieces;
+  copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
+  merge_kernel<T, D><<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B * a.Hkv), kWarpsPerCta * 32, 0, s>>>(a);
 }
 
 }  // namespace
 
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s) {
-  const int nb = (a.n_cap + a.bucket - 1) / a.bucket;
-  const dim3 grid(nb, a.B);
-  const int threads = 32 * a.Hkv;
+  route_kernel<<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B), kWarpsPerCta * 32, 0, s>>>(a);
   if (a.dtype == SELKV_BF16) {
-    if (a.D == 128) launch_merge_t<__nv_bfloat16, 128>(a, grid, threads, s);
-    else launch_merge_t<__nv_bfloat16, 64>(a, grid, threads, s);
+    if (a.D == 128) launch_merge_t<__nv_bfloat16, 128>(a, s);
+    else launch_merge_t<__nv_bfloat16, 64>(a, s);
   } else {
-    if (a.D == 128) launch_merge_t<float, 128>(a, grid, threads, s);
-    else launch_merge_t<float, 64>(a, grid, threads, s);
+    if (a.D == 128) launch_merge_t<float, 128>(a, s);
+    else launch_merge_t<float, 64>(a, s);
   }
+  bias_kernel<<<dim3((a.m_cap + 255) / 256, a.B), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

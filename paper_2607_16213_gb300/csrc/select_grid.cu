@@ -311,7 +311,10 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
     const uint32_t slot = base + wcnt[warp] + __popc(bal & ((1u << lane) - 1u));
     if (j < n) {
       a.slot_of[(size_t)b * a.n_cap + j] = kept ? (int)slot : -1;
-      if (kept && a.dbg_kept_idx != nullptr && (int)slot < a.m_cap) a.dbg_kept_idx[(size_t)b * a.m_cap + slot] = j;
+      if (kept && (int)slot < a.m_cap) {
+        a.kept_pos[(size_t)b * a.m_cap + slot] = j;
+        if (a.dbg_kept_idx != nullptr) a.dbg_kept_idx[(size_t)b * a.m_cap + slot] = j;
+      }
     }
     base += wcnt[kBlock / 32];
     __syncthreads();

@@ -122,6 +122,11 @@ struct CompressArgs {
   float* score;      // [B][Hkv][n_cap]
   uint8_t* kflag;    // [B][n_cap] 1 = kept
   int32_t* slot_of;  // [B][n_cap] slot of a kept position, -1 otherwise
+  int32_t* kept_pos; // [B][m_cap] position of each slot
+  int nbk;           // buckets per sequence at n_cap: ceil(n_cap / bucket)
+  int32_t* tau;      // [B][Hkv][nbk] merge target of each bucket (-1: no kept token)
+  float* atau;       // [B][Hkv][nbk] a of that target
+  float* ratio;      // [B][Hkv][m_cap] attention ratio R of each slot
 };
 
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
