@@ -8,7 +8,7 @@
 //          for a bucket with no kept token);
 //   copy   every kept token's key and value row to its slot of K_c / V_c (keys unchanged) and
 //          ratio 1 for the slot; a thread per 16 bytes, coalesced;
-//   merge  warp per (non-empty bucket X, KV head, sequence b): the evicted tokens of X and of
+//   merge  one-warp CTA per (non-empty bucket X, KV head, sequence b): the evicted tokens of X and of
 //          the empty buckets that the nearest-ring rule gives to X, in ascending position
 //          order, 16 at a time: g_j = clamp(cos(v_j, v_tau), 0, 1) and
 //              v~_tau = (a_tau v_tau + sum g_j a_j v_j) / (a_tau + sum g_j a_j),
@@ -176,24 +176,39 @@ __device__ __forceinline__ float transpose_reduce16(const float (&p)[kBatch], in
 }
 
 template <typename T, int D>
-__global__ __launch_bounds__(kWarpsPerCta * 32) void merge_kernel(CompressArgs a) {
+__global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   constexpr int PER = D / 32;  // elements of a row per lane
-  const int lane = threadIdx.x & 31;
-  const int X = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+  const int lane = threadIdx.x;
+  const int X = blockIdx.x;
   const int kv = blockIdx.y % a.Hkv, b = blockIdx.y / a.Hkv;
   const int n = a.seq_n[b], Bs = a.bucket;
   const int nb = (n + Bs - 1) / Bs;
   if (X >= nb) return;
   const size_t bk = (size_t)b * a.Hkv + kv;
   const int32_t* tau_of = a.tau + bk * a.nbk;
-  const int tau = tau_of[X];
+  const float* atau_of = a.atau + bk * a.nbk;
   const int base = X * Bs;
-  const uint8_t* kf = a.kflag + (size_t)b * a.n_cap;
+  const bool inX = lane < min(Bs, n - base);
+  // One round of independent loads: tau_X and a(tau_X), the 32 buckets on either side (for
+  // the nearest non-empty ones), and the kept flags of X.
+  const int tau = tau_of[X];
+  const float a_tau = atau_of[X];
+  const bool expand = a.empty_bucket == SELKV_EMPTY_EXPAND;
+  const int eL = X - 1 - lane, eR = X + 1 + lane;
+  const int tl = (expand && eL >= 0) ? tau_of[eL] : -1;
+  const int tr = (expand && eR < nb) ? tau_of[eR] : -1;
+  const float al = (expand && eL >= 0) ? atau_of[eL] : 0.f;
+  const float ar = (expand && eR < nb) ? atau_of[eR] : 0.f;
+  const bool keptX = inX && a.kflag[(size_t)b * a.n_cap + base + lane] != 0;
+  const float* A = a.attn + bk * a.n_cap;
+  const float* vn = a.vnorm + bk * a.n_cap;
+  const float AX = inX ? A[base + lane] : 0.f;
+  const float NX = inX ? vn[base + lane] : 0.f;
   if (tau < 0) {
     // Empty bucket: under EXPAND a neighbour's warp owns these tokens; under DROP (or with
     // nothing kept at all) they stay without target.
     if (a.empty_bucket == SELKV_EMPTY_DROP || a.seq_m[b] == 0) {
-      if (lane < min(Bs, n - base)) {
+      if (inX) {
         const size_t o = bk * a.n_cap + base + lane;
         if (a.dbg_target) a.dbg_target[o] = -1;
         if (a.dbg_gate) a.dbg_gate[o] = 0.f;
@@ -202,28 +217,39 @@ __global__ __launch_bounds__(kWarpsPerCta * 32) void merge_kernel(CompressArgs a
     }
     return;
   }
-  const float* A = a.attn + bk * a.n_cap;
-  const float* vn = a.vnorm + bk * a.n_cap;
   const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
-  const float a_tau = a.atau[bk * a.nbk + X];
-  const float vn_tau = vn[tau];
+  const float vn_tau = __shfl_sync(0xffffffffu, NX, tau - base);
   RowSlice<T, PER> vt;
   vt.load(Vb + (size_t)tau * D + lane * PER);
 
   int lo_b = X, hi_b = X;  // buckets whose evicted tokens route to tau
-  if (a.empty_bucket == SELKV_EMPTY_EXPAND) {
-    // nearest non-empty buckets L < X and R > X, probing 32 buckets at a time
-    int L = -1;
-    for (int e0 = X - 1; e0 >= 0 && L < 0; e0 -= 32) {
-      const int e = e0 - lane;
-      const uint32_t m = __ballot_sync(0xffffffffu, e >= 0 && tau_of[e] >= 0);
-      if (m) L = e0 - (__ffs(m) - 1);
+  if (expand) {
+    // nearest non-empty buckets L < X and R > X (a further probe only past 32 empty ones)
+    int L = -1, R = -1;
+    float aL = 0.f, aR = 0.f;
+    uint32_t m = __ballot_sync(0xffffffffu, tl >= 0);
+    if (m) {
+      L = X - __ffs(m);
+      aL = __shfl_sync(0xffffffffu, al, __ffs(m) - 1);
+    } else {
+      for (int e0 = X - 33; e0 >= 0 && L < 0; e0 -= 32) {
+        const int e = e0 - lane;
+        const uint32_t mm = __ballot_sync(0xffffffffu, e >= 0 && tau_of[e] >= 0);
+        if (mm) L = e0 - (__ffs(mm) - 1);
+      }
+      if (L >= 0) aL = atau_of[L];
     }
-    int R = -1;
-    for (int e0 = X + 1; e0 < nb && R < 0; e0 += 32) {
-      const int e = e0 + lane;
-      const uint32_t m = __ballot_sync(0xffffffffu, e < nb && tau_of[e] >= 0);
-      if (m) R = e0 + (__ffs(m) - 1);
+    m = __ballot_sync(0xffffffffu, tr >= 0);
+    if (m) {
+      R = X + __ffs(m);
+      aR = __shfl_sync(0xffffffffu, ar, __ffs(m) - 1);
+    } else {
+      for (int e0 = X + 33; e0 < nb && R < 0; e0 += 32) {
+        const int e = e0 + lane;
+        const uint32_t mm = __ballot_sync(0xffffffffu, e < nb && tau_of[e] >= 0);
+        if (mm) R = e0 + (__ffs(mm) - 1);
+      }
+      if (R >= 0) aR = atau_of[R];
     }
     // An empty e between L and X goes to the nearer one; at equal distance both are in the
     // ring and X wins only with a strictly larger a (tau_L has the lower index).  Towards R,
@@ -232,51 +258,50 @@ __global__ __launch_bounds__(kWarpsPerCta * 32) void merge_kernel(CompressArgs a
       lo_b = 0;
     } else if (L < X - 1) {
       lo_b = (X + L) / 2 + 1;
-      if (((X + L) & 1) == 0 && a_tau > a.atau[bk * a.nbk + L]) lo_b = (X + L) / 2;
+      if (((X + L) & 1) == 0 && a_tau > aL) lo_b = (X + L) / 2;
     }
     if (R < 0) {
       hi_b = nb - 1;
     } else if (R > X + 1) {
       hi_b = (X + R - 1) / 2;
-      if (((X + R) & 1) == 0 && a_tau >= a.atau[bk * a.nbk + R]) hi_b = (X + R) / 2;
+      if (((X + R) & 1) == 0 && a_tau >= aR) hi_b = (X + R) / 2;
     }
   }
-
+  // Contributors: every position of buckets lo_b..hi_b except the kept tokens of X (the other
+  // buckets of the range are empty), in ascending order, up to kBatch at a time per bucket.
+  const uint32_t evX = __ballot_sync(0xffffffffu, inX && !keptX);
   float num[PER];
 #pragma unroll
-  for (int e = 0; e < PER; ++e) num[e] = 0.f;
+  for (int t = 0; t < PER; ++t) num[t] = 0.f;
   float den = 0.f;
   const int own = lane >> 1;  // contributor owned by this lane pair within a batch
   for (int e = lo_b; e <= hi_b; ++e) {
     const int eb = e * Bs;
-    const bool in_e = lane < min(Bs, n - eb);
-    uint32_t rem = __ballot_sync(0xffffffffu, in_e && kf[eb + lane] == 0);
+    const int cnt_e = min(Bs, n - eb);
+    uint32_t rem = e == X ? evX : (cnt_e >= 32 ? 0xffffffffu : ((1u << cnt_e) - 1u));
     // a and ||v|| of bucket e, one position per lane
-    const float Ae = in_e ? A[eb + lane] : 0.f;
-    const float Ne = in_e ? vn[eb + lane] : 0.f;
+    const float Ae = e == X ? AX : (lane < cnt_e ? A[eb + lane] : 0.f);
+    const float Ne = e == X ? NX : (lane < cnt_e ? vn[eb + lane] : 0.f);
     while (rem) {
-      // the next (up to) kBatch contributors, in position order
-      int bit[kBatch];
-      int cnt = 0;
+      // the (up to) kBatch lowest contributors left in this bucket
+      const int cut = __fns(rem, 0, kBatch + 1);  // position of the (kBatch+1)-th set bit
+      const uint32_t bm = (cut < 0 || cut > 31) ? rem : (rem & ((1u << cut) - 1u));
+      rem &= ~bm;
+      const int cnt = __popc(bm);
+      RowSlice<T, PER> vj[kBatch];
+      {
+        uint32_t r = bm;
 #pragma unroll
-      for (int k = 0; k < kBatch; ++k) {
-        bit[k] = -1;
-        if (rem) {
-          bit[k] = __ffs(rem) - 1;
-          rem &= rem - 1u;
-          ++cnt;
+        for (int k = 0; k < kBatch; ++k) {
+          if (r) {
+            vj[k].load(Vb + (size_t)(eb + __ffs(r) - 1) * D + lane * PER);
+            r &= r - 1u;
+          } else {
+            vj[k].zero();
+          }
         }
       }
-      RowSlice<T, PER> vj[kBatch];
-#pragma unroll
-      for (int k = 0; k < kBatch; ++k) {
-        if (bit[k] >= 0) vj[k].load(Vb + (size_t)(eb + bit[k]) * D + lane * PER);
-        else vj[k].zero();
-      }
-      int ob = -1;
-#pragma unroll
-      for (int k = 0; k < kBatch; ++k)
-        if (k == own) ob = bit[k];
+      const int ob = own < cnt ? (int)__fns(bm, 0, own + 1) : -1;  // bit of the owned contributor
       const float ak = __shfl_sync(0xffffffffu, Ae, ob < 0 ? 0 : ob);
       const float nk = __shfl_sync(0xffffffffu, Ne, ob < 0 ? 0 : ob);
       float g;
@@ -352,7 +377,7 @@ void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
   constexpr int kPieces = D * (int)sizeof(T) / 16;
   const size_t copy_threads = (size_t)a.Hkv * a.m_cap * 2 * kPieces;
   copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
-  merge_kernel<T, D><<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B * a.Hkv), kWarpsPerCta * 32, 0, s>>>(a);
+  merge_kernel<T, D><<<dim3(a.nbk, a.B * a.Hkv), 32, 0, s>>>(a);
 }
 
 }  // namespace
