@@ -20,7 +20,7 @@ namespace selkv {
 namespace {
 
 constexpr int kBlock = 512;                 // threads per CTA
-constexpr int kPerThread = 8;               // positions per thread
+constexpr int kPerThread = 2;               // positions per thread
 constexpr int kSpan = kBlock * kPerThread;  // positions per CTA
 constexpr int kBins = 2048;
 __device__ __constant__ int kShift[3] = {21, 10, 0};
@@ -32,7 +32,8 @@ __device__ __forceinline__ bool selected(uint32_t u, int j, const RadixState& s)
 }
 
 // Add this CTA's shared histogram to the unit's global one, then arrive; the last CTA of the
-// unit (of `nblocks`) picks the digit of `pass` and narrows the unit's state.
+// unit (of `nblocks`) reads the unit's histogram back into `sh` (one round of loads), picks
+// the digit of `pass` and narrows the unit's state.
 __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, int pass, int nblocks,
                                  bool* s_last) {
   const int bins = pass == 2 ? 1024 : kBins;
@@ -45,11 +46,13 @@ __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, 
   __syncthreads();
   if (!*s_last) return;
   __threadfence();
+  for (int i = threadIdx.x; i < bins; i += blockDim.x) sh[i] = __ldcg(&ghist[i]);
+  __syncthreads();
   if (threadIdx.x < 32) {
     const int lane = threadIdx.x, per = bins / 32;
     const int hi = bins - 1 - lane * per;  // this lane covers bins hi, hi-1, ..., hi-per+1
     uint32_t tot = 0;
-    for (int t = 0; t < per; ++t) tot += __ldcg(&ghist[hi - t]);
+    for (int t = 0; t < per; ++t) tot += sh[hi - t];
     uint32_t incl = tot;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -64,7 +67,7 @@ __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, 
       int dg = hi - per + 1;
       uint32_t cnt = 0;
       for (int t = 0; t < per; ++t) {
-        const uint32_t c = __ldcg(&ghist[hi - t]);
+        const uint32_t c = sh[hi - t];
         if (cum + c >= krem) {
           dg = hi - t;
           cnt = c;
@@ -198,10 +201,17 @@ __global__ __launch_bounds__(kBlock) void union_kernel(CompressArgs a, SelectWs 
   __shared__ uint32_t sh[kBins];
   __shared__ uint32_t s_cnt;
   __shared__ bool s_last;
+  __shared__ uint32_t s_prefix[32];
+  __shared__ int s_jcut[32];
   const int b = blockIdx.y;
   const int n = a.seq_n[b], ncand = n - a.recent;
   for (int i = threadIdx.x; i < kBins; i += kBlock) sh[i] = 0u;
   if (threadIdx.x == 0) s_cnt = 0u;
+  if (threadIdx.x < a.Hkv) {
+    const RadixState t = w.topk[(size_t)b * a.Hkv + threadIdx.x];
+    s_prefix[threadIdx.x] = t.prefix;
+    s_jcut[threadIdx.x] = t.jcut;
+  }
   __syncthreads();
   const int j0 = blockIdx.x * kSpan;
   uint32_t cnt = 0;
@@ -214,7 +224,8 @@ __global__ __launch_bounds__(kBlock) void union_kernel(CompressArgs a, SelectWs 
     for (int kv = 0; kv < a.Hkv; ++kv) {
       const size_t u = (size_t)b * a.Hkv + kv;
       const float s = a.score[u * a.n_cap + j];
-      const bool mem = j < ncand && selected(__float_as_uint(s), j, w.topk[u]);
+      const uint32_t x = __float_as_uint(s);
+      const bool mem = j < ncand && (x > s_prefix[kv] || (x == s_prefix[kv] && j <= s_jcut[kv]));
       if (a.dbg_topk != nullptr) a.dbg_topk[u * a.n_cap + j] = mem ? 1 : 0;
       in |= mem;
       sum += s;
