@@ -3,6 +3,7 @@
 #include <atomic>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 
 #include "selkv_internal.cuh"
 
@@ -35,6 +36,35 @@ bool shape_ok(const selkv_shape* s) {
 }
 
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// A side stream per device: the value-norm pass (HBM-bound) runs on it next to the scoring
+// passes (bound by the exponentials), forked from and joined back to the caller's stream with
+// events, a pattern that also records into a CUDA graph.  Created on first use outside a
+// capture; if it cannot be had, the pass runs on the caller's stream.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+  bool ready = false, failed = false;
+};
+constexpr int kMaxDevices = 64;
+std::mutex g_side_mu;
+SideStream g_side[kMaxDevices];
+
+// Requires g_side_mu.
+SideStream* side_stream(cudaStream_t caller) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  SideStream& x = g_side[dev];
+  if (!x.ready && !x.failed) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(caller, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return nullptr;
+    x.ready = cudaStreamCreateWithFlags(&x.s, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaEventCreateWithFlags(&x.fork, cudaEventDisableTiming) == cudaSuccess &&
+              cudaEventCreateWithFlags(&x.join, cudaEventDisableTiming) == cudaSuccess;
+    x.failed = !x.ready;
+  }
+  return x.ready ? &x : nullptr;
+}
 
 struct CompressPlan {
   size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
@@ -240,8 +270,19 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = launch_setup(a, tab, st);
-  if (e == cudaSuccess) e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st) : launch_score_simt(a, st);
-  if (e == cudaSuccess) e = launch_vnorm(a, st);
+  {
+    // value norms on the side stream (they need seq_n from the set-up; selection needs them)
+    std::lock_guard<std::mutex> lock(g_side_mu);
+    SideStream* side = e == cudaSuccess ? side_stream(st) : nullptr;
+    if (side != nullptr) {
+      e = cudaEventRecord(side->fork, st);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(side->s, side->fork, 0);
+      if (e == cudaSuccess) e = launch_vnorm(a, side->s);
+      if (e == cudaSuccess) e = cudaEventRecord(side->join, side->s);
+    }
+    if (e == cudaSuccess) e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st) : launch_score_simt(a, st);
+    if (e == cudaSuccess) e = side != nullptr ? cudaStreamWaitEvent(st, side->join, 0) : launch_vnorm(a, st);
+  }
   if (e == cudaSuccess)
     e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
