@@ -18,9 +18,6 @@ namespace {
 std::atomic<uint64_t> g_launches{0};
 constexpr int kCompressKernels = 18;  // with the tensor-core scoring (20 with the CUDA-core one)
 constexpr int kDecodeKernels = 1;
-// SM count used for planning the decode split: fixed, so that workspace sizes do not depend
-// on which device answers (GB300: 152 SMs).
-constexpr int kPlanSMs = 152;
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
@@ -81,7 +78,7 @@ CompressPlan plan_compress(const selkv_shape& s) {
   };
   const size_t B = s.batch, Hkv = s.num_kv_heads, n = s.n_cap;
   p.R = (s.num_q_heads / s.num_kv_heads) * s.obs_window;
-  p.nchunks = score_uses_tc(s.dtype, s.head_dim, p.R) ? score_tc_splits(s.batch, s.num_kv_heads, s.n_cap, kPlanSMs)
+  p.nchunks = score_uses_tc(s.dtype, s.head_dim, p.R) ? score_tc_splits(s.batch, s.num_kv_heads, s.n_cap, p.R, kPlanSMs)
                                                        : (int)((n + kRowChunk - 1) / kRowChunk);
   p.seq_n = take(B * 4);
   p.seq_m = take(B * 4);

@@ -30,7 +30,7 @@ namespace {
 static __device__ __align__(256) unsigned char g_decode_scratch[SELKV_STATIC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-constexpr int kPlanSMs = 152;  // the same split planning as selkv_decode_attn
+
 
 std::mutex g_mu;
 void* g_scratch_ptr[kMaxDevices] = {};

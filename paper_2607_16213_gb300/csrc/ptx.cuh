@@ -121,6 +121,46 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// 2^x for x <= 0 on the FMA and integer pipes, leaving the special-function unit to other
+// work: x = n + f with n = round(x) (adding 1.5 * 2^23 rounds to an integer in the low
+// mantissa bits) and f in [-1/2, 1/2]; 2^f is a degree-5 polynomial (minimax in relative
+// error on [-1/2, 1/2], fitted by Remez exchange; 2.3e-7 relative in this fp32 Horner form,
+// about the error of ex2.approx) and n is added to its exponent field.  Inputs below -127
+// are clamped (the result is then below 2^-126).
+__device__ __forceinline__ float ex2_poly(float x) {
+  x = fmaxf(x, -127.f);
+  const float t = x + 12582912.f;
+  const float f = x - (t - 12582912.f);
+  float p = 1.3276472e-3f;
+  p = fmaf(p, f, 9.6755410e-3f);
+  p = fmaf(p, f, 5.5507131e-2f);
+  p = fmaf(p, f, 2.4022120e-1f);
+  p = fmaf(p, f, 6.9314694e-1f);
+  p = fmaf(p, f, 1.0000001f);
+  const int n = __float_as_int(t) - __float_as_int(12582912.f);
+  return __int_as_float(__float_as_int(p) + (n << 23));
+}
+
+// Packed pairs of fp32 (sm_100 and later): one instruction for two lanes' worth of work.
+__device__ __forceinline__ uint64_t pack_f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack_f2(uint64_t x, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(x));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);

@@ -5,14 +5,18 @@
 // the causal re-pass of Sec. 3.1).  With s'_rj = log2(e) q_r . k_j / sqrt(d):
 //   pass 1: per row, over a slice of the keys: (max_j s'_rj, sum_j 2^(s'_rj - max)),
 //   (fold)  M_r, Z_r over the slices (rowstat_reduce_kernel),
-//   pass 2: a_j = sum_r 2^(s'_rj - M_r) / (G Z_r)   (Eq. 5's a, mean over the group).
-// Both passes are one kernel: a TMA producer warp streams 128-key K tiles (and the group's Q
-// once) into shared memory with 128-byte swizzling; one thread issues tcgen05.mma (bf16 in,
-// fp32 accumulate) into one of two tensor-memory accumulators; eight epilogue warps read the
+//   pass 2: a_j = sum_r 2^(s'_rj - M_r) / (G Z_r) = sum_r 2^(s'_rj - M_r - log2(G Z_r))
+//           (Eq. 5's a, mean over the group).
+// Both passes are one kernel: a TMA producer warp streams K tiles (and the group's Q once)
+// into shared memory with 128-byte swizzling; one thread issues tcgen05.mma (bf16 in, fp32
+// accumulate, N = 256 so each instruction carries a full-width product) into one of two
+// tensor-memory accumulators; sixteen epilogue warps (four per scheduler) read the
 // accumulator with tcgen05.ld and reduce it while the next tile is multiplied.  Pass 1 puts
-// the query rows in the accumulator lanes (M = 128 rows per MMA, N = 128 keys), so each
-// epilogue thread owns a row; pass 2 puts the keys in the lanes (M = 128 keys, N = R rows),
-// so each epilogue thread owns a column sum.
+// 128 query rows in the accumulator lanes (M = 128) and 256 keys in its columns, so a CTA
+// owns one half of the R rows; an epilogue thread owns a row and a quarter of each tile's
+// keys, and the four quarter states of a row are folded at the end.  Pass 2 puts 128 keys in
+// the lanes and the R rows in the columns; an epilogue thread owns a key and a quarter of the
+// rows, and the four quarter sums of a key are added in a fixed order.
 //
 // Every wait is bounded; on timeout the CTA raises SELKV_DEVERR_TIMEOUT, keeps the barrier
 // protocol of its epilogue warps, lets issued copies and MMAs finish (bounded) and frees its
@@ -25,20 +29,25 @@
 namespace selkv {
 namespace {
 
-constexpr int kKeys = 128;  // keys per tile
-constexpr int kEpiWarps = 8;
-constexpr int kProducerWarp = 8, kMmaWarp = 9;
+constexpr int kEpiWarps = 16;
+constexpr int kProducerWarp = 16, kMmaWarp = 17;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
-constexpr int kStages = 4;
 constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 columns
+// Which exponentials of a 32-wide chunk run as ex2_poly on the FMA pipe instead of the
+// special-function unit (6 of 32): the two units then finish a chunk at about the same time.
+__device__ __forceinline__ constexpr bool soft_exp(int i) { return (i & 15) < 3; }
+__device__ __forceinline__ float ex2_mixed(float x, bool soft) { return soft ? ex2_poly(x) : ex2_approx(x); }
 
-template <int D>
+template <int D, int PASS>
 struct SCfg {
+  static constexpr int kKeys = PASS == 1 ? 256 : 128;    // keys per tile
+  static constexpr int kStages = PASS == 1 ? 2 : 4;      // K tiles in flight
+  static constexpr int kRows = PASS == 1 ? 128 : 256;    // Q rows staged per CTA
   static constexpr int kBoxes = D / 64;                  // 128-byte-wide boxes per row
   static constexpr int kKTile = kKeys * D * 2;           // one K tile
-  static constexpr int kQBytes = 256 * D * 2;            // the group's Q, up to 256 rows
+  static constexpr int kQBytes = kRows * D * 2;
   static constexpr int kRing = kStages * kKTile;
-  static constexpr int kMisc = 256 + 256 * 8 + 2 * 128 * 4;
+  static constexpr int kMisc = 256 + 256 * 8 + 2 * 4 * 128 * 4;
   static constexpr int kSmem = 1024 + kQBytes + kRing + kMisc;
 };
 
@@ -46,7 +55,8 @@ template <int D, int PASS>
 __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                                                                 const __grid_constant__ CUtensorMap tmK,
                                                                 CompressArgs a) {
-  using C = SCfg<D>;
+  using C = SCfg<D, PASS>;
+  constexpr int kKeys = C::kKeys, kStages = C::kStages;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -61,23 +71,26 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   uint64_t* done = qbar + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float2* rstat = reinterpret_cast<float2*>(misc + 256);            // pass 2: (M, 1/(G Z))
-  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 2: [2][kKeys]
+  float* rneg = reinterpret_cast<float*>(misc + 256);               // pass 2: -(M + log2(G Z)) per row
+  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 2: [2][4][128]; pass 1: [4][128] float2
 
-  const int split = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
+  const int kv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = a.seq_n[b];
   const int R = a.R;
   const int Rp = (R + 15) & ~15;              // N of the pass-2 MMA
-  const int Rq = R > 128 ? 256 : 128;         // rows of Q staged (whole TMA boxes)
-  const int MT = (R + 127) / 128;             // pass-1 M tiles
+  const int MT = (R + 127) / 128;             // 128-row halves of the R rows
+  const int h = PASS == 1 ? (int)blockIdx.x % MT : 0;           // pass 1: this CTA's rows
+  const int split = PASS == 1 ? (int)blockIdx.x / MT : (int)blockIdx.x;
+  const int nsplit = PASS == 1 ? (int)gridDim.x / MT : (int)gridDim.x;
+  const int Rq = PASS == 1 ? 128 : (R > 128 ? 256 : 128);     // rows of Q staged (whole TMA boxes)
   const int ntiles_all = (n + kKeys - 1) / kKeys;
-  const int per = (ntiles_all + a.nchunks - 1) / a.nchunks;
+  const int per = (ntiles_all + nsplit - 1) / nsplit;
   const int t_begin = split * per;
   const int nt = max(0, min(ntiles_all, t_begin + per) - t_begin);
   const size_t bk = (size_t)b * a.Hkv + kv;
   const int krow0 = (int)(bk * a.n_cap) + t_begin * kKeys;
-  const int qrow0 = (b * a.Hq + kv * a.G) * a.W;
+  const int qrow0 = (b * a.Hq + kv * a.G) * a.W + h * 128;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
@@ -95,8 +108,11 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   }
   if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
   if (PASS == 2)
-    for (int r = threadIdx.x; r < 256; r += blockDim.x)
-      rstat[r] = r < R ? a.rowstat[bk * R + r] : make_float2(0.f, 0.f);
+    for (int r = threadIdx.x; r < 256; r += blockDim.x) {
+      // 2^(s' - M) / (G Z) = 2^(s' - (M + log2(G Z))): the normaliser joins the exponent
+      const float2 st = r < R ? a.rowstat[bk * R + r] : make_float2(0.f, 0.f);
+      rneg[r] = st.y > 0.f ? -(st.x - log2f(st.y)) : -INFINITY;
+    }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -145,9 +161,7 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
           const uint32_t koff = (ks >> 2) * (kKeys * 128) + (ks & 3) * 32;
           const uint32_t qoff = (ks >> 2) * (Rq * 128) + (ks & 3) * 32;
           if (PASS == 1) {
-            for (int mt = 0; mt < MT; ++mt)
-              umma_bf16(tmem + buf * 256 + mt * 128, umma_desc_sw128(qbase + qoff + mt * 128 * 128),
-                        umma_desc_sw128(kbase + koff), idesc, ks > 0);
+            umma_bf16(tmem + buf * 256, umma_desc_sw128(qbase + qoff), umma_desc_sw128(kbase + koff), idesc, ks > 0);
           } else {
             umma_bf16(tmem + buf * 256, umma_desc_sw128(kbase + koff), umma_desc_sw128(qbase + qoff), idesc, ks > 0);
           }
@@ -163,8 +177,8 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
       mbar_wait(done, 0);
     }
   } else {
-    // ---------------- epilogue: warps 0-7 ----------------
-    const int wg = warp >> 2, q = warp & 3;
+    // ---------------- epilogue: warps 0-15 ----------------
+    const int q = warp & 3, part = warp >> 2;  // lane quarter of TMEM, and which part of the work
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const float sc = a.scale_log2;
     // lane 0 waits, the warp follows its verdict (tcgen05.ld below needs the whole warp)
@@ -180,41 +194,50 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
       return __shfl_sync(0xffffffffu, ok, 0) != 0;
     };
     if (PASS == 1) {
-      const int r = wg * 128 + q * 32 + lane;  // query row owned by this thread
+      const int r = h * 128 + q * 32 + lane;    // query row owned by this thread
       const bool row_ok = r < R;
       const int p = n - a.W + (r % a.W);        // its last visible key
-      float m_run = -INFINITY, l_run = 0.f;
+      float m_run = -INFINITY, l_run = 0.f;     // running max (base 2, scaled) and sum
       for (int t = 0; t < nt; ++t) {
         const int buf = t & 1;
         const bool ok = warp_wait(&tfull[buf], (t >> 1) & 1);
         tc_fence_after();
-        if (ok && wg < MT) {
-          const int key0 = (t_begin + t) * kKeys;
-          const bool full_tile = key0 + kKeys - 1 <= n - a.W;  // every row sees every key
+        if (ok) {
+          const int key0 = (t_begin + t) * kKeys + part * 64;
+          const bool full_quarter = key0 + 63 <= n - a.W;  // every row sees every key of the quarter
 #pragma unroll 1
-          for (int c = 0; c < kKeys; c += 32) {
+          for (int c = 0; c < 64; c += 32) {
             float v[32];
-            tmem_ld32(tmem + lane_base + buf * 256 + wg * 128 + c, v);
+            tmem_ld32(tmem + lane_base + buf * 256 + part * 64 + c, v);
             float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (full_tile && row_ok) {
+            if (full_quarter && row_ok) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                v[i] *= sc;
-                cm[i & 3] = fmaxf(cm[i & 3], v[i]);
-              }
+              for (int i = 0; i < 32; ++i) cm[i & 3] = fmaxf(cm[i & 3], v[i]);
             } else {
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
-                v[i] = (row_ok && key0 + c + i <= p) ? v[i] * sc : -INFINITY;
+                v[i] = (row_ok && key0 + c + i <= p) ? v[i] : -INFINITY;
                 cm[i & 3] = fmaxf(cm[i & 3], v[i]);
               }
             }
-            const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
+            // the scale is positive, so max(v) * scale is the max of the scaled logits
+            const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])) * sc);
             if (mn != -INFINITY) {
-              float s4[4] = {0.f, 0.f, 0.f, 0.f};
+              // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
+              const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
+              uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
 #pragma unroll
-              for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_approx(v[i] - mn);
-              l_run = l_run * ex2_approx(m_run - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+              for (int i = 0; i < 32; i += 4) {
+                float x0, x1, x2, x3;
+                unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
+                unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
+                s01 = fadd2(s01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
+                s23 = fadd2(s23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
+              }
+              float s0, s1, s2, s3;
+              unpack_f2(s01, s0, s1);
+              unpack_f2(s23, s2, s3);
+              l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
               m_run = mn;
             }
           }
@@ -223,10 +246,26 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
       }
-      if (row_ok) a.rowpart[(bk * a.nchunks + split) * R + r] = make_float2(m_run, l_run);
+      // fold the four key quarters of each row in quarter order (quarters 1-3 via shared memory)
+      float2* st4 = reinterpret_cast<float2*>(colpart);  // [4][128]
+      if (part > 0) st4[part * 128 + q * 32 + lane] = make_float2(m_run, l_run);
+      named_bar_sync(1, kEpiWarps * 32);
+      if (part == 0 && row_ok) {
+        float2 o[4];
+        o[0] = make_float2(m_run, l_run);
+#pragma unroll
+        for (int k = 1; k < 4; ++k) o[k] = st4[k * 128 + q * 32 + lane];
+        const float M = fmaxf(fmaxf(o[0].x, o[1].x), fmaxf(o[2].x, o[3].x));
+        float L = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) L += o[k].y * ex2_approx(o[k].x - M);
+        }
+        a.rowpart[(bk * a.nchunks + split) * R + r] = make_float2(M, L);
+      }
     } else {
       const int klane = q * 32 + lane;   // key owned by this thread within the tile
-      const int r_lo = wg * 128, r_hi = min(R, r_lo + 128);
+      const int r_lo = part * 64, r_hi = min(R, r_lo + 64);
       for (int t = 0; t < nt; ++t) {
         const int buf = t & 1;
         const bool ok = warp_wait(&tfull[buf], (t >> 1) & 1);
@@ -241,32 +280,41 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
             tmem_ld32(tmem + lane_base + buf * 256 + c, v);
             const int cnt = min(32, r_hi - c);
             if (jrel <= 0 && cnt == 32) {
-              float a4[4] = {0.f, 0.f, 0.f, 0.f};
+              // sum over rows of 2^(v sc - M_r - log2(G Z_r)), pairs of rows packed; four
+              // interleaved partial sums as (0,1) and (2,3)
+              const uint64_t sc2 = pack_f2(sc, sc);
+              uint64_t a01 = pack_f2(0.f, 0.f), a23 = a01;
 #pragma unroll
-              for (int i = 0; i < 32; i += 2) {
-                const float4 st = *reinterpret_cast<const float4*>(&rstat[c + i]);  // rows c+i, c+i+1
-                a4[i & 3] = fmaf(ex2_approx(fmaf(v[i], sc, -st.x)), st.y, a4[i & 3]);
-                a4[(i + 1) & 3] = fmaf(ex2_approx(fmaf(v[i + 1], sc, -st.z)), st.w, a4[(i + 1) & 3]);
+              for (int i = 0; i < 32; i += 4) {
+                const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);  // rows c+i .. c+i+3
+                float x0, x1, x2, x3;
+                unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, pack_f2(nm.x, nm.y)), x0, x1);
+                unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, pack_f2(nm.z, nm.w)), x2, x3);
+                a01 = fadd2(a01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
+                a23 = fadd2(a23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
               }
-              acc += (a4[0] + a4[1]) + (a4[2] + a4[3]);
+              float s0, s1, s2, s3;
+              unpack_f2(a01, s0, s1);
+              unpack_f2(a23, s2, s3);
+              acc += (s0 + s1) + (s2 + s3);
             } else {
 #pragma unroll
               for (int i = 0; i < 32; ++i)
-                if (i < cnt && (jrel <= 0 || (c + i) % a.W >= jrel)) {
-                  const float2 st = rstat[c + i];
-                  acc = fmaf(ex2_approx(fmaf(v[i], sc, -st.x)), st.y, acc);
-                }
+                if (i < cnt && (jrel <= 0 || (c + i) % a.W >= jrel))
+                  acc += ex2_approx(fmaf(v[i], sc, rneg[c + i]));
             }
           }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
-        // fold the two row halves (warpgroups) of this key
-        float* cp = colpart + (t & 1) * kKeys;
-        if (wg == 1) cp[klane] = acc;
-        named_bar_sync(1, kEpiWarps * 32);
-        if (wg == 0 && j < n) a.attn[bk * a.n_cap + j] = acc + cp[klane];
+        // fold the four row quarters of this key, in quarter order; only the four warps of a
+        // lane quarter (one scheduler) share keys, so each quarter has its own barrier
+        float* cp = colpart + (t & 1) * 4 * kKeys;
+        if (part > 0) cp[part * kKeys + klane] = acc;
+        named_bar_sync(2 + q, 4 * 32);
+        if (part == 0 && j < n)
+          a.attn[bk * a.n_cap + j] = ((acc + cp[kKeys + klane]) + cp[2 * kKeys + klane]) + cp[3 * kKeys + klane];
       }
     }
   }
@@ -278,22 +326,37 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   }
 }
 
+// Splits of the keys of one (sequence, KV head): enough CTAs for one per SM, each CTA
+// owning `row_parts` x (a slice of `keys`-key tiles).
+int splits_for(int B, int Hkv, int n_cap, int num_sms, int row_parts, int keys) {
+  const int units = B * Hkv * row_parts;
+  const int tiles = (n_cap + keys - 1) / keys;
+  int s = num_sms / units;
+  if (s > tiles) s = tiles;
+  return s < 1 ? 1 : s;
+}
+
 template <int D>
 cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st) {
-  CUtensorMap tq, tk;
+  using C1 = SCfg<D, 1>;
+  using C2 = SCfg<D, 2>;
+  CUtensorMap tq, tk1, tk2;
   if (!encode_rows_bf16(&tq, a.Q, (uint64_t)a.B * a.Hq * a.W, D, 128) ||
-      !encode_rows_bf16(&tk, a.K, (uint64_t)a.B * a.Hkv * a.n_cap, D, 128))
+      !encode_rows_bf16(&tk1, a.K, (uint64_t)a.B * a.Hkv * a.n_cap, D, C1::kKeys) ||
+      !encode_rows_bf16(&tk2, a.K, (uint64_t)a.B * a.Hkv * a.n_cap, D, C2::kKeys))
     return cudaErrorInvalidValue;
-  const dim3 grid(a.nchunks, a.Hkv, a.B);
+  const int MT = (a.R + 127) / 128;
+  const dim3 grid1(a.nchunks * MT, a.Hkv, a.B);
+  const dim3 grid2(splits_for(a.B, a.Hkv, a.n_cap, kPlanSMs, 1, C2::kKeys), a.Hkv, a.B);
   auto k1 = score_tc_kernel<D, 1>;
   auto k2 = score_tc_kernel<D, 2>;
-  cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, SCfg<D>::kSmem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, SCfg<D>::kSmem);
+  cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, C1::kSmem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, C2::kSmem);
   if (e != cudaSuccess) return e;
-  k1<<<grid, kThreads, SCfg<D>::kSmem, st>>>(tq, tk, a);
+  k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
   e = launch_rowstat_reduce(a, st);
   if (e != cudaSuccess) return e;
-  k2<<<grid, kThreads, SCfg<D>::kSmem, st>>>(tq, tk, a);
+  k2<<<grid2, kThreads, C2::kSmem, st>>>(tq, tk2, a);
   return cudaGetLastError();
 }
 
@@ -301,13 +364,8 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st) {
 
 bool score_uses_tc(int dtype, int D, int R) { return dtype == SELKV_BF16 && (D == 64 || D == 128) && R >= 1 && R <= 256; }
 
-int score_tc_splits(int B, int Hkv, int n_cap, int num_sms) {
-  const int units = B * Hkv;
-  const int tiles = (n_cap + kKeys - 1) / kKeys;
-  int s = num_sms / units;
-  if (s < 1) s = 1;
-  if (s > tiles) s = tiles;
-  return s < 1 ? 1 : s;
+int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms) {
+  return splits_for(B, Hkv, n_cap, num_sms, (R + 127) / 128, SCfg<128, 1>::kKeys);
 }
 
 cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t st) {

@@ -129,6 +129,10 @@ struct CompressArgs {
   float* ratio;      // [B][Hkv][m_cap] attention ratio R of each slot
 };
 
+// SM count used to plan grids and splits: fixed, so that workspace sizes and results do
+// not depend on which device answers (GB300: 152 SMs).
+constexpr int kPlanSMs = 152;
+
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
 
 // Grid-wide exact radix selection (select_grid.cu).
@@ -158,7 +162,7 @@ cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStr
 
 // Scoring: tensor-core path for bf16 with G W <= 256 rows, CUDA-core path otherwise.
 bool score_uses_tc(int dtype, int D, int R);
-int score_tc_splits(int B, int Hkv, int n_cap, int num_sms);
+int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms);  // pass-1 key splits
 cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
