@@ -64,7 +64,7 @@ SideStream* side_stream(cudaStream_t caller) {
 }
 
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
   int nchunks, R;
 };
 
@@ -85,6 +85,7 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.rowpart = take(B * Hkv * (size_t)p.nchunks * p.R * sizeof(float2));
   p.rowstat = take(B * Hkv * (size_t)p.R * sizeof(float2));
   p.attn = take(B * Hkv * n * 4);
+  p.attn_part = score_uses_tc(s.dtype, s.head_dim, p.R) ? take(4 * B * Hkv * n * 4) : 0;
   p.vnorm = take(B * Hkv * n * 4);
   p.score = take(B * Hkv * n * 4);
   p.kflag = take(B * n);
@@ -249,6 +250,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.rowstat = at<float2>(workspace, plan.rowstat);
   a.attn = (debug && debug->attn) ? debug->attn : at<float>(workspace, plan.attn);
   a.vnorm = at<float>(workspace, plan.vnorm);
+  a.attn_parts = score_uses_tc(a.dtype, a.D, a.R) ? 4 : 1;
+  a.attn_part = a.attn_parts == 4 ? at<float>(workspace, plan.attn_part) : nullptr;
   a.score = (debug && debug->score) ? debug->score : at<float>(workspace, plan.score);
   a.kflag = at<uint8_t>(workspace, plan.kflag);
   a.slot_of = at<int32_t>(workspace, plan.slot);

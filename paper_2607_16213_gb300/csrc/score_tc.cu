@@ -16,7 +16,8 @@
 // owns one half of the R rows; an epilogue thread owns a row and a quarter of each tile's
 // keys, and the four quarter states of a row are folded at the end.  Pass 2 puts 128 keys in
 // the lanes and the R rows in the columns; an epilogue thread owns a key and a quarter of the
-// rows, and the four quarter sums of a key are added in a fixed order.
+// rows and writes that quarter's column sum; the pooling kernel of the selection adds the four
+// quarters of a key in a fixed order.
 //
 // Every wait is bounded; on timeout the CTA raises SELKV_DEVERR_TIMEOUT, keeps the barrier
 // protocol of its epilogue warps, lets issued copies and MMAs finish (bounded) and frees its
@@ -33,9 +34,17 @@ constexpr int kEpiWarps = 16;
 constexpr int kProducerWarp = 16, kMmaWarp = 17;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 columns
+#ifndef SELKV_SOFT_EXP
+#define SELKV_SOFT_EXP 0  // of every 16 exponentials, how many run as ex2_poly
+#endif
+#ifndef SELKV_PACKED
+#define SELKV_PACKED 1    // packed f32x2 arguments and sums in the epilogues
+#endif
 // Which exponentials of a 32-wide chunk run as ex2_poly on the FMA pipe instead of the
-// special-function unit (6 of 32): the two units then finish a chunk at about the same time.
-__device__ __forceinline__ constexpr bool soft_exp(int i) { return (i & 15) < 3; }
+// special-function unit.  On GB300 at these shapes the epilogues are bound by instruction
+// issue rather than by the special-function unit, and moving exponentials to the FMA pipe
+// (2 to 10 of 32) only slowed them, so the default is none.
+__device__ __forceinline__ constexpr bool soft_exp(int i) { return (i & 15) < SELKV_SOFT_EXP; }
 __device__ __forceinline__ float ex2_mixed(float x, bool soft) { return soft ? ex2_poly(x) : ex2_approx(x); }
 
 template <int D, int PASS>
@@ -72,7 +81,7 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* rneg = reinterpret_cast<float*>(misc + 256);               // pass 2: -(M + log2(G Z)) per row
-  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 2: [2][4][128]; pass 1: [4][128] float2
+  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [4][128] float2
 
   const int kv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -224,19 +233,29 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
             const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])) * sc);
             if (mn != -INFINITY) {
               // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
-              const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
-              uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
-#pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                float x0, x1, x2, x3;
-                unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
-                unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
-                s01 = fadd2(s01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
-                s23 = fadd2(s23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
-              }
               float s0, s1, s2, s3;
-              unpack_f2(s01, s0, s1);
-              unpack_f2(s23, s2, s3);
+              if (SELKV_PACKED) {
+                const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
+                uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                  float x0, x1, x2, x3;
+                  unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
+                  unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
+                  s01 = fadd2(s01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
+                  s23 = fadd2(s23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
+                }
+                unpack_f2(s01, s0, s1);
+                unpack_f2(s23, s2, s3);
+              } else {
+                float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_mixed(fmaf(v[i], sc, -mn), soft_exp(i));
+                s0 = s4[0];
+                s1 = s4[1];
+                s2 = s4[2];
+                s3 = s4[3];
+              }
               l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
               m_run = mn;
             }
@@ -282,20 +301,36 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
             if (jrel <= 0 && cnt == 32) {
               // sum over rows of 2^(v sc - M_r - log2(G Z_r)), pairs of rows packed; four
               // interleaved partial sums as (0,1) and (2,3)
-              const uint64_t sc2 = pack_f2(sc, sc);
-              uint64_t a01 = pack_f2(0.f, 0.f), a23 = a01;
-#pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);  // rows c+i .. c+i+3
-                float x0, x1, x2, x3;
-                unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, pack_f2(nm.x, nm.y)), x0, x1);
-                unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, pack_f2(nm.z, nm.w)), x2, x3);
-                a01 = fadd2(a01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
-                a23 = fadd2(a23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
-              }
               float s0, s1, s2, s3;
-              unpack_f2(a01, s0, s1);
-              unpack_f2(a23, s2, s3);
+              if (SELKV_PACKED) {
+                const uint64_t sc2 = pack_f2(sc, sc);
+                uint64_t a01 = pack_f2(0.f, 0.f), a23 = a01;
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                  const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);  // rows c+i .. c+i+3
+                  float x0, x1, x2, x3;
+                  unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, pack_f2(nm.x, nm.y)), x0, x1);
+                  unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, pack_f2(nm.z, nm.w)), x2, x3);
+                  a01 = fadd2(a01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
+                  a23 = fadd2(a23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
+                }
+                unpack_f2(a01, s0, s1);
+                unpack_f2(a23, s2, s3);
+              } else {
+                float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                  const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);
+                  s4[0] += ex2_mixed(fmaf(v[i], sc, nm.x), soft_exp(i));
+                  s4[1] += ex2_mixed(fmaf(v[i + 1], sc, nm.y), soft_exp(i + 1));
+                  s4[2] += ex2_mixed(fmaf(v[i + 2], sc, nm.z), soft_exp(i + 2));
+                  s4[3] += ex2_mixed(fmaf(v[i + 3], sc, nm.w), soft_exp(i + 3));
+                }
+                s0 = s4[0];
+                s1 = s4[1];
+                s2 = s4[2];
+                s3 = s4[3];
+              }
               acc += (s0 + s1) + (s2 + s3);
             } else {
 #pragma unroll
@@ -308,13 +343,8 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
-        // fold the four row quarters of this key, in quarter order; only the four warps of a
-        // lane quarter (one scheduler) share keys, so each quarter has its own barrier
-        float* cp = colpart + (t & 1) * 4 * kKeys;
-        if (part > 0) cp[part * kKeys + klane] = acc;
-        named_bar_sync(2 + q, 4 * 32);
-        if (part == 0 && j < n)
-          a.attn[bk * a.n_cap + j] = ((acc + cp[kKeys + klane]) + cp[2 * kKeys + klane]) + cp[3 * kKeys + klane];
+        // this row quarter's column sum; the pooling kernel adds the four quarters in order
+        if (j < n) a.attn_part[((size_t)part * a.B * a.Hkv + bk) * a.n_cap + j] = acc;
       }
     }
   }

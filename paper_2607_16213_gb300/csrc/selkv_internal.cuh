@@ -118,6 +118,8 @@ struct CompressArgs {
   float2* rowpart;   // [B][Hkv][nchunks][R] (max, sum) of 2^(s' - max) per column chunk
   float2* rowstat;   // [B][Hkv][R] (M, 1 / (G * Z))
   float* attn;       // [B][Hkv][n_cap]
+  float* attn_part;  // [4][B][Hkv][n_cap] column sums of four row quarters (tensor-core scoring)
+  int attn_parts;    // 4: attn is the sum of attn_part, formed by the pooling kernel; 1: attn is final
   float* vnorm;      // [B][Hkv][n_cap]
   float* score;      // [B][Hkv][n_cap]
   uint8_t* kflag;    // [B][n_cap] 1 = kept
