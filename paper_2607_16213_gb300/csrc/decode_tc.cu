@@ -549,7 +549,7 @@ cudaError_t launch_tc_t(const DecodeArgs& a, cudaStream_t st) {
   if (!encode_rows_bf16(&tk, a.Kc, rows, D, kBoxRows) || !encode_rows_bf16(&tv, a.Vc, rows, D, kBoxRows))
     return cudaErrorInvalidValue;
   auto kern = decode_tc_kernel<D, R16>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::kSmemBytes);
+  cudaError_t e = set_smem_once<decode_tc_kernel<D, R16>>(Cfg<D>::kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.splits, a.Hkv, a.B);

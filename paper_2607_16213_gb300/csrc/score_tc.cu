@@ -380,8 +380,8 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st) {
   const dim3 grid2(splits_for(a.B, a.Hkv, a.n_cap, kPlanSMs, 1, C2::kKeys), a.Hkv, a.B);
   auto k1 = score_tc_kernel<D, 1>;
   auto k2 = score_tc_kernel<D, 2>;
-  cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, C1::kSmem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, C2::kSmem);
+  cudaError_t e = set_smem_once<score_tc_kernel<D, 1>>(C1::kSmem);
+  if (e == cudaSuccess) e = set_smem_once<score_tc_kernel<D, 2>>(C2::kSmem);
   if (e != cudaSuccess) return e;
   k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
   e = launch_rowstat_reduce(a, st);

@@ -1,6 +1,8 @@
 // Internal declarations shared by the SelKV kernels and the C-ABI host code.
 #pragma once
 
+#include <atomic>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -192,6 +194,21 @@ struct DecodeArgs {
 // every record starts 16-byte aligned and can be moved with one bulk copy.
 __host__ __device__ constexpr size_t decode_record_floats(int G, int S, int D) {
   return (size_t)G * S * D + (((size_t)G * S * 2 + 3) & ~(size_t)3);
+}
+
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per kernel and device (the attribute
+// persists; repeating it costs host time on every launch).  Keyed by the kernel itself.
+template <auto Kern>
+cudaError_t set_smem_once(int bytes) {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+  if (bit != 0 && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(Kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit != 0) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
 }
 
 int decode_splits(int B, int Hkv, int m_cap, int num_sms);
