@@ -9,7 +9,8 @@ Merge-or-Drop and Attention Compensation"):
 
   observation re-pass (Sec. 3.1) -> contribution score (Eq. 1) -> average pooling (Sec. 3.2)
   -> budget m = floor(rho n), recent window m_r (Sec. 3.1) -> per-KV-head top-m_s, union over
-  KV heads, trim by mean score (Eq. 2, Sec. 3.3 "Union selection") -> bucket-attention routing
+  KV heads, trim by mean score (Eq. 2, Sec. 3.3 "Union selection"; or, in per-head mode,
+  each head's own top-m_s, Sec. 3.3 "Per-head selection") -> bucket-attention routing
   (Eq. 3, Sec. 3.4) -> soft cosine gate (Eq. 4, Sec. 3.5) -> gated attention-weighted merge (Eq. 5) -> attention
   ratio (Eq. 6) -> GQA bias alpha*log(mean_kv R) (Sec. 3.6) -> decode with the bias (Alg. 1,
   last step).  RoPE repositioning (Eq. 7) is off, as in the paper's configuration (Sec. 4.1; Eq. 7 is Sec. 3.7).
@@ -38,6 +39,10 @@ path):
   R14 decision MERGE iff g > 0, else DROP.
   R15 a_i = 0 guard: R = 1, and v~ = v_i when the denominator is 0.
   R16 GQA bias = alpha * ln(mean over KV heads of R) (natural log), per layer.
+  R17 per-head mode (Sec. 3.3, MHA models; Sec. 3.6 "per head without cross-head
+      averaging"): each KV head keeps its own top-m_s of its pooled score plus the recent
+      window, routes, gates and merges against that set, and its bias is alpha * ln R of its
+      own entries.  On a GQA model the G query heads of a KV head share its set.
 """
 from __future__ import annotations
 
@@ -48,6 +53,7 @@ from typing import Optional
 import numpy as np
 
 GATE_COSINE, GATE_OPEN, GATE_CLOSED = 0, 1, 2
+SELECT_SHARED, SELECT_PER_HEAD = 0, 1
 EMPTY_EXPAND, EMPTY_DROP = 0, 1
 DECISION_DROP, DECISION_MERGE = 0, 1
 
@@ -61,6 +67,7 @@ class Params:
     recent: int = 16
     gate_mode: int = GATE_COSINE
     empty_bucket: int = EMPTY_EXPAND
+    select_mode: int = SELECT_SHARED
 
 
 # ----------------------------------------------------------------------------------------
@@ -185,6 +192,22 @@ def select_shared(c_pooled: np.ndarray, n: int, m_s: int, recent: int,
     return Selection(per_kv, union, kept_cand, kept, trimmed)
 
 
+def select_per_head(c_pooled: np.ndarray, n: int, m_s: int, recent: int,
+                    follow_per_kv: Optional[np.ndarray] = None) -> np.ndarray:
+    """Per-head selection (Eq. 2; Sec. 3.3 "Per-head selection"; R7, R17): each KV head's
+    top-m_s of its pooled score over the candidates, plus the recent window.  Returns the
+    kept masks [Hkv][n].  follow_per_kv replaces the top-m_s choices as in select_shared."""
+    Hkv, n_cand = c_pooled.shape
+    kept = np.zeros((Hkv, n), dtype=bool)
+    for kv in range(Hkv):
+        if follow_per_kv is not None:
+            kept[kv, :n_cand] = np.asarray(follow_per_kv[kv, :n_cand], dtype=bool)
+        else:
+            kept[kv, :n_cand] = top_k_mask(c_pooled[kv], m_s)
+        kept[kv, n - recent:] = True
+    return kept
+
+
 # ----------------------------------------------------------------------------------------
 # Eq. 3: bucket-attention routing
 # ----------------------------------------------------------------------------------------
@@ -290,6 +313,12 @@ def gqa_bias(R: np.ndarray, alpha: float) -> np.ndarray:
     return alpha * np.log(R.mean(axis=0))
 
 
+def per_head_bias(R: np.ndarray, alpha: float) -> np.ndarray:
+    """Sec. 3.6 with per-head selection: bias_{h,i} = alpha * ln R_{h,i}, no averaging across
+    heads (R17).  R: [Hkv][m]; returns [Hkv][m]."""
+    return alpha * np.log(R)
+
+
 # ----------------------------------------------------------------------------------------
 # Algorithm 1 for one sequence of one layer
 # ----------------------------------------------------------------------------------------
@@ -301,8 +330,8 @@ class CompressResult:
     vnorm: np.ndarray         # [Hkv][n]
     c: np.ndarray             # [Hkv][n] contribution score (Eq. 1)
     c_pooled: np.ndarray      # [Hkv][n_cand]
-    sel: Selection
-    kept_idx: np.ndarray      # [m] ascending
+    sel: Optional[Selection]  # shared mode only
+    kept_idx: np.ndarray      # [m] ascending (shared mode) or [Hkv][m] (per-head mode)
     target: np.ndarray        # [Hkv][n]
     g: np.ndarray             # [Hkv][n]
     sim: np.ndarray           # [Hkv][n]
@@ -310,7 +339,8 @@ class CompressResult:
     K_c: np.ndarray           # [Hkv][m][d]
     V_c: np.ndarray           # [Hkv][m][d]
     R: np.ndarray             # [Hkv][m]
-    bias: np.ndarray          # [m]
+    bias: np.ndarray          # [m] (shared mode) or [Hkv][m] (per-head mode)
+    per_head: bool = False
     extra: dict = field(default_factory=dict)
 
 
@@ -335,6 +365,8 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     vn = value_norms(V, n)
     c = a * vn                                                # Eq. 1
     cp = pool_scores(c, n_cand, params.pool_kernel)           # smoothing
+    if params.select_mode == SELECT_PER_HEAD:
+        return _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target)
     sel = select_shared(cp, n, m_s, params.recent, follow_per_kv, follow_kept)  # step 2
     kept_idx = np.flatnonzero(sel.kept)
     target = np.full((Hkv, n), -1, dtype=np.int64)
@@ -353,6 +385,32 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=sel,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
                           K_c=K[:, kept_idx].copy(), V_c=Vc, R=R, bias=bias)
+
+
+def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target):
+    """Algorithm 1 steps 2-6 with per-head selection (R17): every KV head has its own kept
+    set, targets, merged values and bias row."""
+    Hkv, _, d = K.shape
+    kept = select_per_head(cp, n, m_s, params.recent, follow_per_kv)      # step 2, per head
+    kept_idx = np.stack([np.flatnonzero(kept[kv]) for kv in range(Hkv)])  # [Hkv][m]
+    target = np.full((Hkv, n), -1, dtype=np.int64)
+    g = np.zeros((Hkv, n))
+    sim = np.zeros((Hkv, n))
+    decision = np.zeros((Hkv, n), dtype=np.uint8)
+    Kc = np.empty((Hkv, m, d))
+    Vc = np.empty((Hkv, m, d))
+    R = np.ones((Hkv, m))
+    for kv in range(Hkv):
+        t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
+             else route(a[kv], kept[kv], params.bucket, params.empty_bucket))  # step 3
+        target[kv] = t
+        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
+        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx[kv], t, g[kv])        # steps 5, 6
+        Kc[kv] = K[kv, kept_idx[kv]]
+    return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=None,
+                          kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
+                          K_c=Kc, V_c=Vc, R=R, bias=per_head_bias(R, params.alpha), per_head=True,
+                          extra={"kept": kept})
 
 
 # ----------------------------------------------------------------------------------------

@@ -373,3 +373,92 @@ def test_rejects_budget_below_recent_window():
     wl, K, V, Q, n = _tiny()
     with pytest.raises(ValueError):
         O.compress(K, V, Q, n, 0.01)
+
+
+# ---------------------------------------------------------------- per-head mode (Sec. 3.3, 3.6)
+def test_per_head_bias_worked_example():
+    gd = golden("per_head_bias.json")
+    np.testing.assert_allclose(O.per_head_bias(np.array(gd["R"]), gd["alpha"]), gd["bias"],
+                               rtol=1e-14, atol=1e-16)
+
+
+def _mha(seed, Hkv=4, n=640, d=32, W=16):
+    r = rng(seed)
+    K = r.standard_normal((Hkv, n, d))
+    V = r.standard_normal((Hkv, n, d))
+    Q = r.standard_normal((Hkv, W, d)) * 1.5   # G = 1: one query head per KV head
+    return K, V, Q, n
+
+
+def test_per_head_selection_brute_force():
+    """Eq. 2 per head: each head's kept set is the recent window plus its m_s best pooled
+    scores, checked against a full sort with the (value desc, position asc) key."""
+    K, V, Q, n = _mha(11)
+    p = O.Params(select_mode=O.SELECT_PER_HEAD, recent=8, bucket=16)
+    r = O.compress(K, V, Q, n, 0.25, p)
+    n_cand = n - p.recent
+    for kv in range(K.shape[0]):
+        order = sorted(range(n_cand), key=lambda j: (-r.c_pooled[kv, j], j))
+        expect = sorted(order[:r.m_s]) + list(range(n_cand, n))
+        assert r.kept_idx[kv].tolist() == expect
+
+
+def test_per_head_with_one_kv_head_equals_shared():
+    """With a single KV head the union of one set is that set and no trim happens, so both
+    modes must give the same cache, targets and bias (Sec. 3.3, Sec. 3.6)."""
+    K, V, Q, n = _mha(12, Hkv=1)
+    shared = O.compress(K, V, Q, n, 0.25, O.Params(recent=8, bucket=16))
+    per = O.compress(K, V, Q, n, 0.25, O.Params(recent=8, bucket=16, select_mode=O.SELECT_PER_HEAD))
+    assert per.kept_idx[0].tolist() == shared.kept_idx.tolist()
+    np.testing.assert_array_equal(per.target, shared.target)
+    np.testing.assert_array_equal(per.V_c, shared.V_c)
+    np.testing.assert_array_equal(per.K_c, shared.K_c)
+    np.testing.assert_allclose(per.bias[0], shared.bias, rtol=0, atol=0)
+
+
+def test_per_head_sets_differ_and_follow_their_heads():
+    """Heads whose attention favours different positions keep different sets, each with its
+    own favoured positions (the point of per-head selection, Sec. 3.3)."""
+    K, V, Q, n = _mha(13, Hkv=2)
+    hot = {0: [40, 41, 300], 1: [120, 121, 500]}
+    for kv, pos in hot.items():
+        for j in pos:
+            K[kv, j] = 6.0 * Q[kv].mean(axis=0) / np.linalg.norm(Q[kv].mean(axis=0))
+    r = O.compress(K, V, Q, n, 0.1, O.Params(select_mode=O.SELECT_PER_HEAD, recent=8, bucket=16))
+    s0, s1 = set(r.kept_idx[0].tolist()), set(r.kept_idx[1].tolist())
+    assert s0 != s1
+    assert set(hot[0]) <= s0 and set(hot[1]) <= s1
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_per_head_pipeline_invariants(seed):
+    """Per head: exactly m kept, recent window kept, every target a kept token of that head
+    in the evicted token's bucket when that bucket has one, R >= 1, mass conservation
+    sum_S a_i R_i = sum_S a_i + sum_E g_j a_j, and a closed gate is pure eviction."""
+    K, V, Q, n = _mha(20 + seed)
+    p = O.Params(select_mode=O.SELECT_PER_HEAD, recent=8, bucket=16)
+    r = O.compress(K, V, Q, n, 0.3, p)
+    for kv in range(K.shape[0]):
+        kept = r.kept_idx[kv]
+        assert kept.size == r.m and set(range(n - p.recent, n)) <= set(kept.tolist())
+        ks = set(kept.tolist())
+        for j in range(n):
+            t = int(r.target[kv, j])
+            if j in ks:
+                assert t == -1
+                continue
+            assert t in ks
+            same = [i for i in kept if i // p.bucket == j // p.bucket]
+            if same:
+                assert t // p.bucket == j // p.bucket
+        assert (r.R[kv] >= 1.0 - 1e-15).all()
+        lhs = float((r.a[kv, kept] * r.R[kv]).sum())
+        ev = r.target[kv] >= 0
+        rhs = float(r.a[kv, kept].sum() + (r.g[kv, ev] * r.a[kv, ev]).sum())
+        assert abs(lhs - rhs) <= 1e-12 * rhs
+        np.testing.assert_allclose(r.bias[kv], p.alpha * np.log(r.R[kv]), rtol=0, atol=0)
+    closed = O.compress(K, V, Q, n, 0.3, O.Params(select_mode=O.SELECT_PER_HEAD, recent=8, bucket=16,
+                                                  gate_mode=O.GATE_CLOSED))
+    for kv in range(K.shape[0]):
+        np.testing.assert_allclose(closed.V_c[kv], V[kv, closed.kept_idx[kv]], rtol=1e-15, atol=0)
+    np.testing.assert_array_equal(closed.bias, 0.0)
