@@ -69,6 +69,12 @@ typedef enum selkv_gate_mode {
  * gives them g = 0 and no target. */
 typedef enum selkv_empty_bucket { SELKV_EMPTY_EXPAND = 0, SELKV_EMPTY_DROP = 1 } selkv_empty_bucket;
 
+/* Token selection (Sec. 3.3): SHARED is the union selection of GQA models (every KV head keeps
+ * the same set: each KV head's top-m_s, union, trim by the mean score); PER_HEAD is the
+ * per-head selection of MHA models (each KV head keeps its own top-m_s, and its bias is
+ * alpha * ln R of its own entries, without averaging across heads, Sec. 3.6). */
+typedef enum selkv_select_mode { SELKV_SELECT_SHARED = 0, SELKV_SELECT_PER_HEAD = 1 } selkv_select_mode;
+
 /* Device error bits (selkv_workspace_error). */
 #define SELKV_DEVERR_CAPACITY 0x1u /* decode append would pass m_cap: not appended       */
 #define SELKV_DEVERR_TIMEOUT 0x2u  /* a bounded wait gave up; the launch's output is void  */
@@ -96,6 +102,7 @@ typedef struct selkv_params {
   int32_t recent;       /* recent window m_r always kept, 16 (Sec. 3.1)                 */
   int32_t gate_mode;    /* selkv_gate_mode                                              */
   int32_t empty_bucket; /* selkv_empty_bucket                                           */
+  int32_t select_mode;  /* selkv_select_mode, SHARED for GQA models (Sec. 4.1)            */
 } selkv_params;
 
 /* Optional device outputs of selkv_compress, for inspection and testing.  Any field may be
@@ -104,7 +111,8 @@ typedef struct selkv_compress_debug {
   float* attn;       /* [B][Hkv][n_cap] a: cumulative window attention, group mean     */
   float* score;      /* [B][Hkv][n_cap] pooled contribution score; 0 past candidates   */
   uint8_t* topk;     /* [B][Hkv][n_cap] 1 where KV head kv's own top-m_s chose j       */
-  int32_t* kept_idx; /* [B][m_cap] kept positions, ascending                           */
+  int32_t* kept_idx; /* [B][m_cap] kept positions, ascending; [B][Hkv][m_cap] in the
+                        PER_HEAD selection mode                                        */
   int32_t* target;   /* [B][Hkv][n_cap] merge target of evicted j; -1 for kept j and
                         for tokens left without a target                              */
   float* gate;       /* [B][Hkv][n_cap] g of evicted j (0 for kept j)                  */
@@ -136,11 +144,13 @@ SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t str
  *   c  = a * ||v|| (Eq. 1), average-pooled over the candidates [0, n_b - m_r) (Sec. 3.2);
  *   per-KV-head top-m_s of c (Eq. 2), union over KV heads, trimmed to m_s by the mean score
  *   (Sec. 3.3), plus the recent window: m_b = floor(rho * n_b) kept positions shared by
- *   every head, ties to the lower position;
+ *   every head, ties to the lower position (PER_HEAD mode: each KV head's own top-m_s plus
+ *   the recent window, m_b positions per head);
  *   each evicted j routes to the kept token of its bucket with the largest a (Eq. 3, Sec. 3.4), gets
  *   g = clamp(cos(v_j, v_pi(j)), 0, 1) (Eq. 4) and is merged into V_c with weight g*a_j
  *   (Eq. 5); R = (a_i + sum g a_j) / a_i (Eq. 6); bias = alpha * ln(mean over KV heads R)
- *   (Sec. 3.6, GQA); K_c holds the kept keys unchanged.
+ *   (Sec. 3.6, GQA; PER_HEAD mode: alpha * ln R of each head's own entry); K_c holds the kept
+ *   keys unchanged.
  *
  * n_len     HOST array [B]: prefill lengths, W <= n_b <= n_cap.
  * rho       retention ratio in (0, 1]; m_b = floor(rho * n_b) (double), and
@@ -148,7 +158,7 @@ SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t str
  * K, V      [B][Hkv][n_cap][d]; rows >= n_b are ignored.
  * Q_obs     [B][Hq][W][d]: the last W query rows of each sequence.
  * K_c, V_c  [B][Hkv][m_cap][d] outputs; rows >= m_b untouched.
- * bias      [B][Hkv][m_cap] fp32 output (the same row for every KV head).
+ * bias      [B][Hkv][m_cap] fp32 output (the same row for every KV head in SHARED mode).
  * lengths   [B] int32 device output: m_b.
  * Errors: SELKV_ERR_INVALID_ARG for a NULL tensor, a bad shape, a misaligned pointer or a
  * budget outside the rules above; SELKV_ERR_UNSUPPORTED for d not in {64, 128} or a bucket

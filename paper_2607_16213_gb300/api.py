@@ -70,13 +70,14 @@ def alloc_compressed(shape: B.selkv_shape, device="cuda") -> CompressedCache:
                            lengths=torch.zeros((Bn,), dtype=torch.int32, device=device))
 
 
-def alloc_debug(shape: B.selkv_shape, device="cuda") -> dict:
+def alloc_debug(shape: B.selkv_shape, device="cuda", per_head: bool = False) -> dict:
+    """Debug outputs of selkv_compress (kept_idx is per KV head in the per-head mode)."""
     Bn, H, n, m = shape.batch, shape.num_kv_heads, shape.n_cap, shape.m_cap
     return dict(
         attn=torch.zeros((Bn, H, n), dtype=torch.float32, device=device),
         score=torch.zeros((Bn, H, n), dtype=torch.float32, device=device),
         topk=torch.zeros((Bn, H, n), dtype=torch.uint8, device=device),
-        kept_idx=torch.full((Bn, m), -1, dtype=torch.int32, device=device),
+        kept_idx=torch.full((Bn, H, m) if per_head else (Bn, m), -1, dtype=torch.int32, device=device),
         target=torch.full((Bn, H, n), -7, dtype=torch.int32, device=device),
         gate=torch.zeros((Bn, H, n), dtype=torch.float32, device=device),
         decision=torch.full((Bn, H, n), 9, dtype=torch.uint8, device=device),
@@ -91,7 +92,7 @@ def compress(shape: B.selkv_shape, n_len: Sequence[int], rho: float, K: torch.Te
     """selkv_compress on device tensors; returns the compressed cache (and debug outputs)."""
     params = params or B.selkv_params.defaults()
     out = out or alloc_compressed(shape, K.device)
-    dbg = alloc_debug(shape, K.device) if debug else None
+    dbg = alloc_debug(shape, K.device, per_head=params.select_mode == B.SELKV_SELECT_PER_HEAD) if debug else None
     ws = workspace or Workspace(B.selkv_compress_workspace_size(shape), K.device, stream)
     st = B.selkv_compress(shape, n_len, rho, params, K, V, Q_obs, out.K_c, out.V_c, out.bias,
                           out.lengths, dbg, ws.buf, ws.nbytes, stream)

@@ -88,9 +88,10 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.attn_part = score_uses_tc(s.dtype, s.head_dim, p.R) ? take(4 * B * Hkv * n * 4) : 0;
   p.vnorm = take(B * Hkv * n * 4);
   p.score = take(B * Hkv * n * 4);
-  p.kflag = take(B * n);
-  p.slot = take(B * n * 4);
-  p.kept_pos = take(B * (size_t)s.m_cap * 4);
+  // kept flags, slot maps: per sequence, or per KV head in the per-head mode (sized for that)
+  p.kflag = take(B * Hkv * n);
+  p.slot = take(B * Hkv * n * 4);
+  p.kept_pos = take(B * Hkv * (size_t)s.m_cap * 4);
   // merge targets per bucket, sized for the smallest bucket (the size is a call parameter)
   p.tau = take(B * Hkv * n * 4);
   p.atau = take(B * Hkv * n * 4);
@@ -190,7 +191,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   if (s.obs_window < 1 || s.n_cap < 1) return SELKV_ERR_INVALID_ARG;
   const selkv_params& p = *params;
   if (!std::isfinite(p.alpha) || p.pool_kernel < 1 || (p.pool_kernel & 1) == 0 || p.recent < 0 ||
-      p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1)
+      p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1 ||
+      p.select_mode < 0 || p.select_mode > 1)
     return SELKV_ERR_INVALID_ARG;
   if (p.bucket > 32) return SELKV_ERR_UNSUPPORTED;
   if (!(rho > 0.0 && rho <= 1.0)) return SELKV_ERR_INVALID_ARG;
@@ -235,6 +237,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.recent = p.recent;
   a.gate_mode = p.gate_mode;
   a.empty_bucket = p.empty_bucket;
+  a.per_head = p.select_mode == SELKV_SELECT_PER_HEAD ? 1 : 0;
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
   a.K = K;
   a.V = V;
@@ -286,7 +289,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   if (e == cudaSuccess)
     e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
-  g_launches += score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2;
+  g_launches += (score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2) -
+                (a.per_head ? 4 : 0);  // no union / trim kernels in the per-head mode
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

@@ -47,9 +47,11 @@ __global__ __launch_bounds__(kWarpsPerCta * 32) void route_kernel(CompressArgs a
   const int nb = (n + Bs - 1) / Bs;
   if (X >= nb) return;
   const int p = X * Bs + lane;
-  const bool kept = lane < Bs && p < n && a.kflag[(size_t)b * a.n_cap + p] != 0;
+  const bool valid = lane < Bs && p < n;
+  bool kept = valid && a.kflag[sel_unit(a, b, 0) * a.n_cap + p] != 0;
   for (int kv = 0; kv < a.Hkv; ++kv) {
     const size_t bk = (size_t)b * a.Hkv + kv;
+    if (a.per_head && kv > 0) kept = valid && a.kflag[bk * a.n_cap + p] != 0;
     float v = kept ? a.attn[bk * a.n_cap + p] : -INFINITY;
     int idx = kept ? p : INT_MAX;
     argmax_lanes(v, idx);
@@ -74,7 +76,7 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   const int slot = (int)(ks % a.m_cap);
   const int kv = (int)(ks / a.m_cap);
   if (kv >= a.Hkv || slot >= m) return;
-  const int pos = a.kept_pos[(size_t)b * a.m_cap + slot];
+  const int pos = a.kept_pos[sel_unit(a, b, kv) * a.m_cap + slot];
   const size_t bk = (size_t)b * a.Hkv + kv;
   if (pos < 0 || pos >= a.n_cap) {
     if (piece == 0 && tensor == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
@@ -199,7 +201,8 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   const int tr = (expand && eR < nb) ? tau_of[eR] : -1;
   const float al = (expand && eL >= 0) ? atau_of[eL] : 0.f;
   const float ar = (expand && eR < nb) ? atau_of[eR] : 0.f;
-  const bool keptX = inX && a.kflag[(size_t)b * a.n_cap + base + lane] != 0;
+  const size_t su = sel_unit(a, b, kv);
+  const bool keptX = inX && a.kflag[su * a.n_cap + base + lane] != 0;
   const float* A = a.attn + bk * a.n_cap;
   const float* vn = a.vnorm + bk * a.n_cap;
   const float AX = inX ? A[base + lane] : 0.f;
@@ -343,7 +346,7 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
 #pragma unroll
   for (int t = 0; t < PER; ++t) vm[t] = tot > 0.f ? (a_tau * vt[t] + num[t]) / tot : vt[t];
   const float R_tau = a_tau > 0.f ? tot / a_tau : 1.f;
-  const int slot = a.slot_of[(size_t)b * a.n_cap + tau];
+  const int slot = a.slot_of[su * a.n_cap + tau];
   if (slot < 0 || slot >= a.m_cap) {
     if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_COUNT);
     return;
@@ -361,11 +364,19 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   }
 }
 
-// bias[b][kv][slot] = alpha * ln(mean over KV heads of R[b][kv][slot])   (Sec. 3.6, GQA)
+// bias[b][kv][slot] = alpha * ln(mean over KV heads of R[b][kv][slot])   (Sec. 3.6, GQA);
+// per-head mode: alpha * ln R[b][kv][slot] of each head, no averaging (Sec. 3.6, MHA)
 __global__ __launch_bounds__(256) void bias_kernel(CompressArgs a) {
   const int b = blockIdx.y;
   const int slot = blockIdx.x * blockDim.x + threadIdx.x;
   if (slot >= a.seq_m[b]) return;
+  if (a.per_head) {
+    for (int kv = 0; kv < a.Hkv; ++kv) {
+      const size_t o = ((size_t)b * a.Hkv + kv) * a.m_cap + slot;
+      a.bias[o] = a.alpha * logf(a.ratio[o]);
+    }
+    return;
+  }
   float s = 0.f;
   for (int kv = 0; kv < a.Hkv; ++kv) s += a.ratio[((size_t)b * a.Hkv + kv) * a.m_cap + slot];
   const float bias = a.alpha * logf(s / (float)a.Hkv);

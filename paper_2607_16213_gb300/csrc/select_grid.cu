@@ -264,12 +264,14 @@ __global__ __launch_bounds__(kBlock) void union_kernel(CompressArgs a, SelectWs 
   }
 }
 
-// Kept flags (trimmed union, then the recent window) and per-block counts.  Grid (blocks, B).
+// Kept flags and per-block counts.  Shared mode: the trimmed union, then the recent window;
+// grid (blocks, B).  Per-head mode: the KV head's own top-m_s (whose choice it also reports),
+// then the recent window; grid (blocks, B * Hkv).
 __global__ __launch_bounds__(kBlock) void compact_count_kernel(CompressArgs a, SelectWs w) {
   __shared__ uint32_t s_cnt;
-  const int b = blockIdx.y;
+  const int u = blockIdx.y, b = a.per_head ? u / a.Hkv : u;
   const int n = a.seq_n[b], ncand = n - a.recent;
-  const RadixState st = w.trim[b];
+  const RadixState st = a.per_head ? w.topk[u] : w.trim[b];
   if (threadIdx.x == 0) s_cnt = 0u;
   __syncthreads();
   const int j0 = blockIdx.x * kSpan;
@@ -280,27 +282,34 @@ __global__ __launch_bounds__(kBlock) void compact_count_kernel(CompressArgs a, S
     if (j >= n) continue;
     bool kept = true;
     if (j < ncand) {
-      kept = w.uflag[(size_t)b * a.n_cap + j] != 0 &&
-             selected(__float_as_uint(w.tkey[(size_t)b * a.n_cap + j]), j, st);
+      if (a.per_head) {
+        kept = selected(__float_as_uint(a.score[(size_t)u * a.n_cap + j]), j, st);
+        if (a.dbg_topk != nullptr) a.dbg_topk[(size_t)u * a.n_cap + j] = kept ? 1 : 0;
+      } else {
+        kept = w.uflag[(size_t)b * a.n_cap + j] != 0 &&
+               selected(__float_as_uint(w.tkey[(size_t)b * a.n_cap + j]), j, st);
+      }
+    } else if (a.per_head && a.dbg_topk != nullptr) {
+      a.dbg_topk[(size_t)u * a.n_cap + j] = 0;
     }
-    a.kflag[(size_t)b * a.n_cap + j] = kept ? 1 : 0;
+    a.kflag[(size_t)u * a.n_cap + j] = kept ? 1 : 0;
     cnt += kept ? 1u : 0u;
   }
   atomicAdd(&s_cnt, cnt);
   __syncthreads();
-  if (threadIdx.x == 0) w.blkcnt[(size_t)b * gridDim.x + blockIdx.x] = s_cnt;
+  if (threadIdx.x == 0) w.blkcnt[(size_t)u * gridDim.x + blockIdx.x] = s_cnt;
 }
 
 // Slots in position order: block offset (sum of earlier blocks) + rank within the block.
 __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, SelectWs w) {
   __shared__ uint32_t wcnt[kBlock / 32 + 1];
   __shared__ uint32_t s_off;
-  const int b = blockIdx.y, blk = blockIdx.x;
+  const int u = blockIdx.y, blk = blockIdx.x, b = a.per_head ? u / a.Hkv : u;
   const int n = a.seq_n[b];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (warp == 0) {
     uint32_t s = 0;
-    for (int i = lane; i < blk; i += 32) s += w.blkcnt[(size_t)b * gridDim.x + i];
+    for (int i = lane; i < blk; i += 32) s += w.blkcnt[(size_t)u * gridDim.x + i];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
     if (lane == 0) s_off = s;
@@ -310,7 +319,7 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
   const int j0 = blk * kSpan;
   for (int e = 0; e < kPerThread; ++e) {
     const int j = j0 + e * kBlock + threadIdx.x;
-    const bool kept = j < n && a.kflag[(size_t)b * a.n_cap + j] != 0;
+    const bool kept = j < n && a.kflag[(size_t)u * a.n_cap + j] != 0;
     const unsigned bal = __ballot_sync(0xffffffffu, kept);
     if (lane == 0) wcnt[warp] = __popc(bal);
     __syncthreads();
@@ -328,10 +337,10 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
     __syncthreads();
     const uint32_t slot = base + wcnt[warp] + __popc(bal & ((1u << lane) - 1u));
     if (j < n) {
-      a.slot_of[(size_t)b * a.n_cap + j] = kept ? (int)slot : -1;
+      a.slot_of[(size_t)u * a.n_cap + j] = kept ? (int)slot : -1;
       if (kept && (int)slot < a.m_cap) {
-        a.kept_pos[(size_t)b * a.m_cap + slot] = j;
-        if (a.dbg_kept_idx != nullptr) a.dbg_kept_idx[(size_t)b * a.m_cap + slot] = j;
+        a.kept_pos[(size_t)u * a.m_cap + slot] = j;
+        if (a.dbg_kept_idx != nullptr) a.dbg_kept_idx[(size_t)u * a.m_cap + slot] = j;
       }
     }
     base += wcnt[kBlock / 32];
@@ -371,7 +380,7 @@ __global__ void select_init_kernel(CompressArgs a, SelectWs w) {
 size_t select_ws_bytes(int B, int Hkv, int n_cap) {
   const size_t units = (size_t)B * Hkv;
   const size_t blocks = (size_t)(n_cap + kSpan - 1) / kSpan;
-  return (units + B) * sizeof(RadixState) + (units + B) * 3 * kBins * 4 + (size_t)B * blocks * 4 +
+  return (units + B) * sizeof(RadixState) + (units + B) * 3 * kBins * 4 + units * blocks * 4 +
          (size_t)B * n_cap * 5 + 4 * 256;
 }
 
@@ -391,13 +400,14 @@ SelectWs carve_select_ws(void* base, int B, int Hkv, int n_cap) {
   w.trim_hist = reinterpret_cast<uint32_t*>(take((size_t)B * 3 * kBins * 4));
   w.hist_bytes = (size_t)(reinterpret_cast<char*>(w.trim_hist) - reinterpret_cast<char*>(w.topk_hist)) +
                  (size_t)B * 3 * kBins * 4;
-  w.blkcnt = reinterpret_cast<uint32_t*>(take((size_t)B * blocks * 4));
+  w.blkcnt = reinterpret_cast<uint32_t*>(take(units * blocks * 4));  // per selection unit
   w.tkey = reinterpret_cast<float*>(take((size_t)B * n_cap * 4));
   w.uflag = reinterpret_cast<uint8_t*>(take((size_t)B * n_cap));
   return w;
 }
 
-// Pooling and the whole selection: 10 kernels and one memset, all on `s`, no host sync.
+// Pooling and the whole selection: 10 kernels (6 in the per-head mode) and one memset, all
+// on `s`, no host sync.
 cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStream_t s) {
   const int units = a.B * a.Hkv;
   const int blocks = (a.n_cap + kSpan - 1) / kSpan;
@@ -408,12 +418,15 @@ cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStr
   for (int pass = 1; pass < 3; ++pass)
     hist_kernel<<<dim3(blocks, units), kBlock, 0, s>>>(a, w.topk, w.topk_hist, a.score, nullptr, a.Hkv, pass);
   tie_kernel<<<units, 1024, 0, s>>>(a, w.topk, a.score, nullptr, a.Hkv);
-  union_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w);
-  for (int pass = 1; pass < 3; ++pass)
-    hist_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w.trim, w.trim_hist, w.tkey, w.uflag, 1, pass);
-  tie_kernel<<<a.B, 1024, 0, s>>>(a, w.trim, w.tkey, w.uflag, 1);
-  compact_count_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w);
-  compact_write_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w);
+  if (!a.per_head) {  // union over KV heads and the trim (shared mode only)
+    union_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w);
+    for (int pass = 1; pass < 3; ++pass)
+      hist_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w.trim, w.trim_hist, w.tkey, w.uflag, 1, pass);
+    tie_kernel<<<a.B, 1024, 0, s>>>(a, w.trim, w.tkey, w.uflag, 1);
+  }
+  const int sel_units = a.per_head ? units : a.B;
+  compact_count_kernel<<<dim3(blocks, sel_units), kBlock, 0, s>>>(a, w);
+  compact_write_kernel<<<dim3(blocks, sel_units), kBlock, 0, s>>>(a, w);
   return cudaGetLastError();
 }
 

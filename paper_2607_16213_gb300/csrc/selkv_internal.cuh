@@ -98,6 +98,7 @@ struct CompressArgs {
   int nchunks;    // column chunks of the row-statistics pass
   float alpha;
   int pool_kernel, bucket, recent, gate_mode, empty_bucket;
+  int per_head;   // SELKV_SELECT_PER_HEAD: selection units are (b, kv), not b
   float scale_log2;  // log2(e) / sqrt(d)
   const void* K;
   const void* V;
@@ -124,9 +125,9 @@ struct CompressArgs {
   int attn_parts;    // 4: attn is the sum of attn_part, formed by the pooling kernel; 1: attn is final
   float* vnorm;      // [B][Hkv][n_cap]
   float* score;      // [B][Hkv][n_cap]
-  uint8_t* kflag;    // [B][n_cap] 1 = kept
-  int32_t* slot_of;  // [B][n_cap] slot of a kept position, -1 otherwise
-  int32_t* kept_pos; // [B][m_cap] position of each slot
+  uint8_t* kflag;    // [units][n_cap] 1 = kept (units: B, or B * Hkv in per-head mode)
+  int32_t* slot_of;  // [units][n_cap] slot of a kept position, -1 otherwise
+  int32_t* kept_pos; // [units][m_cap] position of each slot
   int nbk;           // buckets per sequence at n_cap: ceil(n_cap / bucket)
   int32_t* tau;      // [B][Hkv][nbk] merge target of each bucket (-1: no kept token)
   float* atau;       // [B][Hkv][nbk] a of that target
@@ -136,6 +137,11 @@ struct CompressArgs {
 // SM count used to plan grids and splits: fixed, so that workspace sizes and results do
 // not depend on which device answers (GB300: 152 SMs).
 constexpr int kPlanSMs = 152;
+
+// Selection unit of (b, kv): the sequence in the shared mode, the KV head in the per-head mode.
+__host__ __device__ __forceinline__ size_t sel_unit(const CompressArgs& a, int b, int kv) {
+  return a.per_head ? (size_t)b * a.Hkv + kv : (size_t)b;
+}
 
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
 

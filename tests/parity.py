@@ -48,7 +48,8 @@ def to_dev(x: np.ndarray, dtype: str) -> torch.Tensor:
 
 def params_of(p: O.Params) -> S.selkv_params:
     return S.selkv_params(alpha=p.alpha, pool_kernel=p.pool_kernel, bucket=p.bucket,
-                          recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket)
+                          recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket,
+                          select_mode=p.select_mode)
 
 
 def run_compress(wl: synth.Workload, x: dict, p: O.Params, rho=None, extra: int = 0):
@@ -123,6 +124,8 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
             stats.add("topk_near_ties", check_topk_choice(per_kv[kv], cp[kv], m_s, "top-k kv%d" % kv))
     else:
         assert not per_kv.any()
+    if p.select_mode == O.SELECT_PER_HEAD:
+        return _check_per_head(wl, x, host, b, p, stats, n, m, m_s, K, V, a, per_kv)
     # step 2b: union and trim (Sec. 3.3), continuing from the GPU's per-head choice
     sel = O.select_shared(cp, n, m_s, p.recent, follow_per_kv=per_kv)
     kept_idx_g = host["kept_idx"][b, :m].astype(np.int64)
@@ -191,6 +194,74 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
     err_v = np.abs(Vc_g - Vc_o) - tol
     assert err_v.max() <= 0, "V_c error beyond tolerance by %.3g" % err_v.max()
     return dict(n=n, m=m, K_c=K[:, kept_idx_g], V_c=Vc_o, bias=bias_o, a=a, kept_idx=kept_idx_g)
+
+
+def _check_steps_3_to_6(p, stats, kv, n, a_kv, V_kv, kept_g, tgt_g, gate_g, dec_g):
+    """Routing, gate and decision of one KV head against the oracle, continuing from the
+    GPU's kept set; returns the oracle's gates for that head's merge."""
+    ev = np.flatnonzero(~kept_g)
+    assert (tgt_g[kept_g] == -1).all() and (dec_g[kept_g] == 2).all()
+    own = O.route(a_kv, kept_g, p.bucket, p.empty_bucket)
+    diff = ev[tgt_g[ev] != own[ev]]
+    for j in diff:
+        tg, to = int(tgt_g[j]), int(own[j])
+        assert tg >= 0 and to >= 0 and kept_g[tg], "target of %d: gpu %d oracle %d" % (j, tg, to)
+        assert abs(tg // p.bucket - j // p.bucket) == abs(to // p.bucket - j // p.bucket)
+        assert abs(a_kv[tg] - a_kv[to]) <= DELTA * a_kv[to], "routing differs at %d" % j
+    stats.add("route_near_ties", int(diff.size))
+    g_o, sim_o, dec_o = O.gate(V_kv, tgt_g, p.gate_mode)
+    routed = ev[tgt_g[ev] >= 0]
+    err_g = np.abs(gate_g[routed] - g_o[routed])
+    stats["gate_abs_max"] = max(stats.get("gate_abs_max", 0.0), float(err_g.max(initial=0.0)))
+    assert err_g.max(initial=0.0) <= GATE_ATOL, "gate err %.3g" % err_g.max()
+    ddiff = ev[dec_g[ev] != dec_o[ev]]
+    assert (np.abs(sim_o[ddiff]) <= DELTA_SIM).all(), "merge/drop differs away from sim = 0"
+    stats.add("decision_near_ties", int(ddiff.size))
+    stats.add("evicted", int(ev.size))
+    stats.add("merged", int((dec_g[ev] == 1).sum()))
+    return g_o
+
+
+def _check_values(wl, host, b, m, Vc_o, what="V_c"):
+    Vc_g = host["V_c"][b, :, :m].astype(np.float64)
+    if wl.dtype == "bf16":
+        tol = np.abs(Vc_o) * 2.0 ** -8 + 1e-5
+    else:
+        tol = np.abs(Vc_o) * VC_FP32_RTOL + 1e-6
+    err_v = np.abs(Vc_g - Vc_o) - tol
+    assert err_v.max() <= 0, "%s error beyond tolerance by %.3g" % (what, err_v.max())
+
+
+def _check_per_head(wl, x, host, b, p, stats, n, m, m_s, K, V, a, per_kv):
+    """Per-head mode (Sec. 3.3 per-head selection, Sec. 3.6 per-head bias): each KV head's
+    kept set is its own top-m_s plus the recent window; steps 3-6 and the bias per head."""
+    Hkv, n_cand = K.shape[0], n - p.recent
+    tgt_g = host["target"][b, :, :n].astype(np.int64)
+    gate_g = host["gate"][b, :, :n].astype(np.float64)
+    dec_g = host["decision"][b, :, :n]
+    Vc_o = np.empty((Hkv, m, V.shape[2]))
+    R_o = np.empty((Hkv, m))
+    kept_idx_g = host["kept_idx"][b, :, :m].astype(np.int64)
+    for kv in range(Hkv):
+        kept_g = np.zeros(n, dtype=bool)
+        kept_g[kept_idx_g[kv]] = True
+        assert (np.diff(kept_idx_g[kv]) > 0).all() and int(kept_g.sum()) == m
+        expect = per_kv[kv].copy() if m_s > 0 else np.zeros(n_cand, dtype=bool)
+        assert (kept_g[:n_cand] == expect).all() and kept_g[n_cand:].all(), "head %d kept set" % kv
+        g_o = _check_steps_3_to_6(p, stats, kv, n, a[kv], V[kv], kept_g, tgt_g[kv], gate_g[kv], dec_g[kv])
+        Vc_o[kv], R_o[kv] = O.merge(a[kv], V[kv], kept_idx_g[kv], tgt_g[kv], g_o)
+        np.testing.assert_array_equal(host["K_c"][b, kv, :m], K[kv, kept_idx_g[kv]].astype(np.float32))
+    bias_o = O.per_head_bias(R_o, p.alpha)
+    R_g = host["ratio"][b, :, :m].astype(np.float64)
+    err_r = np.abs(R_g - R_o) / R_o
+    stats["ratio_rel_max"] = max(stats.get("ratio_rel_max", 0.0), float(err_r.max()))
+    assert err_r.max() <= RATIO_RTOL, "R rel err %.3g" % err_r.max()
+    err_b = np.abs(host["bias"][b, :, :m].astype(np.float64) - bias_o)
+    stats["bias_abs_max"] = max(stats.get("bias_abs_max", 0.0), float(err_b.max()))
+    assert err_b.max() <= BIAS_ATOL, "bias err %.3g" % err_b.max()
+    _check_values(wl, host, b, m, Vc_o)
+    K_c = np.stack([K[kv, kept_idx_g[kv]] for kv in range(Hkv)])
+    return dict(n=n, m=m, K_c=K_c, V_c=Vc_o, bias=bias_o, a=a, kept_idx=kept_idx_g)
 
 
 def check_decode(out_gpu: np.ndarray, want: np.ndarray, dtype: str, what: str = "decode"):

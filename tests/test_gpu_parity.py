@@ -107,9 +107,10 @@ def test_compress_parity_llama_layer():
     print("llama_layer", dict(st))
 
 
-def _decode_case(wl, layer, steps, use_bias=True):
+def _decode_case(wl, layer, steps, use_bias=True, p=None):
     x = synth.gen_layer(wl, layer, threads=8)
-    p = O.Params()
+    p = p or O.Params()
+    per_head = p.select_mode == O.SELECT_PER_HEAD
     cache, host, _ = run_compress(wl, x, p, extra=steps)
     dec = synth.gen_decode(wl, layer, steps)
     Kc0 = cache.K_c.double().cpu().numpy()
@@ -126,7 +127,12 @@ def _decode_case(wl, layer, steps, use_bias=True):
             L0 = int(lens0[b])
             Kc = np.concatenate([Kc0[b, :, :L0], dec["k_new"][:t + 1, b].transpose(1, 0, 2)], axis=1)
             Vc = np.concatenate([Vc0[b, :, :L0], dec["v_new"][:t + 1, b].transpose(1, 0, 2)], axis=1)
-            bs = np.concatenate([bias0[b, 0, :L0], np.zeros(t + 1)]) if use_bias else None
+            if not use_bias:
+                bs = None
+            elif per_head:   # one bias row per KV head (Sec. 3.6, per-head mode)
+                bs = np.concatenate([bias0[b, :, :L0], np.zeros((wl.num_kv_heads, t + 1))], axis=1)
+            else:
+                bs = np.concatenate([bias0[b, 0, :L0], np.zeros(t + 1)])
             want = O.decode(dec["q"][t, b], Kc, Vc, bs, L0 + t + 1)
             e = check_decode(out[b], want, wl.dtype, "step %d seq %d" % (t, b))
             worst = (max(worst[0], e[0]), max(worst[1], e[1]))
@@ -221,3 +227,62 @@ def test_repeat_runs_are_bitwise_identical():
     _, h2, _ = run_compress(wl, x, p)
     for k in ("attn", "score", "kept_idx", "target", "gate", "V_c", "bias"):
         np.testing.assert_array_equal(h1[k], h2[k], err_msg=k)
+
+
+# ---------------------------------------------------------------- per-head selection mode
+PER_HEAD = {
+    "tiny": SMALL["tiny"],                                          # fp32, G = 2
+    "bf16_mha": synth.WORKLOADS["llama_layer"].with_(name="bf16_mha", batch=2, n=2600,
+                                                     num_q_heads=4, num_kv_heads=4,
+                                                     ragged=(0.6, 1.0), seed=21),   # G = 1
+    "bf16_ragged": SMALL["bf16_ragged"],                            # bf16, G = 4
+}
+
+
+@pytest.mark.parametrize("name", list(PER_HEAD))
+def test_compress_parity_per_head(name):
+    """Sec. 3.3 per-head selection and Sec. 3.6 per-head bias against the oracle."""
+    wl = PER_HEAD[name]
+    x = synth.gen_layer(wl, 0)
+    p = O.Params(select_mode=O.SELECT_PER_HEAD)
+    _, host, _ = run_compress(wl, x, p)
+    st = Stats()
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p, stats=st)
+    print(name, dict(st))
+
+
+def test_per_head_gate_closed_is_eviction():
+    wl = PER_HEAD["bf16_mha"]
+    x = synth.gen_layer(wl, 1)
+    p = O.Params(select_mode=O.SELECT_PER_HEAD, gate_mode=O.GATE_CLOSED)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p)
+        m = int(host["lengths"][b])
+        for kv in range(wl.num_kv_heads):
+            kept = host["kept_idx"][b, kv, :m]
+            np.testing.assert_array_equal(host["V_c"][b, kv, :m], x["V"][b, kv][kept])
+        np.testing.assert_array_equal(host["bias"][b, :, :m], 0.0)
+
+
+def test_per_head_with_one_kv_head_matches_shared():
+    """One KV head: both selection modes give the same cache, bias and targets on the GPU."""
+    wl = SMALL["bf16_ragged"].with_(num_q_heads=4, num_kv_heads=1, batch=2, seed=22)
+    x = synth.gen_layer(wl, 0)
+    _, h_sh, _ = run_compress(wl, x, O.Params())
+    _, h_ph, _ = run_compress(wl, x, O.Params(select_mode=O.SELECT_PER_HEAD))
+    for b in range(wl.batch):
+        m = int(h_sh["lengths"][b])
+        n = int(x["n_len"][b])
+        np.testing.assert_array_equal(h_ph["kept_idx"][b, 0, :m], h_sh["kept_idx"][b, :m])
+        for k in ("K_c", "V_c", "bias", "ratio"):
+            np.testing.assert_array_equal(h_ph[k][b, :, :m], h_sh[k][b, :, :m])
+        np.testing.assert_array_equal(h_ph["target"][b, :, :n], h_sh["target"][b, :, :n])
+
+
+@pytest.mark.parametrize("name", ["tiny", "bf16_mha"])
+def test_decode_parity_per_head(name):
+    """Decode over per-head caches: each KV head's own rows and bias row."""
+    worst = _decode_case(PER_HEAD[name], 0, steps=3, p=O.Params(select_mode=O.SELECT_PER_HEAD))
+    print(name, "per-head decode worst max/mean abs", worst)
