@@ -98,7 +98,7 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------ oracle arm
-def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2):
+def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, per_head: bool = False):
     """Time the fp64 oracle on a bounded sample of one step of `wl`: compression of `layers`
     layers of sequence 0 and `decode_tokens` decode tokens over those layers; the rates are
     scaled to the whole step (all layers, all sequences, all decode steps)."""
@@ -113,7 +113,8 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2):
         K, V, Q = (x["K"][0].astype(np.float64), x["V"][0].astype(np.float64),
                    x["Q_obs"][0].astype(np.float64))
         t0 = time.perf_counter()
-        r = O.compress(K, V, Q, n, wl.rho)
+        r = O.compress(K, V, Q, n, wl.rho,
+                       O.Params(select_mode=O.SELECT_PER_HEAD if per_head else O.SELECT_SHARED))
         t_comp += time.perf_counter() - t0
         ncomp += 1
         dec = synth.gen_decode(wl.with_(batch=1), layer, decode_tokens)
@@ -121,7 +122,7 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2):
         for t in range(decode_tokens):
             Kc = np.concatenate([Kc, dec["k_new"][t, 0][:, None]], axis=1)
             Vc = np.concatenate([Vc, dec["v_new"][t, 0][:, None]], axis=1)
-            bias = np.concatenate([bias, [0.0]])
+            bias = np.concatenate([bias, np.zeros(bias.shape[:-1] + (1,))], axis=-1)
             t0 = time.perf_counter()
             O.decode(dec["q"][t, 0], Kc, Vc, bias, Kc.shape[1])
             t_dec += time.perf_counter() - t0
@@ -268,7 +269,8 @@ def run_gpu(args):
         wl = wl.with_(decode_steps=args.decode_steps)
     if args.layers is not None:
         wl = wl.with_(layers=args.layers)
-    params = S.selkv_params.defaults()
+    params = S.selkv_params.defaults(
+        select_mode=S.SELKV_SELECT_PER_HEAD if args.select_mode == "per_head" else S.SELKV_SELECT_SHARED)
     L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e)
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
@@ -386,7 +388,8 @@ def run_gpu(args):
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
         "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
                    "rho": wl.rho, "decode_steps": L.T, "q_heads": Hq, "kv_heads": Hkv,
-                   "head_dim": d, "obs_window": wl.obs_window, "parallelism": "replicas",
+                   "head_dim": d, "obs_window": wl.obs_window, "select_mode": args.select_mode,
+                   "parallelism": "replicas",
                    "l2": "inputs larger than L2: every token streams all layers' compressed "
                          "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
                    "cuda_graph": True},
@@ -407,7 +410,7 @@ def run_gpu(args):
     if e2e is not None:
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = oracle_sample(wl)
+        line["cpu_baseline"] = oracle_sample(wl, per_head=args.select_mode == "per_head")
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -495,10 +498,10 @@ def run_reference(args):
         wl = wl.with_(decode_steps=args.decode_steps)
     vals = []
     for _ in range(args.warmup):
-        oracle_sample(wl, layers=1, decode_tokens=1)
+        oracle_sample(wl, layers=1, decode_tokens=1, per_head=args.select_mode == "per_head")
     info = None
     for _ in range(args.steps):
-        info = oracle_sample(wl, layers=1, decode_tokens=1)
+        info = oracle_sample(wl, layers=1, decode_tokens=1, per_head=args.select_mode == "per_head")
         vals.append(info["value"])
     v = statistics.median(vals)
     tokens = wl.batch * wl.decode_steps
@@ -507,7 +510,7 @@ def run_reference(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
             "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
-                       "rho": wl.rho, "decode_steps": wl.decode_steps},
+                       "rho": wl.rho, "decode_steps": wl.decode_steps, "select_mode": args.select_mode},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
                              "sample": info["sample"]},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -526,6 +529,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-full", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--select-mode", default="shared", choices=["shared", "per_head"],
+                    help="token selection: shared (GQA union, the default) or per_head (MHA)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

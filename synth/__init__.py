@@ -71,6 +71,7 @@ _LLAMA = dict(dtype="bf16", num_q_heads=32, num_kv_heads=8, head_dim=128, obs_wi
 #: The five workloads.  tiny: single layer, fp32, GQA group 2.  llama_layer: one
 #: Llama-3-8B-shaped layer at 16k.  llama_32l_b4: 32 layers, batch 4, 32k.  long_100k: 32
 #: layers at 100k context.  sweep(): the batched serving grid with ragged lengths.
+#: longchat_mha_31k: the MHA shape of the per-head selection mode.
 WORKLOADS = {
     "tiny": Workload(name="tiny", dtype="fp32", batch=1, num_q_heads=4, num_kv_heads=2,
                      head_dim=64, obs_window=32, n=1024, layers=1, rho=0.25, decode_steps=16,
@@ -81,6 +82,10 @@ WORKLOADS = {
                              decode_steps=256, **_LLAMA),
     "long_100k": Workload(name="long_100k", batch=1, n=100000, layers=32, rho=0.25,
                           decode_steps=256, **_LLAMA),
+    # the paper's MHA setting (LongChat-7B-shaped: 32 query heads = 32 KV heads, 31,500-token
+    # inputs, W = 32), for the per-head selection mode
+    "longchat_mha_31k": Workload(name="longchat_mha_31k", batch=1, n=31500, layers=32, rho=0.25,
+                                 decode_steps=256, **dict(_LLAMA, num_kv_heads=32, obs_window=32)),
 }
 
 

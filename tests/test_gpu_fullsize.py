@@ -25,7 +25,7 @@ def built():
     S.library()
 
 
-def _decode_sampled(wl, cache, layer, seqs, steps=2):
+def _decode_sampled(wl, cache, layer, seqs, steps=2, per_head=False):
     """Decode `steps` tokens (appending) and compare sampled sequences with the oracle's decode
     over the GPU's compressed cache as it stood before each step."""
     dec = synth.gen_decode(wl, layer, steps)
@@ -41,7 +41,10 @@ def _decode_sampled(wl, cache, layer, seqs, steps=2):
             L = int(lens[b])
             K1 = np.concatenate([Kc[b, :, :L], dec["k_new"][t, b][:, None]], axis=1)
             V1 = np.concatenate([Vc[b, :, :L], dec["v_new"][t, b][:, None]], axis=1)
-            b1 = np.concatenate([bias[b, 0, :L], [0.0]])
+            if per_head:   # one bias row per KV head
+                b1 = np.concatenate([bias[b, :, :L], np.zeros((wl.num_kv_heads, 1))], axis=1)
+            else:
+                b1 = np.concatenate([bias[b, 0, :L], [0.0]])
             want = O.decode(dec["q"][t, b], K1, V1, b1, L + 1)
             check_decode(out[b], want, wl.dtype, "layer %d step %d seq %d" % (layer, t, b))
     torch.cuda.synchronize()
@@ -97,3 +100,16 @@ def test_serving_sweep_point(batch, n, rho):
     check_properties(wl, x, host, p)
     print(wl.name, dict(st))
     _decode_sampled(wl, cache, 0, picks, steps=2)
+
+
+def test_longchat_mha_layer_per_head():
+    """One layer of the MHA workload (32 query heads = 32 KV heads, n = 31,500) in the per-head
+    selection mode: stage-by-stage parity of every head, decode with per-head bias rows."""
+    wl = synth.WORKLOADS["longchat_mha_31k"]
+    x = synth.gen_layer(wl, 5, threads=16)
+    p = O.Params(select_mode=O.SELECT_PER_HEAD)
+    cache, host, _ = run_compress(wl, x, p, extra=wl.decode_steps + 1)
+    st = Stats()
+    check_sequence(wl, x, host, 0, p, stats=st)
+    print("longchat_mha_31k per-head", dict(st))
+    _decode_sampled(wl, cache, 5, [0], steps=2, per_head=True)
