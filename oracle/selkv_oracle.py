@@ -13,7 +13,8 @@ Merge-or-Drop and Attention Compensation"):
   each head's own top-m_s, Sec. 3.3 "Per-head selection") -> bucket-attention routing
   (Eq. 3, Sec. 3.4) -> soft cosine gate (Eq. 4, Sec. 3.5) -> gated attention-weighted merge (Eq. 5) -> attention
   ratio (Eq. 6) -> GQA bias alpha*log(mean_kv R) (Sec. 3.6) -> decode with the bias (Alg. 1,
-  last step).  RoPE repositioning (Eq. 7) is off, as in the paper's configuration (Sec. 4.1; Eq. 7 is Sec. 3.7).
+  last step).  RoPE repositioning (Eq. 7, Sec. 3.7) is off by default, as in the paper's
+  configuration (Sec. 4.1), and available as a parameter (R18).
 
 Readings where the paper is silent or garbled (each is a named choice, mirrored by the CUDA
 path):
@@ -43,6 +44,11 @@ path):
       averaging"): each KV head keeps its own top-m_s of its pooled score plus the recent
       window, routes, gates and merges against that set, and its bias is alpha * ln R of its
       own entries.  On a GQA model the G query heads of a KV head share its set.
+  R18 RoPE repositioning (Eq. 7, off by default as in Sec. 4.1): the kept key of slot s,
+      originally at position p_old = its index in the sequence, is re-embedded at p_new = s.
+      RoPE is the plain rotary embedding with base theta: frequency f in [0, d/2) rotates the
+      pair (k[f], k[f + d/2]) ("half" layout) or (k[2f], k[2f + 1]) ("interleaved" layout) by
+      the angle p * theta^(-2f/d).  Values are not rotated.
 """
 from __future__ import annotations
 
@@ -54,6 +60,7 @@ import numpy as np
 
 GATE_COSINE, GATE_OPEN, GATE_CLOSED = 0, 1, 2
 SELECT_SHARED, SELECT_PER_HEAD = 0, 1
+ROPE_OFF, ROPE_HALF, ROPE_INTERLEAVED = 0, 1, 2
 EMPTY_EXPAND, EMPTY_DROP = 0, 1
 DECISION_DROP, DECISION_MERGE = 0, 1
 
@@ -68,6 +75,8 @@ class Params:
     gate_mode: int = GATE_COSINE
     empty_bucket: int = EMPTY_EXPAND
     select_mode: int = SELECT_SHARED
+    rope: int = ROPE_OFF
+    rope_theta: float = 10000.0
 
 
 # ----------------------------------------------------------------------------------------
@@ -347,8 +356,8 @@ class CompressResult:
 def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
              params: Params = Params(), follow_per_kv=None, follow_kept=None,
              follow_target=None) -> CompressResult:
-    """Algorithm 1, steps 1-6, for one sequence of one layer (step 7, RoPE repositioning, is
-    off).  K, V: [Hkv][>=n][d]; Q: [Hq][W][d]; all float64.
+    """Algorithm 1 for one sequence of one layer (step 7, RoPE repositioning, only when
+    params.rope is set).  K, V: [Hkv][>=n][d]; Q: [Hq][W][d]; all float64.
 
     follow_* replace a discrete choice of the oracle by a given one (per-KV-head top-k
     masks, final kept mask, merge targets), so that a test can compare the continuous
@@ -382,9 +391,12 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
         g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
         Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # steps 5, 6
     bias = gqa_bias(R, params.alpha)
+    Kc = K[:, kept_idx].copy()
+    if params.rope != ROPE_OFF:                                         # step 7 (Eq. 7)
+        Kc = np.stack([reposition(Kc[kv], kept_idx, params.rope_theta, params.rope) for kv in range(Hkv)])
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=sel,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
-                          K_c=K[:, kept_idx].copy(), V_c=Vc, R=R, bias=bias)
+                          K_c=Kc, V_c=Vc, R=R, bias=bias)
 
 
 def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target):
@@ -407,10 +419,51 @@ def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, fol
         g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
         Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx[kv], t, g[kv])        # steps 5, 6
         Kc[kv] = K[kv, kept_idx[kv]]
+        if params.rope != ROPE_OFF:                                     # step 7 (Eq. 7)
+            Kc[kv] = reposition(Kc[kv], kept_idx[kv], params.rope_theta, params.rope)
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=None,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
                           K_c=Kc, V_c=Vc, R=R, bias=per_head_bias(R, params.alpha), per_head=True,
                           extra={"kept": kept})
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 7: RoPE repositioning
+# ----------------------------------------------------------------------------------------
+def rope_pairs(d: int, layout: int):
+    """Index pairs (x_f, y_f) rotated together by frequency f (R18)."""
+    f = np.arange(d // 2)
+    if layout == ROPE_HALF:
+        return f, f + d // 2
+    if layout == ROPE_INTERLEAVED:
+        return 2 * f, 2 * f + 1
+    raise ValueError("unknown RoPE layout")
+
+
+def rope(k: np.ndarray, pos: float, theta: float, layout: int) -> np.ndarray:
+    """RoPE(k, pos): rotate each pair of k ([..., d]) by pos * theta^(-2f/d)."""
+    k = np.asarray(k, dtype=np.float64)
+    d = k.shape[-1]
+    xi, yi = rope_pairs(d, layout)
+    ang = pos * theta ** (-2.0 * np.arange(d // 2) / d)
+    c, s = np.cos(ang), np.sin(ang)
+    out = k.copy()
+    out[..., xi] = k[..., xi] * c - k[..., yi] * s
+    out[..., yi] = k[..., xi] * s + k[..., yi] * c
+    return out
+
+
+def rope_inverse(k: np.ndarray, pos: float, theta: float, layout: int) -> np.ndarray:
+    """RoPE^{-1}(k, pos): the rotation by -pos * theta^(-2f/d)."""
+    return rope(k, -pos, theta, layout)
+
+
+def reposition(K_kept: np.ndarray, p_old: np.ndarray, theta: float, layout: int) -> np.ndarray:
+    """Eq. 7: k~_s = RoPE(RoPE^{-1}(k_s, p_old[s]), s) for the kept keys in slot order."""
+    out = np.empty_like(np.asarray(K_kept, dtype=np.float64))
+    for s_, (k, p) in enumerate(zip(K_kept, p_old)):
+        out[s_] = rope(rope_inverse(k, float(p), theta, layout), float(s_), theta, layout)
+    return out
 
 
 # ----------------------------------------------------------------------------------------

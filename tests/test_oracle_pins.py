@@ -462,3 +462,66 @@ def test_per_head_pipeline_invariants(seed):
     for kv in range(K.shape[0]):
         np.testing.assert_allclose(closed.V_c[kv], V[kv, closed.kept_idx[kv]], rtol=1e-15, atol=0)
     np.testing.assert_array_equal(closed.bias, 0.0)
+
+
+# ---------------------------------------------------------------- Eq. 7: RoPE repositioning
+@pytest.mark.parametrize("layout,key", [(O.ROPE_HALF, "half"), (O.ROPE_INTERLEAVED, "interleaved")])
+def test_rope_reposition_worked_example(layout, key):
+    gd = golden("rope_reposition.json")
+    got = O.rope(O.rope_inverse(np.array(gd["k"]), gd["p_old"], gd["theta"], layout), gd["p_new"],
+                 gd["theta"], layout)
+    np.testing.assert_allclose(got, gd[key], rtol=1e-14, atol=1e-15)
+    out = O.reposition(np.array([[9.0, 9, 9, 9], gd["k"]]), np.array([0, gd["p_old"]]), gd["theta"], layout)
+    np.testing.assert_allclose(out[1], gd[key], rtol=1e-14, atol=1e-15)   # slot 1 = p_new
+    np.testing.assert_allclose(out[0], [9.0, 9, 9, 9], rtol=0, atol=1e-15)  # no move: unchanged
+
+
+@pytest.mark.parametrize("layout", [O.ROPE_HALF, O.ROPE_INTERLEAVED])
+def test_rope_reposition_equals_embedding_at_new_position(layout):
+    """A key embedded at p_old and repositioned equals the raw key embedded at p_new,
+    computed independently with complex exponentials: (x + i y) e^{i p w_f}."""
+    r = rng(31)
+    d, theta = 16, 10000.0
+    raw = r.standard_normal((5, d))
+    p_old = np.array([3, 17, 400, 9999, 123456])
+    w = theta ** (-2.0 * np.arange(d // 2) / d)
+    xi, yi = O.rope_pairs(d, layout)
+
+    def embed(k, p):
+        z = (k[xi] + 1j * k[yi]) * np.exp(1j * p * w)
+        out = np.empty(d)
+        out[xi], out[yi] = z.real, z.imag
+        return out
+    K = np.stack([embed(raw[i], p_old[i]) for i in range(5)])
+    got = O.reposition(K, p_old, theta, layout)
+    want = np.stack([embed(raw[s], s) for s in range(5)])
+    np.testing.assert_allclose(got, want, rtol=1e-9, atol=1e-9)
+    np.testing.assert_allclose(np.linalg.norm(got, axis=1), np.linalg.norm(K, axis=1), rtol=1e-13)
+
+
+def test_rope_scores_depend_on_relative_position():
+    """q . k after RoPE depends only on the position difference, so a query at new position
+    t_new scores a repositioned key exactly as a query at t_new + (p_old - p_new) scored the
+    original (the property repositioning relies on)."""
+    r = rng(32)
+    d, theta = 8, 500.0
+    q, k = r.standard_normal(d), r.standard_normal(d)
+    for layout in (O.ROPE_HALF, O.ROPE_INTERLEAVED):
+        k_old = O.rope(k, 50, theta, layout)
+        k_new = O.reposition(np.stack([np.zeros(d), np.zeros(d), k_old]), np.array([0, 1, 50]), theta, layout)[2]
+        s_new = O.rope(q, 10, theta, layout) @ k_new          # query 8 positions after slot 2
+        s_old = O.rope(q, 58, theta, layout) @ k_old          # the same distance in the old frame
+        assert abs(s_new - s_old) < 1e-12
+
+
+def test_compress_with_rope_keeps_values_and_rotates_keys():
+    wl, K, V, Q, n = _tiny(seed=3)
+    base = O.compress(K, V, Q, n, wl.rho)
+    rot = O.compress(K, V, Q, n, wl.rho, O.Params(rope=O.ROPE_HALF, rope_theta=10000.0))
+    np.testing.assert_array_equal(rot.V_c, base.V_c)
+    np.testing.assert_array_equal(rot.bias, base.bias)
+    for kv in range(K.shape[0]):
+        np.testing.assert_allclose(rot.K_c[kv], O.reposition(K[kv, base.kept_idx], base.kept_idx,
+                                                             10000.0, O.ROPE_HALF), rtol=0, atol=0)
+        np.testing.assert_allclose(np.linalg.norm(rot.K_c[kv], axis=1), np.linalg.norm(base.K_c[kv], axis=1),
+                                   rtol=1e-12)
