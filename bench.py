@@ -270,7 +270,9 @@ def run_gpu(args):
     if args.layers is not None:
         wl = wl.with_(layers=args.layers)
     params = S.selkv_params.defaults(
-        select_mode=S.SELKV_SELECT_PER_HEAD if args.select_mode == "per_head" else S.SELKV_SELECT_SHARED)
+        select_mode=S.SELKV_SELECT_PER_HEAD if args.select_mode == "per_head" else S.SELKV_SELECT_SHARED,
+        rope={"off": S.SELKV_ROPE_OFF, "half": S.SELKV_ROPE_HALF,
+              "interleaved": S.SELKV_ROPE_INTERLEAVED}[args.rope], rope_theta=args.rope_theta)
     L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e)
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
@@ -389,6 +391,7 @@ def run_gpu(args):
         "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
                    "rho": wl.rho, "decode_steps": L.T, "q_heads": Hq, "kv_heads": Hkv,
                    "head_dim": d, "obs_window": wl.obs_window, "select_mode": args.select_mode,
+                   "rope": args.rope,
                    "parallelism": "replicas",
                    "l2": "inputs larger than L2: every token streams all layers' compressed "
                          "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
@@ -531,6 +534,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--select-mode", default="shared", choices=["shared", "per_head"],
                     help="token selection: shared (GQA union, the default) or per_head (MHA)")
+    ap.add_argument("--rope", default="off", choices=["off", "half", "interleaved"],
+                    help="RoPE repositioning of the kept keys (Eq. 7; off in the paper's configuration)")
+    ap.add_argument("--rope-theta", type=float, default=500000.0)
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -75,6 +75,18 @@ typedef enum selkv_empty_bucket { SELKV_EMPTY_EXPAND = 0, SELKV_EMPTY_DROP = 1 }
  * alpha * ln R of its own entries, without averaging across heads, Sec. 3.6). */
 typedef enum selkv_select_mode { SELKV_SELECT_SHARED = 0, SELKV_SELECT_PER_HEAD = 1 } selkv_select_mode;
 
+/* RoPE repositioning of the kept keys (Eq. 7, Sec. 3.7; off in the paper's configuration):
+ * the key kept in slot s, originally at position j, becomes RoPE(RoPE^{-1}(k, j), s) for the
+ * plain rotary embedding with base rope_theta, frequency f in [0, d/2) turning the pair
+ * (k[f], k[f + d/2]) (HALF layout) or (k[2f], k[2f + 1]) (INTERLEAVED layout) by
+ * p * rope_theta^(-2f/d).  Positions count from 0 at the first prefill token.  Decode does
+ * not rotate: the caller embeds new queries and keys at positions lengths[b], ... . */
+typedef enum selkv_rope {
+  SELKV_ROPE_OFF = 0,
+  SELKV_ROPE_HALF = 1,
+  SELKV_ROPE_INTERLEAVED = 2
+} selkv_rope;
+
 /* Device error bits (selkv_workspace_error). */
 #define SELKV_DEVERR_CAPACITY 0x1u /* decode append would pass m_cap: not appended       */
 #define SELKV_DEVERR_TIMEOUT 0x2u  /* a bounded wait gave up; the launch's output is void  */
@@ -103,6 +115,8 @@ typedef struct selkv_params {
   int32_t gate_mode;    /* selkv_gate_mode                                              */
   int32_t empty_bucket; /* selkv_empty_bucket                                           */
   int32_t select_mode;  /* selkv_select_mode, SHARED for GQA models (Sec. 4.1)            */
+  int32_t rope;         /* selkv_rope, OFF (Sec. 4.1)                                     */
+  float rope_theta;     /* rotary base, finite and > 0 when rope is on                    */
 } selkv_params;
 
 /* Optional device outputs of selkv_compress, for inspection and testing.  Any field may be
@@ -150,7 +164,7 @@ SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t str
  *   g = clamp(cos(v_j, v_pi(j)), 0, 1) (Eq. 4) and is merged into V_c with weight g*a_j
  *   (Eq. 5); R = (a_i + sum g a_j) / a_i (Eq. 6); bias = alpha * ln(mean over KV heads R)
  *   (Sec. 3.6, GQA; PER_HEAD mode: alpha * ln R of each head's own entry); K_c holds the kept
- *   keys unchanged.
+ *   keys, unchanged or, with params->rope, re-embedded at their slot positions (Eq. 7).
  *
  * n_len     HOST array [B]: prefill lengths, W <= n_b <= n_cap.
  * rho       retention ratio in (0, 1]; m_b = floor(rho * n_b) (double), and

@@ -64,7 +64,7 @@ SideStream* side_stream(cudaStream_t caller) {
 }
 
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
   int nchunks, R;
 };
 
@@ -96,6 +96,8 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.tau = take(B * Hkv * n * 4);
   p.atau = take(B * Hkv * n * 4);
   p.ratio = take(B * Hkv * (size_t)s.m_cap * 4);
+  // RoPE repositioning tables (used only with params->rope): coarse and fine (cos, sin)
+  p.rope_tab = take((size_t)(s.head_dim / 2) * (rope_coarse(s.n_cap) + 256) * 8);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
   p.total = off;
   return p;
@@ -192,7 +194,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   const selkv_params& p = *params;
   if (!std::isfinite(p.alpha) || p.pool_kernel < 1 || (p.pool_kernel & 1) == 0 || p.recent < 0 ||
       p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1 ||
-      p.select_mode < 0 || p.select_mode > 1)
+      p.select_mode < 0 || p.select_mode > 1 || p.rope < 0 || p.rope > 2 ||
+      (p.rope != 0 && !(std::isfinite(p.rope_theta) && p.rope_theta > 0.f)))
     return SELKV_ERR_INVALID_ARG;
   if (p.bucket > 32) return SELKV_ERR_UNSUPPORTED;
   if (!(rho > 0.0 && rho <= 1.0)) return SELKV_ERR_INVALID_ARG;
@@ -238,6 +241,9 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.gate_mode = p.gate_mode;
   a.empty_bucket = p.empty_bucket;
   a.per_head = p.select_mode == SELKV_SELECT_PER_HEAD ? 1 : 0;
+  a.rope = p.rope;
+  a.rope_theta = p.rope_theta;
+  a.rope_hi = rope_coarse(s.n_cap);
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
   a.K = K;
   a.V = V;
@@ -263,6 +269,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.tau = at<int32_t>(workspace, plan.tau);
   a.atau = at<float>(workspace, plan.atau);
   a.ratio = at<float>(workspace, plan.ratio);
+  a.rope_tab = at<float2>(workspace, plan.rope_tab);
   if (debug != nullptr) {
     a.dbg_topk = debug->topk;
     a.dbg_kept_idx = debug->kept_idx;
@@ -290,7 +297,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
   g_launches += (score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2) -
-                (a.per_head ? 4 : 0);  // no union / trim kernels in the per-head mode
+                (a.per_head ? 4 : 0) + (a.rope ? 1 : 0);  // no union / trim in per-head mode
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

@@ -6,8 +6,9 @@
 // Four kernels, in stream order:
 //   route  warp per (bucket X, sequence b): tau_X and a(tau_X) for every KV head (-1 / -inf
 //          for a bucket with no kept token);
-//   copy   every kept token's key and value row to its slot of K_c / V_c (keys unchanged) and
-//          ratio 1 for the slot; a thread per 16 bytes, coalesced;
+//   copy   every kept token's key and value row to its slot of K_c / V_c and ratio 1 for the
+//          slot; a thread per 16 bytes, coalesced.  Keys are unchanged, or, with RoPE
+//          repositioning (Eq. 7), turned by the shift from their position to their slot;
 //   merge  one-warp CTA per (non-empty bucket X, KV head, sequence b): the evicted tokens of X and of
 //          the empty buckets that the nearest-ring rule gives to X, in ascending position
 //          order, 16 at a time: g_j = clamp(cos(v_j, v_tau), 0, 1) and
@@ -19,6 +20,7 @@
 // No floating-point atomics: every sum has a fixed order, so results are reproducible.
 #include <climits>
 
+#include "ptx.cuh"
 #include "selkv_internal.cuh"
 
 namespace selkv {
@@ -62,10 +64,113 @@ __global__ __launch_bounds__(kWarpsPerCta * 32) void route_kernel(CompressArgs a
   }
 }
 
-// One thread per 16 bytes of a kept row: the K and V rows of slot s of (b, kv).
+// RoPE repositioning tables (Eq. 7): for frequency f, w_f = theta^(-2f/d); row c < rope_hi
+// holds (cos, sin) of (256 c) w_f for every f, and row rope_hi + c those of c w_f (c < 256),
+// so a shift e = 256 e_hi + e_lo composes two rows (the frequencies of a row are contiguous).
+// Angles are reduced modulo 2 pi in fp64 before the sine and cosine, so shifts of 10^5
+// positions stay accurate to fp32 rounding.
+constexpr int kRopeRowsPerThread = 8;
+__global__ void rope_table_kernel(CompressArgs a) {
+  const int half = a.D / 2, rows = a.rope_hi + 256;
+  const int groups = (rows + kRopeRowsPerThread - 1) / kRopeRowsPerThread;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= half * groups) return;
+  const int f = i % half, c0 = (i / half) * kRopeRowsPerThread;
+  const double w = pow((double)a.rope_theta, -2.0 * f / a.D);
+  const double two_pi = 6.283185307179586;
+  for (int c = c0; c < min(rows, c0 + kRopeRowsPerThread); ++c) {
+    const double e = c < a.rope_hi ? 256.0 * c : (double)(c - a.rope_hi);
+    double ang = e * w;
+    ang -= two_pi * rint(ang / two_pi);  // in [-pi, pi], exact to fp64 rounding
+    float sn, cs;
+    sincosf((float)ang, &sn, &cs);
+    a.rope_tab[(size_t)c * half + f] = make_float2(cs, sn);
+  }
+}
+
+// (cos, sin) of e w_f for the N consecutive frequencies f0 .. f0 + N - 1 (f0 and N even),
+// from the coarse and the fine row of e.
+template <int N>
+__device__ __forceinline__ void rope_angles(const CompressArgs& a, int f0, int e, float2 (&cs)[N]) {
+  const int half = a.D / 2;
+  const float4* h = reinterpret_cast<const float4*>(a.rope_tab + (size_t)(e >> 8) * half + f0);
+  const float4* l = reinterpret_cast<const float4*>(a.rope_tab + (size_t)(a.rope_hi + (e & 255)) * half + f0);
+#pragma unroll
+  for (int t = 0; t < N / 2; ++t) {
+    const float4 hv = h[t], lv = l[t];
+    cs[2 * t] = make_float2(hv.x * lv.x - hv.y * lv.y, hv.y * lv.x + hv.x * lv.y);
+    cs[2 * t + 1] = make_float2(hv.z * lv.z - hv.w * lv.w, hv.w * lv.z + hv.z * lv.w);
+  }
+}
+
+// Turn the pair (x, y) back by e w_f (from position j to slot j - e).
+__device__ __forceinline__ void rope_back(float& x, float& y, float2 cs) {
+  const float nx = x * cs.x + y * cs.y, ny = y * cs.x - x * cs.y;
+  x = nx;
+  y = ny;
+}
+
+template <typename T>
+__device__ __forceinline__ void unpack16(const uint4& u, float* x);
+template <>
+__device__ __forceinline__ void unpack16<__nv_bfloat16>(const uint4& u, float* x) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    x[2 * i] = bf16_lo(w[i]);
+    x[2 * i + 1] = bf16_hi(w[i]);
+  }
+}
+template <>
+__device__ __forceinline__ void unpack16<float>(const uint4& u, float* x) {
+  x[0] = __uint_as_float(u.x);
+  x[1] = __uint_as_float(u.y);
+  x[2] = __uint_as_float(u.z);
+  x[3] = __uint_as_float(u.w);
+}
+template <typename T>
+__device__ __forceinline__ void unpack8(const uint2& u, float* x);
+template <>
+__device__ __forceinline__ void unpack8<__nv_bfloat16>(const uint2& u, float* x) {
+  x[0] = bf16_lo(u.x);
+  x[1] = bf16_hi(u.x);
+  x[2] = bf16_lo(u.y);
+  x[3] = bf16_hi(u.y);
+}
+template <>
+__device__ __forceinline__ void unpack8<float>(const uint2& u, float* x) {
+  x[0] = __uint_as_float(u.x);
+  x[1] = __uint_as_float(u.y);
+}
+template <typename T>
+__device__ __forceinline__ uint2 pack8(const float* x);
+template <>
+__device__ __forceinline__ uint2 pack8<__nv_bfloat16>(const float* x) {
+  return make_uint2(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]));
+}
+template <>
+__device__ __forceinline__ uint2 pack8<float>(const float* x) {
+  return make_uint2(__float_as_uint(x[0]), __float_as_uint(x[1]));
+}
+template <typename T>
+__device__ __forceinline__ uint4 pack16(const float* x);
+template <>
+__device__ __forceinline__ uint4 pack16<__nv_bfloat16>(const float* x) {
+  return make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+}
+template <>
+__device__ __forceinline__ uint4 pack16<float>(const float* x) {
+  return make_uint4(__float_as_uint(x[0]), __float_as_uint(x[1]), __float_as_uint(x[2]), __float_as_uint(x[3]));
+}
+
+// One thread per 16 bytes of a kept row: the K and V rows of slot s of (b, kv).  With RoPE
+// repositioning a key row is turned by the shift e = position - slot; in the HALF layout the
+// thread of piece p takes the 8-byte pieces p and p + (pieces per row) of the row, so its
+// elements pair with the ones d/2 further on (the pairs (f, f + d/2)).
 template <typename T, int D>
 __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   constexpr int kPieces = D * (int)sizeof(T) / 16;  // 16-byte pieces per row
+  constexpr int kEpp = 16 / (int)sizeof(T);          // elements per piece
   const int b = blockIdx.y;
   const int m = a.seq_m[b];
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -84,7 +189,37 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   }
   const uint4* src = reinterpret_cast<const uint4*>(static_cast<const T*>(tensor ? a.V : a.K) + (bk * a.n_cap + pos) * D);
   uint4* dst = reinterpret_cast<uint4*>(static_cast<T*>(tensor ? a.Vc : a.Kc) + (bk * a.m_cap + slot) * D);
-  dst[piece] = src[piece];
+  if (tensor == 0 && a.rope != SELKV_ROPE_OFF) {
+    const int e = max(0, pos - slot);  // kept positions ascend with their slots
+    if (a.rope == SELKV_ROPE_HALF) {
+      // lane `piece` takes elements [h0, h0 + kEpp/2) of the first half and their partners
+      // (+ d/2) in the second half: 8-byte pieces, every lane of the row busy
+      constexpr int kH = kEpp / 2;
+      const int h0 = piece * kH;
+      const uint2* s8 = reinterpret_cast<const uint2*>(src);
+      uint2* d8 = reinterpret_cast<uint2*>(dst);
+      const uint2 xu = s8[piece], yu = s8[piece + kPieces];
+      float x[kH], y[kH];
+      unpack8<T>(xu, x);
+      unpack8<T>(yu, y);
+      float2 cs[kH];
+      rope_angles<kH>(a, h0, e, cs);
+#pragma unroll
+      for (int t = 0; t < kH; ++t) rope_back(x[t], y[t], cs[t]);
+      d8[piece] = pack8<T>(x);
+      d8[piece + kPieces] = pack8<T>(y);
+    } else {
+      float x[kEpp];
+      unpack16<T>(src[piece], x);
+      float2 cs[kEpp / 2];
+      rope_angles<kEpp / 2>(a, piece * kEpp / 2, e, cs);
+#pragma unroll
+      for (int t = 0; t < kEpp; t += 2) rope_back(x[t], x[t + 1], cs[t / 2]);
+      dst[piece] = pack16<T>(x);
+    }
+  } else {
+    dst[piece] = src[piece];
+  }
   if (piece == 0 && tensor == 0) {
     a.ratio[bk * a.m_cap + slot] = 1.f;
     if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = 1.f;
@@ -394,6 +529,11 @@ void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
 }  // namespace
 
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s) {
+  if (a.rope != SELKV_ROPE_OFF) {
+    const int groups = (a.rope_hi + 256 + kRopeRowsPerThread - 1) / kRopeRowsPerThread;
+    const int threads = a.D / 2 * groups;
+    rope_table_kernel<<<(threads + 127) / 128, 128, 0, s>>>(a);
+  }
   route_kernel<<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B), kWarpsPerCta * 32, 0, s>>>(a);
   if (a.dtype == SELKV_BF16) {
     if (a.D == 128) launch_merge_t<__nv_bfloat16, 128>(a, s);

@@ -99,6 +99,10 @@ struct CompressArgs {
   float alpha;
   int pool_kernel, bucket, recent, gate_mode, empty_bucket;
   int per_head;   // SELKV_SELECT_PER_HEAD: selection units are (b, kv), not b
+  int rope;       // selkv_rope layout of the kept keys' repositioning (0: off)
+  float rope_theta;
+  int rope_hi;    // coarse table entries: position shifts up to 256 * rope_hi
+  float2* rope_tab;  // [rope_hi + 256][d/2] (cos, sin) of e * w_f: rows e = 256 c (c < rope_hi), then e = c
   float scale_log2;  // log2(e) / sqrt(d)
   const void* K;
   const void* V;
@@ -142,6 +146,10 @@ constexpr int kPlanSMs = 152;
 __host__ __device__ __forceinline__ size_t sel_unit(const CompressArgs& a, int b, int kv) {
   return a.per_head ? (size_t)b * a.Hkv + kv : (size_t)b;
 }
+
+// Coarse RoPE table entries for caches of n_cap rows: position shifts e < n_cap split as
+// e = 256 e_hi + e_lo.
+__host__ __device__ constexpr int rope_coarse(int n_cap) { return n_cap / 256 + 1; }
 
 constexpr int kRowChunk = 512;  // columns per CTA in the row-statistics pass
 

@@ -49,7 +49,7 @@ def to_dev(x: np.ndarray, dtype: str) -> torch.Tensor:
 def params_of(p: O.Params) -> S.selkv_params:
     return S.selkv_params(alpha=p.alpha, pool_kernel=p.pool_kernel, bucket=p.bucket,
                           recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket,
-                          select_mode=p.select_mode)
+                          select_mode=p.select_mode, rope=p.rope, rope_theta=p.rope_theta)
 
 
 def run_compress(wl: synth.Workload, x: dict, p: O.Params, rho=None, extra: int = 0):
@@ -174,7 +174,8 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
     bias_o = O.gqa_bias(R_o, p.alpha)
 
     # continuous outputs
-    np.testing.assert_array_equal(host["K_c"][b, :, :m], K[:, kept_idx_g].astype(np.float32))
+    for kv in range(Hkv):
+        check_keys(host["K_c"][b, kv, :m], K[kv, kept_idx_g], kept_idx_g, p, wl.dtype)
     R_g = host["ratio"][b, :, :m].astype(np.float64)
     err_r = np.abs(R_g - R_o) / R_o
     stats["ratio_rel_max"] = max(stats.get("ratio_rel_max", 0.0), float(err_r.max()))
@@ -194,6 +195,20 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
     err_v = np.abs(Vc_g - Vc_o) - tol
     assert err_v.max() <= 0, "V_c error beyond tolerance by %.3g" % err_v.max()
     return dict(n=n, m=m, K_c=K[:, kept_idx_g], V_c=Vc_o, bias=bias_o, a=a, kept_idx=kept_idx_g)
+
+
+def check_keys(host_Kc: np.ndarray, K_kept: np.ndarray, kept_idx: np.ndarray, p: O.Params, dtype: str):
+    """K_c rows of one KV head: the kept keys unchanged, or with RoPE repositioning (Eq. 7) the
+    oracle's re-embedded keys within one rounding to the storage type plus fp32 angle error
+    (4e-6 of the row norm)."""
+    if p.rope == O.ROPE_OFF:
+        np.testing.assert_array_equal(host_Kc, K_kept.astype(np.float32))
+        return
+    want = O.reposition(K_kept, kept_idx, p.rope_theta, p.rope)
+    rel = 2.0 ** -8 if dtype == "bf16" else 0.0
+    tol = np.abs(want) * rel + 4e-6 * np.linalg.norm(want, axis=1, keepdims=True)
+    err = np.abs(host_Kc.astype(np.float64) - want) - tol
+    assert err.max() <= 0, "repositioned keys beyond tolerance by %.3g" % err.max()
 
 
 def _check_steps_3_to_6(p, stats, kv, n, a_kv, V_kv, kept_g, tgt_g, gate_g, dec_g):
@@ -250,7 +265,7 @@ def _check_per_head(wl, x, host, b, p, stats, n, m, m_s, K, V, a, per_kv):
         assert (kept_g[:n_cand] == expect).all() and kept_g[n_cand:].all(), "head %d kept set" % kv
         g_o = _check_steps_3_to_6(p, stats, kv, n, a[kv], V[kv], kept_g, tgt_g[kv], gate_g[kv], dec_g[kv])
         Vc_o[kv], R_o[kv] = O.merge(a[kv], V[kv], kept_idx_g[kv], tgt_g[kv], g_o)
-        np.testing.assert_array_equal(host["K_c"][b, kv, :m], K[kv, kept_idx_g[kv]].astype(np.float32))
+        check_keys(host["K_c"][b, kv, :m], K[kv, kept_idx_g[kv]], kept_idx_g[kv], p, wl.dtype)
     bias_o = O.per_head_bias(R_o, p.alpha)
     R_g = host["ratio"][b, :, :m].astype(np.float64)
     err_r = np.abs(R_g - R_o) / R_o

@@ -13,7 +13,7 @@ from oracle import selkv_oracle as O
 from paper_2607_16213_gb300 import api
 import paper_2607_16213_gb300 as S
 
-from parity import Stats, check_decode, check_properties, check_sequence, run_compress, to_dev
+from parity import Stats, check_decode, check_keys, check_properties, check_sequence, run_compress, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -113,3 +113,17 @@ def test_longchat_mha_layer_per_head():
     check_sequence(wl, x, host, 0, p, stats=st)
     print("longchat_mha_31k per-head", dict(st))
     _decode_sampled(wl, cache, 5, [0], steps=2, per_head=True)
+
+
+def test_long_100k_layer_rope_shifts():
+    """RoPE repositioning at 100k context (shifts up to ~75,000 positions, base 500,000): every
+    KV head's repositioned keys against the oracle's Eq. 7."""
+    wl = synth.WORKLOADS["long_100k"]
+    x = synth.gen_layer(wl, 9, threads=16)
+    p = O.Params(rope=O.ROPE_HALF, rope_theta=500000.0)
+    _, host, _ = run_compress(wl, x, p)
+    m = int(host["lengths"][0])
+    kept = host["kept_idx"][0, :m].astype(np.int64)
+    assert kept[-1] - (m - 1) > 50000
+    for kv in range(wl.num_kv_heads):
+        check_keys(host["K_c"][0, kv, :m], x["K"][0, kv][kept].astype(np.float64), kept, p, wl.dtype)

@@ -286,3 +286,28 @@ def test_decode_parity_per_head(name):
     """Decode over per-head caches: each KV head's own rows and bias row."""
     worst = _decode_case(PER_HEAD[name], 0, steps=3, p=O.Params(select_mode=O.SELECT_PER_HEAD))
     print(name, "per-head decode worst max/mean abs", worst)
+
+
+# ---------------------------------------------------------------- Eq. 7: RoPE repositioning
+@pytest.mark.parametrize("name,layout,mode", [
+    ("tiny", O.ROPE_HALF, O.SELECT_SHARED),
+    ("bf16_ragged", O.ROPE_HALF, O.SELECT_SHARED),
+    ("bf16_d64_g4", O.ROPE_INTERLEAVED, O.SELECT_SHARED),
+    ("fp32_d128", O.ROPE_INTERLEAVED, O.SELECT_SHARED),
+])
+def test_compress_rope_reposition(name, layout, mode):
+    wl = SMALL[name]
+    x = synth.gen_layer(wl, 3)
+    p = O.Params(rope=layout, rope_theta=10000.0, select_mode=mode)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p)
+
+
+def test_compress_rope_reposition_per_head_large_base():
+    wl = PER_HEAD["bf16_mha"]
+    x = synth.gen_layer(wl, 4)
+    p = O.Params(rope=O.ROPE_HALF, rope_theta=500000.0, select_mode=O.SELECT_PER_HEAD)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p)
