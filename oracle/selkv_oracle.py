@@ -49,6 +49,10 @@ path):
       RoPE is the plain rotary embedding with base theta: frequency f in [0, d/2) rotates the
       pair (k[f], k[f + d/2]) ("half" layout) or (k[2f], k[2f + 1]) ("interleaved" layout) by
       the angle p * theta^(-2f/d).  Values are not rotated.
+  R19 count bias (the KeepKV compensation Sec. 3.6 replaces, kept as a variant): M_i = number
+      of evicted tokens merged into kept token i (routed to i with g > 0); bias = alpha *
+      ln(1 + mean over KV heads of M_i) in the shared mode, alpha * ln(1 + M_{h,i}) per head
+      in the per-head mode (alpha = 1 is KeepKV's log(1 + M_i)).
 """
 from __future__ import annotations
 
@@ -61,6 +65,7 @@ import numpy as np
 GATE_COSINE, GATE_OPEN, GATE_CLOSED = 0, 1, 2
 SELECT_SHARED, SELECT_PER_HEAD = 0, 1
 ROPE_OFF, ROPE_HALF, ROPE_INTERLEAVED = 0, 1, 2
+BIAS_RATIO, BIAS_COUNT = 0, 1
 EMPTY_EXPAND, EMPTY_DROP = 0, 1
 DECISION_DROP, DECISION_MERGE = 0, 1
 
@@ -77,6 +82,7 @@ class Params:
     select_mode: int = SELECT_SHARED
     rope: int = ROPE_OFF
     rope_theta: float = 10000.0
+    bias_mode: int = BIAS_RATIO
 
 
 # ----------------------------------------------------------------------------------------
@@ -322,6 +328,21 @@ def gqa_bias(R: np.ndarray, alpha: float) -> np.ndarray:
     return alpha * np.log(R.mean(axis=0))
 
 
+def merge_counts(kept_idx: np.ndarray, target: np.ndarray, g: np.ndarray) -> np.ndarray:
+    """M_i: the evicted tokens merged into each kept token (routed to it with g > 0), in
+    kept_idx order (R19)."""
+    slot = {int(i): s for s, i in enumerate(kept_idx)}
+    M = np.zeros(kept_idx.shape[0])
+    for j in np.flatnonzero((target >= 0) & (g > 0)):
+        M[slot[int(target[j])]] += 1
+    return M
+
+
+def count_bias(M: np.ndarray, alpha: float, per_head: bool) -> np.ndarray:
+    """R19: alpha * ln(1 + mean_kv M) (shared; M [Hkv][m] -> [m]) or alpha * ln(1 + M) per head."""
+    return alpha * np.log1p(M) if per_head else alpha * np.log1p(M.mean(axis=0))
+
+
 def per_head_bias(R: np.ndarray, alpha: float) -> np.ndarray:
     """Sec. 3.6 with per-head selection: bias_{h,i} = alpha * ln R_{h,i}, no averaging across
     heads (R17).  R: [Hkv][m]; returns [Hkv][m]."""
@@ -390,7 +411,11 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
         target[kv] = t
         g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
         Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # steps 5, 6
-    bias = gqa_bias(R, params.alpha)
+    if params.bias_mode == BIAS_COUNT:
+        bias = count_bias(np.stack([merge_counts(kept_idx, target[kv], g[kv]) for kv in range(Hkv)]),
+                          params.alpha, per_head=False)
+    else:
+        bias = gqa_bias(R, params.alpha)
     Kc = K[:, kept_idx].copy()
     if params.rope != ROPE_OFF:                                         # step 7 (Eq. 7)
         Kc = np.stack([reposition(Kc[kv], kept_idx, params.rope_theta, params.rope) for kv in range(Hkv)])
@@ -423,7 +448,11 @@ def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, fol
             Kc[kv] = reposition(Kc[kv], kept_idx[kv], params.rope_theta, params.rope)
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=None,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
-                          K_c=Kc, V_c=Vc, R=R, bias=per_head_bias(R, params.alpha), per_head=True,
+                          K_c=Kc, V_c=Vc, R=R,
+                          bias=(count_bias(np.stack([merge_counts(kept_idx[kv], target[kv], g[kv])
+                                                     for kv in range(Hkv)]), params.alpha, per_head=True)
+                                if params.bias_mode == BIAS_COUNT else per_head_bias(R, params.alpha)),
+                          per_head=True,
                           extra={"kept": kept})
 
 

@@ -525,3 +525,35 @@ def test_compress_with_rope_keeps_values_and_rotates_keys():
                                                              10000.0, O.ROPE_HALF), rtol=0, atol=0)
         np.testing.assert_allclose(np.linalg.norm(rot.K_c[kv], axis=1), np.linalg.norm(base.K_c[kv], axis=1),
                                    rtol=1e-12)
+
+
+# ---------------------------------------------------------------- count bias (KeepKV, Sec. 3.6)
+def test_count_bias_worked_example():
+    """Hand-worked: kept tokens 0 and 3; tokens 1, 2 routed to 0 with g = 0.5 and 0 (only one
+    merges), token 4 routed to 3 with g = 1: M = (1, 1) for this head; with a second head
+    where M = (3, 0), the shared bias is ln(1 + 2) and ln(1 + 0.5); per head it is ln 2, ln 2
+    and ln 4, ln 1 (alpha = 1, KeepKV's log(1 + M))."""
+    kept = np.array([0, 3])
+    target = np.array([-1, 0, 0, -1, 3])
+    g = np.array([0.0, 0.5, 0.0, 0.0, 1.0])
+    M0 = O.merge_counts(kept, target, g)
+    assert M0.tolist() == [1.0, 1.0]
+    M = np.stack([M0, np.array([3.0, 0.0])])
+    np.testing.assert_allclose(O.count_bias(M, 1.0, per_head=False), [math.log(3.0), math.log(1.5)], rtol=1e-15)
+    np.testing.assert_allclose(O.count_bias(M, 1.0, per_head=True),
+                               [[math.log(2.0), math.log(2.0)], [math.log(4.0), 0.0]], rtol=1e-15)
+
+
+def test_count_bias_compress_matches_explicit_counts():
+    wl, K, V, Q, n = _tiny(seed=4)
+    for mode in (O.SELECT_SHARED, O.SELECT_PER_HEAD):
+        r = O.compress(K, V, Q, n, wl.rho, O.Params(bias_mode=O.BIAS_COUNT, select_mode=mode))
+        Hkv = K.shape[0]
+        kept = r.kept_idx if mode == O.SELECT_PER_HEAD else np.stack([r.kept_idx] * Hkv)
+        M = np.array([[sum(1 for j in range(n) if r.target[kv, j] == i and r.g[kv, j] > 0) for i in kept[kv]]
+                      for kv in range(Hkv)], dtype=float)
+        want = 0.5 * np.log(1.0 + (M if mode == O.SELECT_PER_HEAD else M.mean(axis=0)))
+        np.testing.assert_allclose(r.bias, want, rtol=1e-14, atol=0)
+        closed = O.compress(K, V, Q, n, wl.rho, O.Params(bias_mode=O.BIAS_COUNT, select_mode=mode,
+                                                          gate_mode=O.GATE_CLOSED))
+        np.testing.assert_array_equal(closed.bias, 0.0)   # nothing merges, so no count
