@@ -81,6 +81,11 @@ typedef enum selkv_select_mode { SELKV_SELECT_SHARED = 0, SELKV_SELECT_PER_HEAD 
  * (k[f], k[f + d/2]) (HALF layout) or (k[2f], k[2f + 1]) (INTERLEAVED layout) by
  * p * rope_theta^(-2f/d).  Positions count from 0 at the first prefill token.  Decode does
  * not rotate: the caller embeds new queries and keys at positions lengths[b], ... . */
+/* Attention compensation (Sec. 3.6): RATIO is SelKV's alpha * ln R (Eq. 6); COUNT is the
+ * KeepKV-style alpha * ln(1 + M), M the evicted tokens merged into the kept token (routed to
+ * it with g > 0), averaged over KV heads in SHARED mode (alpha = 1: KeepKV's log(1 + M)). */
+typedef enum selkv_bias_mode { SELKV_BIAS_RATIO = 0, SELKV_BIAS_COUNT = 1 } selkv_bias_mode;
+
 typedef enum selkv_rope {
   SELKV_ROPE_OFF = 0,
   SELKV_ROPE_HALF = 1,
@@ -117,6 +122,7 @@ typedef struct selkv_params {
   int32_t select_mode;  /* selkv_select_mode, SHARED for GQA models (Sec. 4.1)            */
   int32_t rope;         /* selkv_rope, OFF (Sec. 4.1)                                     */
   float rope_theta;     /* rotary base, finite and > 0 when rope is on                    */
+  int32_t bias_mode;    /* selkv_bias_mode, RATIO (Sec. 3.6)                              */
 } selkv_params;
 
 /* Optional device outputs of selkv_compress, for inspection and testing.  Any field may be

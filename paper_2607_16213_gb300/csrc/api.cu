@@ -64,7 +64,7 @@ SideStream* side_stream(cudaStream_t caller) {
 }
 
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, mcount, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
   int nchunks, R;
 };
 
@@ -96,6 +96,7 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.tau = take(B * Hkv * n * 4);
   p.atau = take(B * Hkv * n * 4);
   p.ratio = take(B * Hkv * (size_t)s.m_cap * 4);
+  p.mcount = take(B * Hkv * (size_t)s.m_cap * 4);
   // RoPE repositioning tables (used only with params->rope): coarse and fine (cos, sin)
   p.rope_tab = take((size_t)(s.head_dim / 2) * (rope_coarse(s.n_cap) + 256) * 8);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
@@ -194,7 +195,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   const selkv_params& p = *params;
   if (!std::isfinite(p.alpha) || p.pool_kernel < 1 || (p.pool_kernel & 1) == 0 || p.recent < 0 ||
       p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1 ||
-      p.select_mode < 0 || p.select_mode > 1 || p.rope < 0 || p.rope > 2 ||
+      p.select_mode < 0 || p.select_mode > 1 || p.rope < 0 || p.rope > 2 || p.bias_mode < 0 || p.bias_mode > 1 ||
       (p.rope != 0 && !(std::isfinite(p.rope_theta) && p.rope_theta > 0.f)))
     return SELKV_ERR_INVALID_ARG;
   if (p.bucket > 32) return SELKV_ERR_UNSUPPORTED;
@@ -242,6 +243,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.empty_bucket = p.empty_bucket;
   a.per_head = p.select_mode == SELKV_SELECT_PER_HEAD ? 1 : 0;
   a.rope = p.rope;
+  a.bias_count = p.bias_mode == SELKV_BIAS_COUNT ? 1 : 0;
   a.rope_theta = p.rope_theta;
   a.rope_hi = rope_coarse(s.n_cap);
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
@@ -269,6 +271,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.tau = at<int32_t>(workspace, plan.tau);
   a.atau = at<float>(workspace, plan.atau);
   a.ratio = at<float>(workspace, plan.ratio);
+  a.mcount = at<float>(workspace, plan.mcount);
   a.rope_tab = at<float2>(workspace, plan.rope_tab);
   if (debug != nullptr) {
     a.dbg_topk = debug->topk;

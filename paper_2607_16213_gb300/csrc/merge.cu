@@ -222,6 +222,7 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   }
   if (piece == 0 && tensor == 0) {
     a.ratio[bk * a.m_cap + slot] = 1.f;
+    a.mcount[bk * a.m_cap + slot] = 0.f;
     if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = 1.f;
     const size_t o = bk * a.n_cap + pos;
     if (a.dbg_target) a.dbg_target[o] = -1;
@@ -412,6 +413,7 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
 #pragma unroll
   for (int t = 0; t < PER; ++t) num[t] = 0.f;
   float den = 0.f;
+  int merged = 0;             // contributors with g > 0 (the count bias)
   const int own = lane >> 1;  // contributor owned by this lane pair within a batch
   for (int e = lo_b; e <= hi_b; ++e) {
     const int eb = e * Bs;
@@ -460,6 +462,7 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
         g = fminf(fmaxf(sim, 0.f), 1.f);
       }
       const float w = ob >= 0 ? g * ak : 0.f;
+      merged += __popc(__ballot_sync(0xffffffffu, ob >= 0 && g > 0.f) & 0x55555555u);
       if (ob >= 0 && (lane & 1) == 0) {
         const size_t o = bk * a.n_cap + eb + ob;
         if (a.dbg_target) a.dbg_target[o] = tau;
@@ -495,26 +498,30 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   }
   if (lane == 0) {
     a.ratio[bk * a.m_cap + slot] = R_tau;
+    a.mcount[bk * a.m_cap + slot] = (float)merged;
     if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = R_tau;
   }
 }
 
 // bias[b][kv][slot] = alpha * ln(mean over KV heads of R[b][kv][slot])   (Sec. 3.6, GQA);
-// per-head mode: alpha * ln R[b][kv][slot] of each head, no averaging (Sec. 3.6, MHA)
+// per-head mode: alpha * ln R[b][kv][slot] of each head, no averaging (Sec. 3.6, MHA).  The
+// count variant uses ln(1 + M) of the merge counts M instead of ln R.
 __global__ __launch_bounds__(256) void bias_kernel(CompressArgs a) {
   const int b = blockIdx.y;
   const int slot = blockIdx.x * blockDim.x + threadIdx.x;
   if (slot >= a.seq_m[b]) return;
+  const float* src = a.bias_count ? a.mcount : a.ratio;
   if (a.per_head) {
     for (int kv = 0; kv < a.Hkv; ++kv) {
       const size_t o = ((size_t)b * a.Hkv + kv) * a.m_cap + slot;
-      a.bias[o] = a.alpha * logf(a.ratio[o]);
+      a.bias[o] = a.alpha * (a.bias_count ? log1pf(src[o]) : logf(src[o]));
     }
     return;
   }
   float s = 0.f;
-  for (int kv = 0; kv < a.Hkv; ++kv) s += a.ratio[((size_t)b * a.Hkv + kv) * a.m_cap + slot];
-  const float bias = a.alpha * logf(s / (float)a.Hkv);
+  for (int kv = 0; kv < a.Hkv; ++kv) s += src[((size_t)b * a.Hkv + kv) * a.m_cap + slot];
+  const float mean = s / (float)a.Hkv;
+  const float bias = a.alpha * (a.bias_count ? log1pf(mean) : logf(mean));
   for (int kv = 0; kv < a.Hkv; ++kv) a.bias[((size_t)b * a.Hkv + kv) * a.m_cap + slot] = bias;
 }
 

@@ -100,6 +100,7 @@ struct CompressArgs {
   int pool_kernel, bucket, recent, gate_mode, empty_bucket;
   int per_head;   // SELKV_SELECT_PER_HEAD: selection units are (b, kv), not b
   int rope;       // selkv_rope layout of the kept keys' repositioning (0: off)
+  int bias_count; // SELKV_BIAS_COUNT: bias from merge counts instead of ratios
   float rope_theta;
   int rope_hi;    // coarse table entries: position shifts up to 256 * rope_hi
   float2* rope_tab;  // [rope_hi + 256][d/2] (cos, sin) of e * w_f: rows e = 256 c (c < rope_hi), then e = c
@@ -136,6 +137,7 @@ struct CompressArgs {
   int32_t* tau;      // [B][Hkv][nbk] merge target of each bucket (-1: no kept token)
   float* atau;       // [B][Hkv][nbk] a of that target
   float* ratio;      // [B][Hkv][m_cap] attention ratio R of each slot
+  float* mcount;     // [B][Hkv][m_cap] evicted tokens merged into each slot (g > 0)
 };
 
 // SM count used to plan grids and splits: fixed, so that workspace sizes and results do

@@ -49,7 +49,8 @@ def to_dev(x: np.ndarray, dtype: str) -> torch.Tensor:
 def params_of(p: O.Params) -> S.selkv_params:
     return S.selkv_params(alpha=p.alpha, pool_kernel=p.pool_kernel, bucket=p.bucket,
                           recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket,
-                          select_mode=p.select_mode, rope=p.rope, rope_theta=p.rope_theta)
+                          select_mode=p.select_mode, rope=p.rope, rope_theta=p.rope_theta,
+                          bias_mode=p.bias_mode)
 
 
 def run_compress(wl: synth.Workload, x: dict, p: O.Params, rho=None, extra: int = 0):
@@ -171,7 +172,11 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
         stats.add("evicted", int(ev.size))
         stats.add("merged", int((dec_g[kv, ev] == 1).sum()))
         Vc_o[kv], R_o[kv] = O.merge(a[kv], V[kv], kept_idx_g, tgt_g[kv], g_o)
-    bias_o = O.gqa_bias(R_o, p.alpha)
+    if p.bias_mode == O.BIAS_COUNT:   # counts from the GPU's own targets and gates
+        M = np.stack([O.merge_counts(kept_idx_g, tgt_g[kv], gate_g[kv]) for kv in range(Hkv)])
+        bias_o = O.count_bias(M, p.alpha, per_head=False)
+    else:
+        bias_o = O.gqa_bias(R_o, p.alpha)
 
     # continuous outputs
     for kv in range(Hkv):
@@ -266,7 +271,11 @@ def _check_per_head(wl, x, host, b, p, stats, n, m, m_s, K, V, a, per_kv):
         g_o = _check_steps_3_to_6(p, stats, kv, n, a[kv], V[kv], kept_g, tgt_g[kv], gate_g[kv], dec_g[kv])
         Vc_o[kv], R_o[kv] = O.merge(a[kv], V[kv], kept_idx_g[kv], tgt_g[kv], g_o)
         check_keys(host["K_c"][b, kv, :m], K[kv, kept_idx_g[kv]], kept_idx_g[kv], p, wl.dtype)
-    bias_o = O.per_head_bias(R_o, p.alpha)
+    if p.bias_mode == O.BIAS_COUNT:
+        M = np.stack([O.merge_counts(kept_idx_g[kv], tgt_g[kv], gate_g[kv]) for kv in range(Hkv)])
+        bias_o = O.count_bias(M, p.alpha, per_head=True)
+    else:
+        bias_o = O.per_head_bias(R_o, p.alpha)
     R_g = host["ratio"][b, :, :m].astype(np.float64)
     err_r = np.abs(R_g - R_o) / R_o
     stats["ratio_rel_max"] = max(stats.get("ratio_rel_max", 0.0), float(err_r.max()))

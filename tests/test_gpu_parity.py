@@ -311,3 +311,18 @@ def test_compress_rope_reposition_per_head_large_base():
     _, host, _ = run_compress(wl, x, p)
     for b in range(wl.batch):
         check_sequence(wl, x, host, b, p)
+
+
+# ---------------------------------------------------------------- count bias (KeepKV variant)
+@pytest.mark.parametrize("name,mode,alpha", [
+    ("bf16_ragged", O.SELECT_SHARED, 1.0),
+    ("tiny", O.SELECT_SHARED, 0.5),
+    ("bf16_mha", O.SELECT_PER_HEAD, 1.0),
+])
+def test_compress_count_bias(name, mode, alpha):
+    wl = SMALL.get(name) or PER_HEAD[name]
+    x = synth.gen_layer(wl, 5)
+    p = O.Params(bias_mode=O.BIAS_COUNT, select_mode=mode, alpha=alpha)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p)
