@@ -53,6 +53,9 @@ path):
       of evicted tokens merged into kept token i (routed to i with g > 0); bias = alpha *
       ln(1 + mean over KV heads of M_i) in the shared mode, alpha * ln(1 + M_{h,i}) per head
       in the per-head mode (alpha = 1 is KeepKV's log(1 + M_i)).
+  R20 full cosine routing (the alternative Sec. 3.4 prices at O(H |S| |E| d)): pi(j) is the
+      kept token of the head with the largest cos(v_j, v_i) over all kept tokens, with the
+      original (pre-merge) values; ties to the lower position; a zero norm gives cosine 0.
 """
 from __future__ import annotations
 
@@ -66,6 +69,7 @@ GATE_COSINE, GATE_OPEN, GATE_CLOSED = 0, 1, 2
 SELECT_SHARED, SELECT_PER_HEAD = 0, 1
 ROPE_OFF, ROPE_HALF, ROPE_INTERLEAVED = 0, 1, 2
 BIAS_RATIO, BIAS_COUNT = 0, 1
+ROUTE_BUCKET, ROUTE_COSINE = 0, 1
 EMPTY_EXPAND, EMPTY_DROP = 0, 1
 DECISION_DROP, DECISION_MERGE = 0, 1
 
@@ -83,6 +87,7 @@ class Params:
     rope: int = ROPE_OFF
     rope_theta: float = 10000.0
     bias_mode: int = BIAS_RATIO
+    routing: int = ROUTE_BUCKET
 
 
 # ----------------------------------------------------------------------------------------
@@ -269,6 +274,25 @@ def route(a_kv: np.ndarray, kept: np.ndarray, bucket: int, empty_policy: int) ->
     return target
 
 
+def route_cosine(V_kv: np.ndarray, kept: np.ndarray) -> np.ndarray:
+    """Full cosine routing (R20): every evicted j goes to the kept i with the largest
+    cos(v_j, v_i) (ties to the lower i; a zero norm gives cosine 0).  -1 for kept tokens."""
+    V_kv = np.asarray(V_kv, dtype=np.float64)
+    n = kept.shape[0]
+    ki = np.flatnonzero(kept)
+    target = np.full(n, -1, dtype=np.int64)
+    if ki.size == 0:
+        return target
+    norms = np.linalg.norm(V_kv[:n], axis=1)
+    Vk = V_kv[ki]
+    nk = norms[ki]
+    for j in np.flatnonzero(~kept):
+        cos = np.where((nk > 0) & (norms[j] > 0), (Vk @ V_kv[j]) / np.where(nk > 0, nk, 1.0) /
+                       (norms[j] if norms[j] > 0 else 1.0), 0.0)
+        target[j] = int(ki[int(np.argmax(cos))])   # argmax keeps the first (lowest) maximum
+    return target
+
+
 # ----------------------------------------------------------------------------------------
 # Eq. 4: soft cosine gate
 # ----------------------------------------------------------------------------------------
@@ -407,7 +431,7 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     R = np.ones((Hkv, kept_idx.size))
     for kv in range(Hkv):
         t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
-             else route(a[kv], sel.kept, params.bucket, params.empty_bucket))   # step 3
+             else _route(a[kv], V[kv], sel.kept, params))                      # step 3
         target[kv] = t
         g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
         Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # steps 5, 6
@@ -422,6 +446,13 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=sel,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
                           K_c=Kc, V_c=Vc, R=R, bias=bias)
+
+
+def _route(a_kv, V_kv, kept, params):
+    """Step 3 of Algorithm 1 under the routing of params (Eq. 3 buckets, or R20 cosine)."""
+    if params.routing == ROUTE_COSINE:
+        return route_cosine(V_kv, kept)
+    return route(a_kv, kept, params.bucket, params.empty_bucket)
 
 
 def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target):
@@ -439,7 +470,7 @@ def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, fol
     R = np.ones((Hkv, m))
     for kv in range(Hkv):
         t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
-             else route(a[kv], kept[kv], params.bucket, params.empty_bucket))  # step 3
+             else _route(a[kv], V[kv], kept[kv], params))                      # step 3
         target[kv] = t
         g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
         Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx[kv], t, g[kv])        # steps 5, 6

@@ -557,3 +557,53 @@ def test_count_bias_compress_matches_explicit_counts():
         closed = O.compress(K, V, Q, n, wl.rho, O.Params(bias_mode=O.BIAS_COUNT, select_mode=mode,
                                                           gate_mode=O.GATE_CLOSED))
         np.testing.assert_array_equal(closed.bias, 0.0)   # nothing merges, so no count
+
+
+# ---------------------------------------------------------------- full cosine routing (Sec. 3.4)
+def test_cosine_routing_worked_example():
+    """Hand-worked: kept tokens 0 (v = (1, 0)) and 2 (v = (0, 1)); token 1 = (1, 1) ties
+    (cos 1/sqrt 2 with both) and goes to the lower position 0; token 3 = (-1, 3) is closer to
+    (0, 1); token 4 = (0, 0) has cosine 0 with both and goes to 0."""
+    V = np.array([[1.0, 0], [1, 1], [0, 1], [-1, 3], [0, 0]])
+    kept = np.array([True, False, True, False, False])
+    assert O.route_cosine(V, kept).tolist() == [-1, 0, -1, 2, 0]
+
+
+def test_cosine_routing_brute_force():
+    r = rng(41)
+    n, d = 120, 8
+    V = r.standard_normal((n, d))
+    V[7] = 0.0
+    kept = np.zeros(n, dtype=bool)
+    kept[r.choice(n, 30, replace=False)] = True
+    t = O.route_cosine(V, kept)
+    for j in range(n):
+        if kept[j]:
+            assert t[j] == -1
+            continue
+        best, bi = -2.0, -1
+        for i in range(n):
+            if not kept[i]:
+                continue
+            den = math.sqrt(float(V[j] @ V[j])) * math.sqrt(float(V[i] @ V[i]))
+            c = float(V[j] @ V[i]) / den if den > 0 else 0.0
+            if c > best:
+                best, bi = c, i
+        assert t[j] == bi
+
+
+def test_cosine_routing_gate_is_the_max_cosine():
+    """With cosine routing the gate of j is its largest cosine to any kept token, clamped."""
+    wl, K, V, Q, n = _tiny(seed=5)
+    r = O.compress(K, V, Q, n, wl.rho, O.Params(routing=O.ROUTE_COSINE))
+    ki = r.kept_idx
+    for kv in range(K.shape[0]):
+        Vk = V[kv, ki]
+        nk = np.linalg.norm(Vk, axis=1)
+        for j in np.flatnonzero(r.target[kv] >= 0)[:60]:
+            cos = (Vk @ V[kv, j]) / (nk * np.linalg.norm(V[kv, j]))
+            assert abs(r.g[kv, j] - min(max(cos.max(), 0.0), 1.0)) < 1e-12
+        ev = r.target[kv] >= 0
+        lhs = float((r.a[kv, ki] * r.R[kv]).sum())
+        rhs = float(r.a[kv, ki].sum() + (r.g[kv, ev] * r.a[kv, ev]).sum())
+        assert abs(lhs - rhs) <= 1e-12 * rhs      # mass conservation holds for any routing
