@@ -272,7 +272,8 @@ def run_gpu(args):
     params = S.selkv_params.defaults(
         select_mode=S.SELKV_SELECT_PER_HEAD if args.select_mode == "per_head" else S.SELKV_SELECT_SHARED,
         rope={"off": S.SELKV_ROPE_OFF, "half": S.SELKV_ROPE_HALF,
-              "interleaved": S.SELKV_ROPE_INTERLEAVED}[args.rope], rope_theta=args.rope_theta)
+              "interleaved": S.SELKV_ROPE_INTERLEAVED}[args.rope], rope_theta=args.rope_theta,
+        routing=S.SELKV_ROUTE_COSINE if args.routing == "cosine" else S.SELKV_ROUTE_BUCKET)
     L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e)
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
@@ -391,7 +392,7 @@ def run_gpu(args):
         "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
                    "rho": wl.rho, "decode_steps": L.T, "q_heads": Hq, "kv_heads": Hkv,
                    "head_dim": d, "obs_window": wl.obs_window, "select_mode": args.select_mode,
-                   "rope": args.rope,
+                   "rope": args.rope, "routing": args.routing,
                    "parallelism": "replicas",
                    "l2": "inputs larger than L2: every token streams all layers' compressed "
                          "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
@@ -412,7 +413,7 @@ def run_gpu(args):
     }
     if e2e is not None:
         line["e2e"] = e2e
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.routing == "bucket":
         line["cpu_baseline"] = oracle_sample(wl, per_head=args.select_mode == "per_head")
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -537,6 +538,9 @@ def main():
     ap.add_argument("--rope", default="off", choices=["off", "half", "interleaved"],
                     help="RoPE repositioning of the kept keys (Eq. 7; off in the paper's configuration)")
     ap.add_argument("--rope-theta", type=float, default=500000.0)
+    ap.add_argument("--routing", default="bucket", choices=["bucket", "cosine"],
+                    help="routing of the evicted tokens: bucket (Eq. 3, the default) or the full "
+                         "cosine routing of Sec. 3.4 (the oracle baseline is not sampled for it)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

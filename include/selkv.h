@@ -86,6 +86,13 @@ typedef enum selkv_select_mode { SELKV_SELECT_SHARED = 0, SELKV_SELECT_PER_HEAD 
  * it with g > 0), averaged over KV heads in SHARED mode (alpha = 1: KeepKV's log(1 + M)). */
 typedef enum selkv_bias_mode { SELKV_BIAS_RATIO = 0, SELKV_BIAS_COUNT = 1 } selkv_bias_mode;
 
+/* Routing of the evicted tokens (Sec. 3.4): BUCKET is the paper's bucket attention routing
+ * (Eq. 3, with empty_bucket); COSINE is the full cosine routing that Sec. 3.4 sets against it
+ * (cost O(|S| |E| d) per KV head): evicted j goes to the kept token i of its KV head with the
+ * largest cos(v_j, v_i) over ALL kept tokens (original values; ties to the lower position; a
+ * zero norm gives cosine 0).  The gate, merge and bias are the same in both. */
+typedef enum selkv_routing { SELKV_ROUTE_BUCKET = 0, SELKV_ROUTE_COSINE = 1 } selkv_routing;
+
 typedef enum selkv_rope {
   SELKV_ROPE_OFF = 0,
   SELKV_ROPE_HALF = 1,
@@ -123,6 +130,7 @@ typedef struct selkv_params {
   int32_t rope;         /* selkv_rope, OFF (Sec. 4.1)                                     */
   float rope_theta;     /* rotary base, finite and > 0 when rope is on                    */
   int32_t bias_mode;    /* selkv_bias_mode, RATIO (Sec. 3.6)                              */
+  int32_t routing;      /* selkv_routing, BUCKET (Sec. 3.4)                               */
 } selkv_params;
 
 /* Optional device outputs of selkv_compress, for inspection and testing.  Any field may be

@@ -11,7 +11,7 @@ from ._binding import (  # noqa: F401
     SELKV_ERR_DEVICE, SELKV_BF16, SELKV_FP32, SELKV_GATE_COSINE, SELKV_GATE_OPEN,
     SELKV_GATE_CLOSED, SELKV_EMPTY_EXPAND, SELKV_EMPTY_DROP, SELKV_SELECT_SHARED,
     SELKV_SELECT_PER_HEAD, SELKV_ROPE_OFF, SELKV_ROPE_HALF, SELKV_ROPE_INTERLEAVED,
-    SELKV_BIAS_RATIO, SELKV_BIAS_COUNT,
+    SELKV_BIAS_RATIO, SELKV_BIAS_COUNT, SELKV_ROUTE_BUCKET, SELKV_ROUTE_COSINE,
     SELKV_DEVERR_CAPACITY,
     SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT, SELKV_MAX_BATCH,
     SelKVError, selkv_shape, selkv_params, selkv_compress_debug, library, library_path,

@@ -17,6 +17,7 @@ SELKV_EMPTY_EXPAND, SELKV_EMPTY_DROP = 0, 1
 SELKV_SELECT_SHARED, SELKV_SELECT_PER_HEAD = 0, 1
 SELKV_ROPE_OFF, SELKV_ROPE_HALF, SELKV_ROPE_INTERLEAVED = 0, 1, 2
 SELKV_BIAS_RATIO, SELKV_BIAS_COUNT = 0, 1
+SELKV_ROUTE_BUCKET, SELKV_ROUTE_COSINE = 0, 1
 SELKV_DEVERR_CAPACITY, SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT = 1, 2, 4, 8
 SELKV_MAX_BATCH = 1024
 SELKV_STATIC_SCRATCH_BYTES = 4 << 20
@@ -40,14 +41,16 @@ class selkv_shape(ctypes.Structure):
 class selkv_params(ctypes.Structure):
     _fields_ = [("alpha", c_f32), ("pool_kernel", c_i32), ("bucket", c_i32), ("recent", c_i32),
                 ("gate_mode", c_i32), ("empty_bucket", c_i32), ("select_mode", c_i32),
-                ("rope", c_i32), ("rope_theta", c_f32), ("bias_mode", c_i32)]
+                ("rope", c_i32), ("rope_theta", c_f32), ("bias_mode", c_i32),
+                ("routing", c_i32)]
 
     @classmethod
     def defaults(cls, **kw) -> "selkv_params":
         """The paper's configuration (Sec. 4.1 / App. F): alpha 0.5, K 5, B 32, m_r 16."""
         p = dict(alpha=0.5, pool_kernel=5, bucket=32, recent=16, gate_mode=SELKV_GATE_COSINE,
                  empty_bucket=SELKV_EMPTY_EXPAND, select_mode=SELKV_SELECT_SHARED,
-                 rope=SELKV_ROPE_OFF, rope_theta=10000.0, bias_mode=SELKV_BIAS_RATIO)
+                 rope=SELKV_ROPE_OFF, rope_theta=10000.0, bias_mode=SELKV_BIAS_RATIO,
+                 routing=SELKV_ROUTE_BUCKET)
         p.update(kw)
         return cls(**p)
 

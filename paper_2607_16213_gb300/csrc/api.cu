@@ -65,6 +65,7 @@ SideStream* side_stream(cudaStream_t caller) {
 
 struct CompressPlan {
   size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, mcount, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
+  size_t cos_invn, cos_rank, cos_order, cos_cnt, cos_total, cos_base;
   int nchunks, R;
 };
 
@@ -99,6 +100,15 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.mcount = take(B * Hkv * (size_t)s.m_cap * 4);
   // RoPE repositioning tables (used only with params->rope): coarse and fine (cos, sin)
   p.rope_tab = take((size_t)(s.head_dim / 2) * (rope_coarse(s.n_cap) + 256) * 8);
+  // full cosine routing (used only with params->routing == COSINE; its target slots and gates
+  // live in tau / atau)
+  const size_t mpad = ((size_t)s.m_cap + 255) / 256 * 256;
+  p.cos_invn = take(B * Hkv * mpad * 4);
+  p.cos_rank = take(B * Hkv * n * 4);
+  p.cos_order = take(B * Hkv * n * 4);
+  p.cos_cnt = take(B * Hkv * (size_t)cos_chunks_for(s.n_cap) * s.m_cap * 4);
+  p.cos_total = take(B * Hkv * (size_t)s.m_cap * 4);
+  p.cos_base = take(B * Hkv * (size_t)s.m_cap * 4);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
   p.total = off;
   return p;
@@ -196,6 +206,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   if (!std::isfinite(p.alpha) || p.pool_kernel < 1 || (p.pool_kernel & 1) == 0 || p.recent < 0 ||
       p.bucket < 1 || p.gate_mode < 0 || p.gate_mode > 2 || p.empty_bucket < 0 || p.empty_bucket > 1 ||
       p.select_mode < 0 || p.select_mode > 1 || p.rope < 0 || p.rope > 2 || p.bias_mode < 0 || p.bias_mode > 1 ||
+      p.routing < 0 || p.routing > 1 ||
       (p.rope != 0 && !(std::isfinite(p.rope_theta) && p.rope_theta > 0.f)))
     return SELKV_ERR_INVALID_ARG;
   if (p.bucket > 32) return SELKV_ERR_UNSUPPORTED;
@@ -273,6 +284,18 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.ratio = at<float>(workspace, plan.ratio);
   a.mcount = at<float>(workspace, plan.mcount);
   a.rope_tab = at<float2>(workspace, plan.rope_tab);
+  a.routing = p.routing;
+  a.cos_chunks = cos_chunks_for(s.n_cap);
+  a.cos_chunk = cos_chunk_len(s.n_cap);
+  a.cos_mpad = (s.m_cap + 255) / 256 * 256;
+  a.cos_tslot = a.tau;
+  a.cos_g = a.atau;
+  a.cos_invn = at<float>(workspace, plan.cos_invn);
+  a.cos_rank = at<int32_t>(workspace, plan.cos_rank);
+  a.cos_order = at<int32_t>(workspace, plan.cos_order);
+  a.cos_cnt = at<int32_t>(workspace, plan.cos_cnt);
+  a.cos_total = at<int32_t>(workspace, plan.cos_total);
+  a.cos_base = at<int32_t>(workspace, plan.cos_base);
   if (debug != nullptr) {
     a.dbg_topk = debug->topk;
     a.dbg_kept_idx = debug->kept_idx;
@@ -300,7 +323,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
   g_launches += (score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2) -
-                (a.per_head ? 4 : 0) + (a.rope ? 1 : 0);  // no union / trim in per-head mode
+                (a.per_head ? 4 : 0) + (a.rope ? 1 : 0) +  // no union / trim in per-head mode
+                (a.routing == SELKV_ROUTE_COSINE ? (s.m_cap > 0 ? cosine_kernels(a.dtype, a.D) : 0) - 2 : 0);
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

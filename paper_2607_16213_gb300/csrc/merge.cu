@@ -1,5 +1,7 @@
 // Bucket-attention routing, soft cosine gate, gated merge, attention ratio and the
-// compressed-cache write-out of SelKV (Eq. 3-6, Sec. 3.6 GQA bias).
+// compressed-cache write-out of SelKV (Eq. 3-6, Sec. 3.6 GQA bias).  With the full cosine
+// routing the route and merge kernels give way to those of route_cosine.cu, launched after
+// the copy.
 //
 // Under Eq. 3 (argmax over the kept tokens of a bucket of the cumulative attention a) every
 // evicted token of a bucket routes to the same kept token tau_X, so the merge is a gather.
@@ -220,6 +222,10 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   } else {
     dst[piece] = src[piece];
   }
+  if (piece == 0 && tensor == 1 && a.routing == SELKV_ROUTE_COSINE) {
+    const float nv = a.vnorm[bk * a.n_cap + pos];
+    a.cos_invn[bk * a.cos_mpad + slot] = nv > 0.f ? 1.f / nv : 0.f;
+  }
   if (piece == 0 && tensor == 0) {
     a.ratio[bk * a.m_cap + slot] = 1.f;
     a.mcount[bk * a.m_cap + slot] = 0.f;
@@ -230,49 +236,6 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
     if (a.dbg_decision) a.dbg_decision[o] = 2;
   }
 }
-
-// One lane's PER consecutive elements of a row, kept in the storage type.
-template <typename T, int PER>
-struct RowSlice;
-template <>
-struct RowSlice<__nv_bfloat16, 4> {
-  uint2 w;
-  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint2*>(p); }
-  __device__ __forceinline__ void zero() { w = make_uint2(0u, 0u); }
-  __device__ __forceinline__ float operator[](int e) const {
-    const uint32_t x = e < 2 ? w.x : w.y;
-    return (e & 1) ? bf16_hi(x) : bf16_lo(x);
-  }
-};
-template <>
-struct RowSlice<__nv_bfloat16, 2> {
-  uint32_t w;
-  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint32_t*>(p); }
-  __device__ __forceinline__ void zero() { w = 0u; }
-  __device__ __forceinline__ float operator[](int e) const { return (e & 1) ? bf16_hi(w) : bf16_lo(w); }
-};
-template <int PER>
-struct RowSlice<float, PER> {
-  float x[PER];
-  __device__ __forceinline__ void load(const float* p) {
-    if constexpr (PER == 4) {
-      const float4 v = *reinterpret_cast<const float4*>(p);
-      x[0] = v.x;
-      x[1] = v.y;
-      x[2] = v.z;
-      x[3] = v.w;
-    } else {
-      const float2 v = *reinterpret_cast<const float2*>(p);
-      x[0] = v.x;
-      x[1] = v.y;
-    }
-  }
-  __device__ __forceinline__ void zero() {
-#pragma unroll
-    for (int e = 0; e < PER; ++e) x[e] = 0.f;
-  }
-  __device__ __forceinline__ float operator[](int e) const { return x[e]; }
-};
 
 // Sum kBatch per-lane partials p[k] over the 32 lanes with the batch spread over the lanes:
 // each butterfly level keeps half of the values and adds the partner's copy of them, so lanes
@@ -530,7 +493,7 @@ void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
   constexpr int kPieces = D * (int)sizeof(T) / 16;
   const size_t copy_threads = (size_t)a.Hkv * a.m_cap * 2 * kPieces;
   copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
-  merge_kernel<T, D><<<dim3(a.nbk, a.B * a.Hkv), 32, 0, s>>>(a);
+  if (a.routing == SELKV_ROUTE_BUCKET) merge_kernel<T, D><<<dim3(a.nbk, a.B * a.Hkv), 32, 0, s>>>(a);
 }
 
 }  // namespace
@@ -541,13 +504,18 @@ cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s) {
     const int threads = a.D / 2 * groups;
     rope_table_kernel<<<(threads + 127) / 128, 128, 0, s>>>(a);
   }
-  route_kernel<<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B), kWarpsPerCta * 32, 0, s>>>(a);
+  if (a.routing == SELKV_ROUTE_BUCKET)
+    route_kernel<<<dim3((a.nbk + kWarpsPerCta - 1) / kWarpsPerCta, a.B), kWarpsPerCta * 32, 0, s>>>(a);
   if (a.dtype == SELKV_BF16) {
     if (a.D == 128) launch_merge_t<__nv_bfloat16, 128>(a, s);
     else launch_merge_t<__nv_bfloat16, 64>(a, s);
   } else {
     if (a.D == 128) launch_merge_t<float, 128>(a, s);
     else launch_merge_t<float, 64>(a, s);
+  }
+  if (a.routing == SELKV_ROUTE_COSINE) {
+    const cudaError_t e = launch_route_cosine(a, s);
+    if (e != cudaSuccess) return e;
   }
   bias_kernel<<<dim3((a.m_cap + 255) / 256, a.B), 256, 0, s>>>(a);
   return cudaGetLastError();

@@ -75,6 +75,49 @@ __device__ __forceinline__ void store4(float* p, const float (&x)[4]) {
   *reinterpret_cast<float4*>(p) = make_float4(x[0], x[1], x[2], x[3]);
 }
 
+// One lane's PER consecutive elements of a row, kept in the storage type.
+template <typename T, int PER>
+struct RowSlice;
+template <>
+struct RowSlice<__nv_bfloat16, 4> {
+  uint2 w;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint2*>(p); }
+  __device__ __forceinline__ void zero() { w = make_uint2(0u, 0u); }
+  __device__ __forceinline__ float operator[](int e) const {
+    const uint32_t x = e < 2 ? w.x : w.y;
+    return (e & 1) ? bf16_hi(x) : bf16_lo(x);
+  }
+};
+template <>
+struct RowSlice<__nv_bfloat16, 2> {
+  uint32_t w;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { w = *reinterpret_cast<const uint32_t*>(p); }
+  __device__ __forceinline__ void zero() { w = 0u; }
+  __device__ __forceinline__ float operator[](int e) const { return (e & 1) ? bf16_hi(w) : bf16_lo(w); }
+};
+template <int PER>
+struct RowSlice<float, PER> {
+  float x[PER];
+  __device__ __forceinline__ void load(const float* p) {
+    if constexpr (PER == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(p);
+      x[0] = v.x;
+      x[1] = v.y;
+      x[2] = v.z;
+      x[3] = v.w;
+    } else {
+      const float2 v = *reinterpret_cast<const float2*>(p);
+      x[0] = v.x;
+      x[1] = v.y;
+    }
+  }
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int e = 0; e < PER; ++e) x[e] = 0.f;
+  }
+  __device__ __forceinline__ float operator[](int e) const { return x[e]; }
+};
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -138,6 +181,19 @@ struct CompressArgs {
   float* atau;       // [B][Hkv][nbk] a of that target
   float* ratio;      // [B][Hkv][m_cap] attention ratio R of each slot
   float* mcount;     // [B][Hkv][m_cap] evicted tokens merged into each slot (g > 0)
+  // full cosine routing (routing == SELKV_ROUTE_COSINE)
+  int routing;
+  int cos_chunks;      // position chunks of the stable counting sort by target slot
+  int cos_chunk;       // positions per chunk (a multiple of 32)
+  int cos_mpad;        // m_cap rounded up to a whole 256-slot tile
+  int32_t* cos_tslot;  // [B][Hkv][n_cap] target slot of an evicted j merged with g > 0, else -1
+  float* cos_g;        // [B][Hkv][n_cap] gate g of an evicted j
+  float* cos_invn;     // [B][Hkv][cos_mpad] 1 / ||v|| of each slot's kept value (0 for a zero norm)
+  int32_t* cos_rank;   // [B][Hkv][n_cap] rank of j among the earlier j of its chunk with its target
+  int32_t* cos_order;  // [B][Hkv][n_cap] contributors grouped by target slot, ascending within
+  int32_t* cos_cnt;    // [B][Hkv][cos_chunks][m_cap] contributors per (chunk, slot), then their prefix
+  int32_t* cos_total;  // [B][Hkv][m_cap] contributors per slot
+  int32_t* cos_base;   // [B][Hkv][m_cap] first entry of each slot in cos_order
 };
 
 // SM count used to plan grids and splits: fixed, so that workspace sizes and results do
@@ -186,6 +242,16 @@ int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms);  // pass-1 k
 cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
+// Full cosine routing after the kept rows are in place: argmax, gate, grouping and merge.
+cudaError_t launch_route_cosine(const CompressArgs& a, cudaStream_t s);
+int cosine_kernels(int dtype, int D);  // kernels launch_route_cosine enqueues
+// Chunks of the counting sort for caches of n_cap positions, and the chunk length.
+__host__ __device__ constexpr int cos_chunks_for(int n_cap) {
+  return n_cap <= 2048 ? 1 : (n_cap + 2047) / 2048 < 32 ? (n_cap + 2047) / 2048 : 32;
+}
+__host__ __device__ constexpr int cos_chunk_len(int n_cap) {
+  return ((n_cap + cos_chunks_for(n_cap) - 1) / cos_chunks_for(n_cap) + 31) / 32 * 32;
+}
 
 // ---- decode -------------------------------------------------------------------------------
 struct DecodeArgs {

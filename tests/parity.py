@@ -11,6 +11,8 @@ Margins (derived from the arithmetic):
              relative error of a few 1e-6 (fp32 sums of exponentials whose arguments carry
              rounding error), so near-ties closer than 1e-4 relative may resolve either way.
   DELTA_SIM  absolute margin on the cosine around 0 (merge vs drop).
+  DELTA_COS  absolute margin between two cosines (full cosine routing): the GPU's cosines are
+             fp32 sums of d products (exact for bf16 inputs), a few 1e-7 off the exact value.
 """
 from __future__ import annotations
 
@@ -26,6 +28,7 @@ import paper_2607_16213_gb300 as S
 
 DELTA = 1e-4
 DELTA_SIM = 1e-5
+DELTA_COS = 1e-5
 
 # continuous tolerances
 ATTN_RTOL = 5e-5        # a and pooled scores: relative to the value (plus a tiny floor)
@@ -50,7 +53,7 @@ def params_of(p: O.Params) -> S.selkv_params:
     return S.selkv_params(alpha=p.alpha, pool_kernel=p.pool_kernel, bucket=p.bucket,
                           recent=p.recent, gate_mode=p.gate_mode, empty_bucket=p.empty_bucket,
                           select_mode=p.select_mode, rope=p.rope, rope_theta=p.rope_theta,
-                          bias_mode=p.bias_mode)
+                          bias_mode=p.bias_mode, routing=p.routing)
 
 
 def run_compress(wl: synth.Workload, x: dict, p: O.Params, rho=None, extra: int = 0):
@@ -152,15 +155,7 @@ def check_sequence(wl, x, host, b: int, p: O.Params, rho=None, stats: Stats = No
     ev = np.flatnonzero(~kept_g)
     for kv in range(Hkv):
         assert (tgt_g[kv, kept_g] == -1).all() and (dec_g[kv, kept_g] == 2).all()
-        own = O.route(a[kv], kept_g, p.bucket, p.empty_bucket)
-        diff = ev[tgt_g[kv, ev] != own[ev]]
-        for j in diff:
-            tg, to = int(tgt_g[kv, j]), int(own[j])
-            assert tg >= 0 and to >= 0 and kept_g[tg], "target of %d: gpu %d oracle %d" % (j, tg, to)
-            # same ring distance, a within DELTA of the oracle's choice
-            assert abs(tg // p.bucket - j // p.bucket) == abs(to // p.bucket - j // p.bucket)
-            assert abs(a[kv, tg] - a[kv, to]) <= DELTA * a[kv, to], "routing differs at %d" % j
-        stats.add("route_near_ties", int(diff.size))
+        _check_routing(p, stats, a[kv], V[kv], kept_g, tgt_g[kv], ev)
         g_o, sim_o, dec_o = O.gate(V[kv], tgt_g[kv], p.gate_mode)
         routed = ev[tgt_g[kv, ev] >= 0]
         err_g = np.abs(gate_g[kv, routed] - g_o[routed])
@@ -216,19 +211,38 @@ def check_keys(host_Kc: np.ndarray, K_kept: np.ndarray, kept_idx: np.ndarray, p:
     assert err.max() <= 0, "repositioned keys beyond tolerance by %.3g" % err.max()
 
 
+def _cos(x: np.ndarray, y: np.ndarray) -> float:
+    den = math.sqrt(float(x @ x)) * math.sqrt(float(y @ y))
+    return float(x @ y) / den if den > 0 else 0.0
+
+
+def _check_routing(p, stats, a_kv, V_kv, kept_g, tgt_g, ev):
+    """Step 3 of one KV head: the GPU's targets against the oracle's, exact except at near
+    ties (bucket routing: the same ring distance and a within DELTA; cosine routing: cosines
+    within DELTA_COS)."""
+    if p.routing == O.ROUTE_COSINE:
+        own = O.route_cosine(V_kv, kept_g)
+    else:
+        own = O.route(a_kv, kept_g, p.bucket, p.empty_bucket)
+    diff = ev[tgt_g[ev] != own[ev]]
+    for j in diff:
+        tg, to = int(tgt_g[j]), int(own[j])
+        assert tg >= 0 and to >= 0 and kept_g[tg], "target of %d: gpu %d oracle %d" % (j, tg, to)
+        if p.routing == O.ROUTE_COSINE:
+            assert _cos(V_kv[j], V_kv[to]) - _cos(V_kv[j], V_kv[tg]) <= DELTA_COS, "routing differs at %d" % j
+        else:
+            # same ring distance, a within DELTA of the oracle's choice
+            assert abs(tg // p.bucket - j // p.bucket) == abs(to // p.bucket - j // p.bucket)
+            assert abs(a_kv[tg] - a_kv[to]) <= DELTA * a_kv[to], "routing differs at %d" % j
+    stats.add("route_near_ties", int(diff.size))
+
+
 def _check_steps_3_to_6(p, stats, kv, n, a_kv, V_kv, kept_g, tgt_g, gate_g, dec_g):
     """Routing, gate and decision of one KV head against the oracle, continuing from the
     GPU's kept set; returns the oracle's gates for that head's merge."""
     ev = np.flatnonzero(~kept_g)
     assert (tgt_g[kept_g] == -1).all() and (dec_g[kept_g] == 2).all()
-    own = O.route(a_kv, kept_g, p.bucket, p.empty_bucket)
-    diff = ev[tgt_g[ev] != own[ev]]
-    for j in diff:
-        tg, to = int(tgt_g[j]), int(own[j])
-        assert tg >= 0 and to >= 0 and kept_g[tg], "target of %d: gpu %d oracle %d" % (j, tg, to)
-        assert abs(tg // p.bucket - j // p.bucket) == abs(to // p.bucket - j // p.bucket)
-        assert abs(a_kv[tg] - a_kv[to]) <= DELTA * a_kv[to], "routing differs at %d" % j
-    stats.add("route_near_ties", int(diff.size))
+    _check_routing(p, stats, a_kv, V_kv, kept_g, tgt_g, ev)
     g_o, sim_o, dec_o = O.gate(V_kv, tgt_g, p.gate_mode)
     routed = ev[tgt_g[ev] >= 0]
     err_g = np.abs(gate_g[routed] - g_o[routed])

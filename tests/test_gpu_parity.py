@@ -326,3 +326,72 @@ def test_compress_count_bias(name, mode, alpha):
     _, host, _ = run_compress(wl, x, p)
     for b in range(wl.batch):
         check_sequence(wl, x, host, b, p)
+
+
+# ---------------------------------------------------------------- full cosine routing (Sec. 3.4)
+@pytest.mark.parametrize("name,mode", [
+    ("tiny", O.SELECT_SHARED),
+    ("bf16_ragged", O.SELECT_SHARED),
+    ("bf16_d64_g4", O.SELECT_SHARED),
+    ("fp32_d128", O.SELECT_SHARED),
+    ("bf16_mha", O.SELECT_PER_HEAD),
+])
+def test_compress_cosine_routing(name, mode):
+    wl = SMALL.get(name) or PER_HEAD[name]
+    x = synth.gen_layer(wl, 6)
+    p = O.Params(routing=O.ROUTE_COSINE, select_mode=mode)
+    _, host, _ = run_compress(wl, x, p)
+    st = Stats()
+    for b in range(wl.batch):
+        check_sequence(wl, x, host, b, p, stats=st)
+    print(name, dict(st))
+
+
+@pytest.mark.parametrize("case", [
+    dict(p=dict(gate_mode=O.GATE_OPEN)),
+    dict(p=dict(gate_mode=O.GATE_CLOSED)),
+    dict(p=dict(bias_mode=O.BIAS_COUNT, alpha=1.0)),
+    dict(rho=1.0),                                   # nothing evicted
+    dict(rho=16 / 3001 + 1e-9),                      # only the recent window is kept
+    dict(rho=0.9),                                   # several 256-slot tiles and a ragged one
+])
+def test_compress_cosine_routing_cases(case):
+    wl = SMALL["bf16_ragged"].with_(batch=1, ragged=None)
+    x = synth.gen_layer(wl, 7)
+    p = O.Params(routing=O.ROUTE_COSINE, **case.get("p", {}))
+    rho = case.get("rho", wl.rho)
+    _, host, _ = run_compress(wl, x, p, rho=rho)
+    check_sequence(wl, x, host, 0, p, rho=rho)
+
+
+def test_cosine_routing_repeat_is_bitwise_identical():
+    wl = SMALL["bf16_ragged"]
+    x = synth.gen_layer(wl, 8)
+    p = O.Params(routing=O.ROUTE_COSINE)
+    _, h1, _ = run_compress(wl, x, p)
+    _, h2, _ = run_compress(wl, x, p)
+    for k in ("target", "gate", "V_c", "ratio", "bias"):
+        np.testing.assert_array_equal(h1[k], h2[k], err_msg=k)
+
+
+def test_cosine_routing_hub_and_zero_rows():
+    """Adversarial values: many evicted rows parallel to one kept row (a hub slot with hundreds
+    of contributors), zero value rows, and exact ties between kept rows."""
+    wl = SMALL["bf16_ragged"].with_(batch=1, ragged=None, seed=31)
+    x = synth.gen_layer(wl, 0)
+    V = x["V"]
+    V0 = V[0]                                   # [Hkv][n_cap][d], a view
+    r = np.random.default_rng(5)
+    n = wl.n
+    hub = r.choice(n, 700, replace=False)
+    # powers of two keep the copies exact in bf16
+    V0[:, hub] = V0[:, hub[:1]] * r.choice([0.5, 1.0, 2.0], size=(1, 700, 1)).astype(V.dtype)
+    V0[:, r.choice(n, 40, replace=False)] = 0
+    twins = r.choice(n, 60, replace=False)
+    V0[:, twins[30:]] = V0[:, twins[:30]]
+    x["V"] = V
+    p = O.Params(routing=O.ROUTE_COSINE)
+    _, host, _ = run_compress(wl, x, p)
+    st = Stats()
+    check_sequence(wl, x, host, 0, p, stats=st)
+    print(dict(st))
