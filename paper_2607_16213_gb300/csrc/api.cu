@@ -65,7 +65,7 @@ SideStream* side_stream(cudaStream_t caller) {
 
 struct CompressPlan {
   size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, mcount, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
-  size_t cos_invn, cos_rank, cos_order, cos_cnt, cos_total, cos_base;
+  size_t ev_pos, cos_invn, cos_rank, cos_order, cos_cnt, cos_seg;
   int nchunks, R;
 };
 
@@ -103,12 +103,12 @@ CompressPlan plan_compress(const selkv_shape& s) {
   // full cosine routing (used only with params->routing == COSINE; its target slots and gates
   // live in tau / atau)
   const size_t mpad = ((size_t)s.m_cap + 255) / 256 * 256;
+  p.ev_pos = take(B * Hkv * n * 4);
   p.cos_invn = take(B * Hkv * mpad * 4);
   p.cos_rank = take(B * Hkv * n * 4);
   p.cos_order = take(B * Hkv * n * 4);
   p.cos_cnt = take(B * Hkv * (size_t)cos_chunks_for(s.n_cap) * s.m_cap * 4);
-  p.cos_total = take(B * Hkv * (size_t)s.m_cap * 4);
-  p.cos_base = take(B * Hkv * (size_t)s.m_cap * 4);
+  p.cos_seg = take(B * Hkv * (size_t)s.m_cap * 8);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
   p.total = off;
   return p;
@@ -290,12 +290,12 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.cos_mpad = (s.m_cap + 255) / 256 * 256;
   a.cos_tslot = a.tau;
   a.cos_g = a.atau;
+  a.ev_pos = at<int32_t>(workspace, plan.ev_pos);
   a.cos_invn = at<float>(workspace, plan.cos_invn);
   a.cos_rank = at<int32_t>(workspace, plan.cos_rank);
   a.cos_order = at<int32_t>(workspace, plan.cos_order);
   a.cos_cnt = at<int32_t>(workspace, plan.cos_cnt);
-  a.cos_total = at<int32_t>(workspace, plan.cos_total);
-  a.cos_base = at<int32_t>(workspace, plan.cos_base);
+  a.cos_seg = at<int2>(workspace, plan.cos_seg);
   if (debug != nullptr) {
     a.dbg_topk = debug->topk;
     a.dbg_kept_idx = debug->kept_idx;

@@ -225,6 +225,7 @@ __global__ __launch_bounds__(256) void copy_kernel(CompressArgs a) {
   if (piece == 0 && tensor == 1 && a.routing == SELKV_ROUTE_COSINE) {
     const float nv = a.vnorm[bk * a.n_cap + pos];
     a.cos_invn[bk * a.cos_mpad + slot] = nv > 0.f ? 1.f / nv : 0.f;
+    a.cos_tslot[bk * a.n_cap + pos] = -1;  // a kept token routes nowhere
   }
   if (piece == 0 && tensor == 0) {
     a.ratio[bk * a.m_cap + slot] = 1.f;

@@ -8,13 +8,13 @@
 // |S| |E| d multiply-adds per KV head, run on the tensor cores for bf16 caches.  Kernels, in
 // stream order (after the copy kernel has put the kept rows into V_c and 1 / ||v_i|| into
 // cos_invn):
-//   argmax   a CTA per 128 positions of one (sequence, KV head): the 128 value rows stay in
-//            shared memory (the MMA's A), 256-slot tiles of the kept rows stream in by TMA (B),
-//            tcgen05.mma accumulates 128 x 256 products in tensor memory, and sixteen epilogue
-//            warps keep each row's running (max s_ji, slot) over a quarter of each tile's
-//            columns; the quarters are folded in column order at the end.  The row's target,
-//            gate g = clamp(s / ||v_j||, 0, 1) and decision are written there.  fp32 caches use
-//            a CUDA-core kernel with the same outputs.
+//   argmax   a CTA per 128 evicted positions of one (sequence, KV head): their value rows are
+//            gathered once into shared memory (the MMA's A), 256-slot tiles of the kept rows
+//            stream in by TMA (B), tcgen05.mma accumulates 128 x 256 products in tensor memory,
+//            and sixteen epilogue warps keep each row's running (max s_ji, slot) over a quarter
+//            of each tile's columns; the quarters are folded in column order at the end.  The
+//            row's target, gate g = clamp(s / ||v_j||, 0, 1) and decision are written there.
+//            fp32 caches use a CUDA-core kernel with the same outputs.
 //   rank     stable counting sort of the contributors (g > 0) by target slot, part 1: a warp per
 //            (chunk of positions, block of 2048 slots) walks its chunk in ascending order and
 //            gives each contributor its rank among the earlier ones of the chunk with the
@@ -35,14 +35,11 @@ namespace selkv {
 namespace {
 
 // ---- row finish: target, gate and decision of position j --------------------------------
+// (Evicted positions only; the copy kernel writes the entries of the kept ones.)
 __device__ __forceinline__ void cos_finish(const CompressArgs& a, int b, int kv, int j, float best, int bcol) {
   const size_t bk = (size_t)b * a.Hkv + kv;
   const size_t o = bk * a.n_cap + j;
   const size_t su = sel_unit(a, b, kv);
-  if (a.kflag[su * a.n_cap + j]) {  // kept: the copy kernel wrote its debug entries
-    a.cos_tslot[o] = -1;
-    return;
-  }
   float g = 0.f;
   int tpos = -1;
   if (bcol >= 0) {
@@ -72,7 +69,7 @@ constexpr int kProducerWarp = 16, kMmaWarp = 17;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kCols = 256;                 // kept slots per tile: the MMA's N
 constexpr int kChunkBytes = kCols * 128;   // one 64-element-wide box of a tile
-constexpr int kRingChunks = 4;
+constexpr int kRingChunks = 4;             // two tiles in flight at d = 128
 constexpr uint32_t kTmemCols = 512;        // two 256-column accumulators
 
 template <int D>
@@ -82,6 +79,7 @@ struct CosCfg {
   static constexpr int kRing = kRingChunks * kChunkBytes;
   static constexpr int kMisc = 256 + 3 * 128 * 8;
   static constexpr int kSmem = 1024 + kABytes + kRing + kMisc;
+  static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
 };
 
 __device__ __forceinline__ uint64_t fmul2(uint64_t x, uint64_t y) {
@@ -94,20 +92,27 @@ __device__ __forceinline__ float fmax3(float x, float y, float z) {
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(x), "f"(y), "f"(z));
   return d;
 }
+__device__ __forceinline__ float max32(const float (&x)[32]) {
+  float mx[11];
+#pragma unroll
+  for (int i = 0; i < 10; ++i) mx[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
+  mx[10] = fmaxf(x[30], x[31]);
+  const float m0 = fmax3(mx[0], mx[1], mx[2]), m1 = fmax3(mx[3], mx[4], mx[5]);
+  const float m2 = fmax3(mx[6], mx[7], mx[8]), m3 = fmax3(mx[9], mx[10], m0);
+  return fmax3(m1, m2, m3);
+}
 
 template <int D>
-__global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_constant__ CUtensorMap tmA,
-                                                              const __grid_constant__ CUtensorMap tmB,
-                                                              CompressArgs a) {
+__global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_constant__ CUtensorMap tmB, CompressArgs a) {
   using C = CosCfg<D>;
   const int kv = blockIdx.y, b = blockIdx.z;
-  const int n = a.seq_n[b], m = a.seq_m[b];
+  const int n = a.seq_n[b], m = a.seq_m[b], ne = n - m;
   const int r0 = blockIdx.x * 128;
-  if (r0 >= n) return;
+  if (r0 >= ne) return;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  unsigned char* As = smem;               // [kBoxes][128 rows][128 B]
+  unsigned char* As = smem;                 // [kBoxes][128 rows][128 B]
   unsigned char* ring = smem + C::kABytes;  // [kRingChunks][256 rows][128 B]
   unsigned char* misc = ring + C::kRing;
   uint64_t* full = reinterpret_cast<uint64_t*>(misc);
@@ -122,6 +127,7 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const size_t bk = (size_t)b * a.Hkv + kv;
+  const size_t su = sel_unit(a, b, kv);
   const int nt = (m + kCols - 1) / kCols;
   const int nchunks = nt * C::kBoxes;
 
@@ -147,11 +153,7 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
 
   if (warp == kProducerWarp) {
     if (lane == 0 && nt > 0) {
-      prefetch_tensormap(&tmA);
       prefetch_tensormap(&tmB);
-      mbar_arrive_expect_tx(abar, C::kABytes);
-      for (int bx = 0; bx < C::kBoxes; ++bx)
-        tma_load_2d(As + bx * 128 * 128, &tmA, bx * 64, (int)(bk * a.n_cap) + r0, abar);
       const int brow0 = (int)(bk * a.m_cap);
       int issued = 0;
       for (int c = 0; c < nchunks; ++c) {
@@ -167,7 +169,6 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
       }
       for (int c = max(0, issued - kRingChunks); c < issued; ++c)
         mbar_wait(&full[c % kRingChunks], (c / kRingChunks) & 1);
-      mbar_wait(abar, 0);
     }
   } else if (warp == kMmaWarp) {
     if (lane == 0 && nt > 0) {
@@ -191,7 +192,7 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
           for (int ks = 0; ks < 4; ++ks)
             umma_bf16(tmem + buf * kCols, umma_desc_sw128(abase + bx * 128 * 128 + ks * 32),
                       umma_desc_sw128(rbase + st * kChunkBytes + ks * 32), idesc, (bx | ks) > 0);
-          umma_commit(&empty[st]);  // the chunk's smem is free once these MMAs have read it
+          umma_commit(&empty[st]);  // the stage is free once these MMAs have read it
         }
         if (!ok) break;
         umma_commit(&tfull[buf]);
@@ -205,6 +206,23 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
     }
   } else {
     // ---------------- epilogue: warps 0-15 ----------------
+    const int32_t* ev = a.ev_pos + su * a.n_cap;  // evicted positions, ascending
+    {
+      // gather the 128 evicted value rows into the swizzled A layout (rows past the evicted
+      // count repeat the last one; their results are not written)
+      constexpr int kRowChunks = D / 8;  // 16-byte pieces per row
+      const __nv_bfloat16* Vb = static_cast<const __nv_bfloat16*>(a.V) + bk * a.n_cap * D;
+      const uint32_t abase = smem_u32(As);
+      for (int i = threadIdx.x; i < 128 * kRowChunks; i += kEpiWarps * 32) {
+        const int r = i / kRowChunks, ch = i % kRowChunks;
+        const int j = ev[min(r0 + r, ne - 1)];
+        cp_async16_cg(abase + (ch >> 3) * (128 * 128) + swz128(r, ch & 7), Vb + (size_t)j * D + ch * 8);
+      }
+      cp_async_wait_all();
+      fence_proxy_async_smem();  // visible to the tensor cores (async proxy)
+      named_bar_sync(1, kEpiWarps * 32);
+      if (threadIdx.x == 0) mbar_arrive(abar);
+    }
     const int q = warp & 3, part = warp >> 2;  // TMEM lane quarter (rows), column quarter of a tile
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const float* invn = a.cos_invn + bk * a.cos_mpad;
@@ -231,33 +249,26 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
           float v[32];
           tmem_ld32(tmem + lane_base + buf * kCols + part * 64 + c, v);
           const int col0 = t * kCols + part * 64 + c;
-          if (col0 >= m) continue;
+          if (col0 >= m) continue;  // uniform across the warp
           // s = acc / ||v_i||, pairs packed; slots past m take -inf
           const float4* w4 = reinterpret_cast<const float4*>(invn + col0);
-          float s[32];
 #pragma unroll
           for (int i = 0; i < 32; i += 4) {
             const float4 w = __ldg(w4 + i / 4);
-            unpack_f2(fmul2(pack_f2(v[i], v[i + 1]), pack_f2(w.x, w.y)), s[i], s[i + 1]);
-            unpack_f2(fmul2(pack_f2(v[i + 2], v[i + 3]), pack_f2(w.z, w.w)), s[i + 2], s[i + 3]);
+            unpack_f2(fmul2(pack_f2(v[i], v[i + 1]), pack_f2(w.x, w.y)), v[i], v[i + 1]);
+            unpack_f2(fmul2(pack_f2(v[i + 2], v[i + 3]), pack_f2(w.z, w.w)), v[i + 2], v[i + 3]);
           }
           if (col0 + 32 > m) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) s[i] = col0 + i < m ? s[i] : -INFINITY;
+            for (int i = 0; i < 32; ++i) v[i] = col0 + i < m ? v[i] : -INFINITY;
           }
-          float mx[11];
-#pragma unroll
-          for (int i = 0; i < 10; ++i) mx[i] = fmax3(s[3 * i], s[3 * i + 1], s[3 * i + 2]);
-          mx[10] = fmaxf(s[30], s[31]);
-          const float m0 = fmax3(mx[0], mx[1], mx[2]), m1 = fmax3(mx[3], mx[4], mx[5]);
-          const float m2 = fmax3(mx[6], mx[7], mx[8]), m3 = fmax3(mx[9], mx[10], m0);
-          const float cmax = fmax3(m1, m2, m3);
+          const float cmax = max32(v);
           if (cmax > best) {  // strictly larger: an equal value at a later slot does not win
-            uint32_t hit = 0;
+            int first = 31;   // the lowest slot holding the maximum
 #pragma unroll
-            for (int i = 0; i < 32; ++i) hit |= (s[i] == cmax ? 1u : 0u) << i;
+            for (int i = 30; i >= 0; --i) first = v[i] == cmax ? i : first;
             best = cmax;
-            bcol = col0 + __ffs(hit) - 1;
+            bcol = col0 + first;
           }
         }
       }
@@ -269,13 +280,13 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
     const int r = q * 32 + lane;
     if (part > 0) fold[(part - 1) * 128 + r] = make_float2(best, __int_as_float(bcol));
     named_bar_sync(1, kEpiWarps * 32);
-    if (part == 0 && r0 + r < n) {
+    if (part == 0 && r0 + r < ne) {
 #pragma unroll
       for (int k = 0; k < 3; ++k) {
         const float2 f = fold[k * 128 + r];
         argmax_take(best, bcol, f.x, __float_as_int(f.y));
       }
-      cos_finish(a, b, kv, r0 + r, best, bcol);
+      cos_finish(a, b, kv, ev[r0 + r], best, bcol);
     }
   }
   tc_fence_before();
@@ -287,18 +298,19 @@ __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_consta
 }
 
 // ---- argmax on the CUDA cores (fp32 caches) ----------------------------------------------
-// A warp per position j: lane l takes the slots l, l + 32, ... in ascending order, then the
-// warp reduces (max, lower slot).
+// A warp per evicted position j: lane l takes the slots l, l + 32, ... in ascending order, then
+// the warp reduces (max, lower slot).
 constexpr int kSimtRows = 8;
 template <typename T, int D>
 __global__ __launch_bounds__(kSimtRows * 32) void cos_simt_kernel(CompressArgs a) {
   const int kv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.x * kSimtRows + warp;
+  const int e = blockIdx.x * kSimtRows + warp;  // evicted rank
   const int n = a.seq_n[b], m = a.seq_m[b];
   __shared__ float vj[kSimtRows][D];
-  if (j >= n) return;
+  if (e >= n - m) return;
   const size_t bk = (size_t)b * a.Hkv + kv;
+  const int j = a.ev_pos[sel_unit(a, b, kv) * a.n_cap + e];
   const T* row = static_cast<const T*>(a.V) + (bk * a.n_cap + j) * D;
   for (int d = lane; d < D; d += 32) vj[warp][d] = load1(row + d);
   __syncwarp();
@@ -342,19 +354,28 @@ __global__ __launch_bounds__(32) void cos_rank_kernel(CompressArgs a) {
   const int j_lo = c * a.cos_chunk, j_hi = min(n, j_lo + a.cos_chunk);
   const int32_t* ts = a.cos_tslot + (size_t)bk * a.n_cap;
   int32_t* rank = a.cos_rank + (size_t)bk * a.n_cap;
-  for (int j0 = j_lo; j0 < j_hi; j0 += 32) {
-    const int j = j0 + lane;
-    const int t = j < j_hi ? ts[j] : -1;
-    const bool mine = t >= s0 && t < s0 + ns;
-    const uint32_t peers = __match_any_sync(0xffffffffu, mine ? t : -1);
-    const int before = mine ? cnt[t - s0] : 0;
-    __syncwarp();
-    if (mine) {
-      const int lt = __popc(peers & ((1u << lane) - 1u));
-      if (lt == 0) cnt[t - s0] = before + __popc(peers);
-      rank[j] = before + lt;
+  constexpr int kRounds = 8;  // targets loaded ahead, 32 positions per round
+  for (int j0 = j_lo; j0 < j_hi; j0 += kRounds * 32) {
+    int tv[kRounds];
+#pragma unroll
+    for (int k = 0; k < kRounds; ++k) {
+      const int j = j0 + k * 32 + lane;
+      tv[k] = j < j_hi ? ts[j] : -1;
     }
-    __syncwarp();
+#pragma unroll
+    for (int k = 0; k < kRounds; ++k) {
+      const int j = j0 + k * 32 + lane, t = tv[k];
+      const bool mine = t >= s0 && t < s0 + ns;
+      const uint32_t peers = __match_any_sync(0xffffffffu, mine ? t : -1);
+      const int before = mine ? cnt[t - s0] : 0;
+      __syncwarp();
+      if (mine) {
+        const int lt = __popc(peers & ((1u << lane) - 1u));
+        if (lt == 0) cnt[t - s0] = before + __popc(peers);
+        rank[j] = before + lt;
+      }
+      __syncwarp();
+    }
   }
   int32_t* out = a.cos_cnt + ((size_t)bk * a.cos_chunks + c) * a.m_cap + s0;
   for (int k = lane; k < ns; k += 32) out[k] = cnt[k];
@@ -365,13 +386,16 @@ __global__ __launch_bounds__(256) void cos_colscan_kernel(CompressArgs a) {
   const int slot = blockIdx.x * blockDim.x + threadIdx.x;
   if (slot >= a.seq_m[b]) return;
   int32_t* col = a.cos_cnt + (size_t)bk * a.cos_chunks * a.m_cap + slot;
+  int x[kMaxCosChunks];
+#pragma unroll
+  for (int c = 0; c < kMaxCosChunks; ++c) x[c] = c < a.cos_chunks ? col[(size_t)c * a.m_cap] : 0;
   int run = 0;
-  for (int c = 0; c < a.cos_chunks; ++c) {
-    const int x = col[(size_t)c * a.m_cap];
-    col[(size_t)c * a.m_cap] = run;
-    run += x;
+#pragma unroll
+  for (int c = 0; c < kMaxCosChunks; ++c) {
+    if (c < a.cos_chunks) col[(size_t)c * a.m_cap] = run;
+    run += x[c];
   }
-  a.cos_total[(size_t)bk * a.m_cap + slot] = run;
+  a.cos_seg[(size_t)bk * a.m_cap + slot].y = run;
 }
 
 __global__ __launch_bounds__(1024) void cos_slotscan_kernel(CompressArgs a) {
@@ -379,12 +403,14 @@ __global__ __launch_bounds__(1024) void cos_slotscan_kernel(CompressArgs a) {
   const int m = a.seq_m[b];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __shared__ int wsum[32];
-  const int32_t* tot = a.cos_total + (size_t)bk * a.m_cap;
-  int32_t* base = a.cos_base + (size_t)bk * a.m_cap;
+  int2* seg = a.cos_seg + (size_t)bk * a.m_cap;
   int carry = 0;
-  for (int s0 = 0; s0 < m; s0 += 1024) {
-    const int s = s0 + threadIdx.x;
-    const int x = s < m ? tot[s] : 0;
+  for (int s0 = 0; s0 < m; s0 += 4096) {
+    const int s = s0 + 4 * threadIdx.x;  // four consecutive slots per thread
+    int e[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) e[k] = s + k < m ? seg[s + k].y : 0;
+    const int x = (e[0] + e[1]) + (e[2] + e[3]);
     int v = x;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -403,7 +429,12 @@ __global__ __launch_bounds__(1024) void cos_slotscan_kernel(CompressArgs a) {
       wsum[lane] = w;
     }
     __syncthreads();
-    if (s < m) base[s] = carry + (warp > 0 ? wsum[warp - 1] : 0) + v - x;
+    int run = carry + (warp > 0 ? wsum[warp - 1] : 0) + v - x;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (s + k < m) seg[s + k].x = run;
+      run += e[k];
+    }
     carry += wsum[31];
     __syncthreads();  // wsum is rewritten by the next round
   }
@@ -418,7 +449,7 @@ __global__ __launch_bounds__(256) void cos_scatter_kernel(CompressArgs a) {
   const int t = a.cos_tslot[o];
   if (t < 0) return;
   const int c = j / a.cos_chunk;
-  const int dest = a.cos_base[(size_t)bk * a.m_cap + t] +
+  const int dest = a.cos_seg[(size_t)bk * a.m_cap + t].x +
                    a.cos_cnt[((size_t)bk * a.cos_chunks + c) * a.m_cap + t] + a.cos_rank[o];
   if (dest < 0 || dest >= n) {
     raise_flag(a.flags, SELKV_DEVERR_COUNT);
@@ -429,7 +460,7 @@ __global__ __launch_bounds__(256) void cos_scatter_kernel(CompressArgs a) {
 
 // ---- gated merge over each slot's contributors (Eq. 5, Eq. 6) ----------------------------
 constexpr int kMergeWarps = 8;
-constexpr int kBatch = 16;  // contributor rows in flight per lane
+constexpr int kBatch = 8;  // contributor rows in flight per lane
 
 template <typename T, int D>
 __global__ __launch_bounds__(kMergeWarps * 32) void cos_merge_kernel(CompressArgs a) {
@@ -439,10 +470,10 @@ __global__ __launch_bounds__(kMergeWarps * 32) void cos_merge_kernel(CompressArg
   const int slot = blockIdx.x * kMergeWarps + warp;
   if (slot >= a.seq_m[b]) return;
   const size_t sm = (size_t)bk * a.m_cap + slot;
-  const int cnt = a.cos_total[sm];
-  if (cnt == 0) return;  // V_c keeps the kept value, R = 1 (copy kernel)
-  const int beg = a.cos_base[sm];
+  const int2 sg = a.cos_seg[sm];  // (first entry, contributors)
   const int pos = a.kept_pos[sel_unit(a, b, kv) * a.m_cap + slot];
+  const int cnt = sg.y, beg = sg.x;
+  if (cnt == 0) return;  // V_c keeps the kept value, R = 1 (copy kernel)
   const T* Vb = static_cast<const T*>(a.V) + (size_t)bk * a.n_cap * D;
   const float* A = a.attn + (size_t)bk * a.n_cap;
   const float* Gt = a.cos_g + (size_t)bk * a.n_cap;
@@ -498,15 +529,12 @@ __global__ __launch_bounds__(kMergeWarps * 32) void cos_merge_kernel(CompressArg
 template <int D>
 cudaError_t launch_argmax_tc(const CompressArgs& a, cudaStream_t st) {
   using C = CosCfg<D>;
-  if ((uint64_t)a.B * a.Hkv * a.n_cap >= (1ull << 31) || (uint64_t)a.B * a.Hkv * a.m_cap >= (1ull << 31))
-    return cudaErrorInvalidValue;  // TMA row coordinates are 32-bit
-  CUtensorMap ta, tb;
-  if (!encode_rows_bf16(&ta, a.V, (uint64_t)a.B * a.Hkv * a.n_cap, D, 128) ||
-      !encode_rows_bf16(&tb, a.Vc, (uint64_t)a.B * a.Hkv * a.m_cap, D, kCols))
-    return cudaErrorInvalidValue;
+  if ((uint64_t)a.B * a.Hkv * a.m_cap >= (1ull << 31)) return cudaErrorInvalidValue;  // 32-bit TMA rows
+  CUtensorMap tb;
+  if (!encode_rows_bf16(&tb, a.Vc, (uint64_t)a.B * a.Hkv * a.m_cap, D, kCols)) return cudaErrorInvalidValue;
   cudaError_t e = set_smem_once<cos_tc_kernel<D>>(C::kSmem);
   if (e != cudaSuccess) return e;
-  cos_tc_kernel<D><<<dim3((a.n_cap + 127) / 128, a.Hkv, a.B), kThreads, C::kSmem, st>>>(ta, tb, a);
+  cos_tc_kernel<D><<<dim3((a.n_cap + 127) / 128, a.Hkv, a.B), kThreads, C::kSmem, st>>>(tb, a);
   return cudaGetLastError();
 }
 

@@ -338,6 +338,8 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
     const uint32_t slot = base + wcnt[warp] + __popc(bal & ((1u << lane) - 1u));
     if (j < n) {
       a.slot_of[(size_t)u * a.n_cap + j] = kept ? (int)slot : -1;
+      // with the full cosine routing: the evicted positions in order (slot = kept ones before j)
+      if (!kept && a.routing == SELKV_ROUTE_COSINE) a.ev_pos[(size_t)u * a.n_cap + (j - (int)slot)] = j;
       if (kept && (int)slot < a.m_cap) {
         a.kept_pos[(size_t)u * a.m_cap + slot] = j;
         if (a.dbg_kept_idx != nullptr) a.dbg_kept_idx[(size_t)u * a.m_cap + slot] = j;

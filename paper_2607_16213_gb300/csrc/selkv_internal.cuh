@@ -186,14 +186,14 @@ struct CompressArgs {
   int cos_chunks;      // position chunks of the stable counting sort by target slot
   int cos_chunk;       // positions per chunk (a multiple of 32)
   int cos_mpad;        // m_cap rounded up to a whole 256-slot tile
+  int32_t* ev_pos;     // [units][n_cap] evicted positions in ascending order
   int32_t* cos_tslot;  // [B][Hkv][n_cap] target slot of an evicted j merged with g > 0, else -1
   float* cos_g;        // [B][Hkv][n_cap] gate g of an evicted j
   float* cos_invn;     // [B][Hkv][cos_mpad] 1 / ||v|| of each slot's kept value (0 for a zero norm)
   int32_t* cos_rank;   // [B][Hkv][n_cap] rank of j among the earlier j of its chunk with its target
   int32_t* cos_order;  // [B][Hkv][n_cap] contributors grouped by target slot, ascending within
   int32_t* cos_cnt;    // [B][Hkv][cos_chunks][m_cap] contributors per (chunk, slot), then their prefix
-  int32_t* cos_total;  // [B][Hkv][m_cap] contributors per slot
-  int32_t* cos_base;   // [B][Hkv][m_cap] first entry of each slot in cos_order
+  int2* cos_seg;       // [B][Hkv][m_cap] (first entry in cos_order, contributors) of each slot
 };
 
 // SM count used to plan grids and splits: fixed, so that workspace sizes and results do
@@ -246,8 +246,9 @@ cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_route_cosine(const CompressArgs& a, cudaStream_t s);
 int cosine_kernels(int dtype, int D);  // kernels launch_route_cosine enqueues
 // Chunks of the counting sort for caches of n_cap positions, and the chunk length.
+constexpr int kMaxCosChunks = 32;
 __host__ __device__ constexpr int cos_chunks_for(int n_cap) {
-  return n_cap <= 2048 ? 1 : (n_cap + 2047) / 2048 < 32 ? (n_cap + 2047) / 2048 : 32;
+  return n_cap <= 2048 ? 1 : (n_cap + 2047) / 2048 < kMaxCosChunks ? (n_cap + 2047) / 2048 : kMaxCosChunks;
 }
 __host__ __device__ constexpr int cos_chunk_len(int n_cap) {
   return ((n_cap + cos_chunks_for(n_cap) - 1) / cos_chunks_for(n_cap) + 31) / 32 * 32;
