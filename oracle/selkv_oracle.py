@@ -56,6 +56,12 @@ path):
   R20 full cosine routing (the alternative Sec. 3.4 prices at O(H |S| |E| d)): pi(j) is the
       kept token of the head with the largest cos(v_j, v_i) over all kept tokens, with the
       original (pre-merge) values; ties to the lower position; a zero norm gives cosine 0.
+  R21 compensation averaged across layers (the overview of Sec. 3 offers it next to the per-
+      layer bias): one value per (sequence, position), shared by every layer, is the mean over
+      the L layers of the layer's per-slot quantity at that position (the KV-head mean R of
+      R16, or M of R19; per KV head in the per-head mode), a layer that evicted the position
+      counting the neutral value (R = 1, M = 0); every layer's slot holding the position then
+      gets alpha * ln(mean R), or alpha * ln(1 + mean M).
 """
 from __future__ import annotations
 
@@ -365,6 +371,29 @@ def merge_counts(kept_idx: np.ndarray, target: np.ndarray, g: np.ndarray) -> np.
 def count_bias(M: np.ndarray, alpha: float, per_head: bool) -> np.ndarray:
     """R19: alpha * ln(1 + mean_kv M) (shared; M [Hkv][m] -> [m]) or alpha * ln(1 + M) per head."""
     return alpha * np.log1p(M) if per_head else alpha * np.log1p(M.mean(axis=0))
+
+
+def layer_average_bias(q_layers, kept_layers, n: int, alpha: float, count: bool) -> list:
+    """R21: the per-layer biases of one sequence replaced by their cross-layer average.
+    q_layers[l]: layer l's per-slot quantity (KV-head mean R, or mean M in the count variant),
+    shape [m] in the shared mode or [Hkv][m] per head; kept_layers[l]: the positions of those
+    slots, same shape.  Returns the new bias of every layer, same shapes."""
+    neutral = 0.0 if count else 1.0
+    first = np.asarray(q_layers[0], dtype=np.float64)
+    total = np.zeros(first.shape[:-1] + (n,))   # sum over layers, neutral where evicted
+    L = len(q_layers)
+    for q, kept in zip(q_layers, kept_layers):
+        q = np.asarray(q, dtype=np.float64)
+        kept = np.asarray(kept, dtype=np.int64)
+        here = np.full(total.shape, neutral)
+        np.put_along_axis(here, kept, q, axis=-1)
+        total += here
+    mean = total / L
+    out = []
+    for kept in kept_layers:
+        mk = np.take_along_axis(mean, np.asarray(kept, dtype=np.int64), axis=-1)
+        out.append(alpha * (np.log1p(mk) if count else np.log(mk)))
+    return out
 
 
 def per_head_bias(R: np.ndarray, alpha: float) -> np.ndarray:

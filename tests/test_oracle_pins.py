@@ -607,3 +607,44 @@ def test_cosine_routing_gate_is_the_max_cosine():
         lhs = float((r.a[kv, ki] * r.R[kv]).sum())
         rhs = float(r.a[kv, ki].sum() + (r.g[kv, ev] * r.a[kv, ev]).sum())
         assert abs(lhs - rhs) <= 1e-12 * rhs      # mass conservation holds for any routing
+
+
+# ---------------------------------------------------------------- compensation averaged across layers
+def test_layer_average_bias_worked_example():
+    """Hand-worked, n = 4, two layers: layer 0 keeps positions 0 and 2 with R = 2 and 4, layer 1
+    keeps 2 and 3 with R = 2 and 3.  Per position the mean over layers (R = 1 where a layer
+    evicted it): 0 -> (2 + 1) / 2 = 1.5, 2 -> (4 + 2) / 2 = 3, 3 -> (1 + 3) / 2 = 2."""
+    out = O.layer_average_bias([np.array([2.0, 4.0]), np.array([2.0, 3.0])],
+                               [np.array([0, 2]), np.array([2, 3])], 4, 0.5, count=False)
+    np.testing.assert_allclose(out[0], 0.5 * np.log([1.5, 3.0]), rtol=0, atol=1e-15)
+    np.testing.assert_allclose(out[1], 0.5 * np.log([3.0, 2.0]), rtol=0, atol=1e-15)
+    # the count variant: M = 0 where evicted, bias = alpha ln(1 + mean M)
+    out = O.layer_average_bias([np.array([2.0, 4.0]), np.array([2.0, 3.0])],
+                               [np.array([0, 2]), np.array([2, 3])], 4, 1.0, count=True)
+    np.testing.assert_allclose(out[0], np.log([2.0, 4.0]), rtol=0, atol=1e-15)   # 1 + 1, 1 + 3
+    np.testing.assert_allclose(out[1], np.log([4.0, 2.5]), rtol=0, atol=1e-15)   # 1 + 3, 1 + 1.5
+
+
+def test_layer_average_bias_reductions():
+    """One layer, or identical layers, give back the per-layer bias (Sec. 3.6, R16 / R19); the
+    result does not depend on the order of the layers; per-head shapes average per head."""
+    r = rng(51)
+    n, m, Hkv = 300, 80, 3
+    kept = np.sort(r.choice(n, m, replace=False))
+    R = 1.0 + r.exponential(1.0, size=m)
+    np.testing.assert_allclose(O.layer_average_bias([R], [kept], n, 0.5, False)[0], 0.5 * np.log(R), atol=1e-15)
+    for out in O.layer_average_bias([R, R, R], [kept, kept, kept], n, 0.5, False):
+        np.testing.assert_allclose(out, 0.5 * np.log(R), atol=1e-14)
+    layers = [(1.0 + r.exponential(1.0, size=m), np.sort(r.choice(n, m, replace=False))) for _ in range(4)]
+    a = O.layer_average_bias([q for q, _ in layers], [k for _, k in layers], n, 0.5, False)
+    perm = [2, 0, 3, 1]
+    b = O.layer_average_bias([layers[i][0] for i in perm], [layers[i][1] for i in perm], n, 0.5, False)
+    for i, pi in enumerate(perm):
+        np.testing.assert_allclose(b[i], a[pi], atol=1e-14)
+    Rh = [1.0 + r.exponential(1.0, size=(Hkv, m)) for _ in range(2)]
+    Kh = [np.sort(np.stack([r.choice(n, m, replace=False) for _ in range(Hkv)]), axis=1) for _ in range(2)]
+    out = O.layer_average_bias(Rh, Kh, n, 0.5, False)
+    for h in range(Hkv):
+        want = O.layer_average_bias([Rh[0][h], Rh[1][h]], [Kh[0][h], Kh[1][h]], n, 0.5, False)
+        np.testing.assert_allclose(out[0][h], want[0], atol=1e-15)
+        np.testing.assert_allclose(out[1][h], want[1], atol=1e-15)
