@@ -187,7 +187,7 @@ class HostArena:
 class Layered:
     """Device-resident inputs and outputs of every layer."""
 
-    def __init__(self, wl, torch, api, S, dev, pinned_host: bool):
+    def __init__(self, wl, torch, api, S, dev, pinned_host: bool, layer_average: bool = False):
         self.wl = wl
         B, Hq, Hkv, d, W = wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.obs_window
         tdt = api.torch_dtype(api.dtype_code(wl.dtype))
@@ -227,17 +227,36 @@ class Layered:
         self.out = torch.empty((self.T, wl.layers, B, Hq, d), dtype=tdt, device=dev)
         self.cws = api.Workspace(S.selkv_compress_workspace_size(self.shape), dev)
         self.dws = api.Workspace(S.selkv_decode_workspace_size(self.shape), dev)
+        # compensation averaged across layers: each layer's kept positions are kept for it
+        self.layer_average = layer_average
+        # (sized for the per-head mode's [B][Hkv][m_cap]; the shared mode uses the first B m_cap)
+        self.kept = [torch.empty((B, Hkv, self.m_cap), dtype=torch.int32, device=dev) for _ in range(wl.layers)] \
+            if layer_average else []
+        self.aws = api.Workspace(S.selkv_layer_average_workspace_size(self.shape), dev) if layer_average else None
+
+
+def compress_layers(L: Layered, S, params, stream_ptr, before_layer=None):
+    """Enqueue the compression of every layer (and, with layer averaging, the average)."""
+    wl = L.wl
+    for layer in range(wl.layers):
+        if before_layer is not None:
+            before_layer(layer)
+        c = L.caches[layer]
+        dbg = {"kept_idx": L.kept[layer]} if L.layer_average else None
+        S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
+                                 c.K_c, c.V_c, c.bias, c.lengths, dbg, L.cws.buf, L.cws.nbytes,
+                                 stream_ptr), "compress")
+    if L.layer_average:
+        S.check(S.selkv_layer_average_bias(L.shape, params, L.kept, [c.bias for c in L.caches],
+                                           L.caches[0].lengths, L.aws.buf, L.aws.nbytes, stream_ptr),
+                "layer average")
 
 
 def issue_step(L: Layered, S, params, stream_ptr, decode_ranges=None):
     """Enqueue one step on the stream; returns the number of kernels enqueued."""
     wl = L.wl
     k0 = S.selkv_kernel_launches()
-    for layer in range(wl.layers):
-        c = L.caches[layer]
-        S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
-                                 c.K_c, c.V_c, c.bias, c.lengths, None, L.cws.buf, L.cws.nbytes,
-                                 stream_ptr), "compress")
+    compress_layers(L, S, params, stream_ptr)
     if decode_ranges is not None:
         decode_ranges[0]()
     for t in range(L.T):
@@ -274,7 +293,7 @@ def run_gpu(args):
         rope={"off": S.SELKV_ROPE_OFF, "half": S.SELKV_ROPE_HALF,
               "interleaved": S.SELKV_ROPE_INTERLEAVED}[args.rope], rope_theta=args.rope_theta,
         routing=S.SELKV_ROUTE_COSINE if args.routing == "cosine" else S.SELKV_ROUTE_BUCKET)
-    L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e)
+    L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e, layer_average=args.layer_average)
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
     peaks, peak_src = load_peaks()
@@ -288,11 +307,7 @@ def run_gpu(args):
     g_comp = torch.cuda.CUDAGraph()
     g_dec = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_comp, stream=stream):
-        for layer in range(wl.layers):
-            c = L.caches[layer]
-            S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
-                                     c.K_c, c.V_c, c.bias, c.lengths, None, L.cws.buf, L.cws.nbytes,
-                                     stream.cuda_stream), "compress")
+        compress_layers(L, S, params, stream.cuda_stream)
     with torch.cuda.graph(g_dec, stream=stream):
         for t in range(L.T):
             for layer in range(wl.layers):
@@ -393,6 +408,7 @@ def run_gpu(args):
                    "rho": wl.rho, "decode_steps": L.T, "q_heads": Hq, "kv_heads": Hkv,
                    "head_dim": d, "obs_window": wl.obs_window, "select_mode": args.select_mode,
                    "rope": args.rope, "routing": args.routing,
+                   "compensation": "averaged across layers" if args.layer_average else "per layer",
                    "parallelism": "replicas",
                    "l2": "inputs larger than L2: every token streams all layers' compressed "
                          "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
@@ -413,7 +429,7 @@ def run_gpu(args):
     }
     if e2e is not None:
         line["e2e"] = e2e
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.routing == "bucket":
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.routing == "bucket" and not args.layer_average:
         line["cpu_baseline"] = oracle_sample(wl, per_head=args.select_mode == "per_head")
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -453,10 +469,7 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int):
                 L.Q[layer].copy_(hQ, non_blocking=True)
                 arrived[layer].record(copy_stream)
         with torch.cuda.stream(stream):
-            for layer in range(wl.layers):
-                stream.wait_event(arrived[layer])
-                api.compress(L.shape, L.n_len, wl.rho, L.K[layer], L.V[layer], L.Q[layer], params=params,
-                             out=L.caches[layer], workspace=L.cws, stream=sp)
+            compress_layers(L, S, params, sp, before_layer=lambda layer: stream.wait_event(arrived[layer]))
             for t in range(L.T):
                 dq.copy_(hq[t], non_blocking=True)
                 dk.copy_(hk[t], non_blocking=True)
@@ -541,6 +554,8 @@ def main():
     ap.add_argument("--routing", default="bucket", choices=["bucket", "cosine"],
                     help="routing of the evicted tokens: bucket (Eq. 3, the default) or the full "
                          "cosine routing of Sec. 3.4 (the oracle baseline is not sampled for it)")
+    ap.add_argument("--layer-average", action="store_true",
+                    help="compensation averaged across layers instead of per layer (Sec. 3 overview)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -174,11 +174,13 @@ SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t str
  *   (Sec. 3.3), plus the recent window: m_b = floor(rho * n_b) kept positions shared by
  *   every head, ties to the lower position (PER_HEAD mode: each KV head's own top-m_s plus
  *   the recent window, m_b positions per head);
- *   each evicted j routes to the kept token of its bucket with the largest a (Eq. 3, Sec. 3.4), gets
+ *   each evicted j routes to the kept token of its bucket with the largest a (Eq. 3, Sec. 3.4;
+ *   COSINE routing: to the kept token with the largest cos(v_j, v_i)), gets
  *   g = clamp(cos(v_j, v_pi(j)), 0, 1) (Eq. 4) and is merged into V_c with weight g*a_j
  *   (Eq. 5); R = (a_i + sum g a_j) / a_i (Eq. 6); bias = alpha * ln(mean over KV heads R)
- *   (Sec. 3.6, GQA; PER_HEAD mode: alpha * ln R of each head's own entry); K_c holds the kept
- *   keys, unchanged or, with params->rope, re-embedded at their slot positions (Eq. 7).
+ *   (Sec. 3.6, GQA; PER_HEAD mode: alpha * ln R of each head's own entry; COUNT bias:
+ *   alpha * ln(1 + M) of the merge counts instead); K_c holds the kept keys, unchanged or,
+ *   with params->rope, re-embedded at their slot positions (Eq. 7).
  *
  * n_len     HOST array [B]: prefill lengths, W <= n_b <= n_cap.
  * rho       retention ratio in (0, 1]; m_b = floor(rho * n_b) (double), and
@@ -199,6 +201,40 @@ SELKV_API selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n
                             const void* Q_obs, void* K_c, void* V_c, float* bias,
                             int32_t* lengths, const selkv_compress_debug* debug,
                             void* workspace, size_t workspace_bytes, selkv_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------
+ * Compensation averaged across layers (the overview of Sec. 3 offers it next to the
+ * per-layer bias of Sec. 3.6).  After the L layers of a model have been compressed with the
+ * same params, every layer's bias is replaced by one value per position shared by all
+ * layers: for each sequence b (and KV head in the PER_HEAD mode) and position p, the mean over
+ * the L layers of the layer's per-slot quantity at p -- the R of the bias (the KV-head mean in
+ * the SHARED mode) or, with the COUNT bias, M -- a layer that evicted p counting R = 1
+ * (M = 0); the slot of every layer that holds p then gets alpha * ln(mean R), or
+ * alpha * ln(1 + mean M).  The per-slot quantity is read back from each bias
+ * (alpha * ln(1 + x), x = R - 1 or M), so call this once per compression; with alpha = 0 the
+ * biases stay 0 and nothing is launched.
+ *
+ * params      the params given to selkv_compress (alpha, bias_mode, select_mode are read).
+ * num_layers  L, 1 .. 128.
+ * kept_idx    HOST array [L] of device pointers: each layer's kept positions as written to
+ *             selkv_compress_debug.kept_idx ([B][m_cap]; [B][Hkv][m_cap] in PER_HEAD mode).
+ * bias        HOST array [L] of device pointers: each layer's bias [B][Hkv][m_cap], read and
+ *             overwritten (slots >= lengths[b] untouched).
+ * lengths     [B] int32 device: the compressed lengths m_b, the same for every layer (call
+ *             before decode appends).
+ * The sums are taken layer by layer in order (bitwise reproducible).  Errors:
+ * SELKV_ERR_INVALID_ARG for NULL or misaligned pointers, L outside 1..128 or bad params;
+ * SELKV_ERR_WORKSPACE when workspace_bytes < selkv_layer_average_workspace_size (the
+ * workspace is initialised once with selkv_workspace_init); a kept position outside
+ * [0, n_cap) sets SELKV_DEVERR_COUNT.
+ * ------------------------------------------------------------------------------------- */
+SELKV_API size_t selkv_layer_average_workspace_size(const selkv_shape* shape);
+
+SELKV_API selkv_status selkv_layer_average_bias(const selkv_shape* shape, const selkv_params* params,
+                                                int32_t num_layers, const int32_t* const* kept_idx,
+                                                float* const* bias, const int32_t* lengths,
+                                                void* workspace, size_t workspace_bytes,
+                                                selkv_stream_t stream);
 
 /* ---------------------------------------------------------------------------------------
  * Compensated decode attention (Algorithm 1, "Decode with compressed cache + alpha log R";

@@ -18,5 +18,6 @@ from ._binding import (  # noqa: F401
     exported_symbols, check, selkv_status_string, selkv_kernel_launches, selkv_workspace_init,
     selkv_workspace_error, selkv_compress_workspace_size, selkv_compress,
     selkv_decode_workspace_size, selkv_decode_attn, selkv_decode_attn_static,
+    selkv_layer_average_workspace_size, selkv_layer_average_bias,
     SELKV_STATIC_SCRATCH_BYTES,
 )

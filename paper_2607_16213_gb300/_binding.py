@@ -86,6 +86,10 @@ def library() -> ctypes.CDLL:
         "selkv_compress": (c_i32, [ctypes.POINTER(selkv_shape), ctypes.POINTER(c_i32), c_f64,
                                    ctypes.POINTER(selkv_params), c_vp, c_vp, c_vp, c_vp, c_vp, c_vp,
                                    c_vp, ctypes.POINTER(selkv_compress_debug), c_vp, c_sz, c_vp]),
+        "selkv_layer_average_workspace_size": (c_sz, [ctypes.POINTER(selkv_shape)]),
+        "selkv_layer_average_bias": (c_i32, [ctypes.POINTER(selkv_shape), ctypes.POINTER(selkv_params), c_i32,
+                                             ctypes.POINTER(c_vp), ctypes.POINTER(c_vp), c_vp, c_vp, c_sz,
+                                             c_vp]),
         "selkv_decode_workspace_size": (c_sz, [ctypes.POINTER(selkv_shape)]),
         "selkv_decode_attn": (c_i32, [ctypes.POINTER(selkv_shape), c_vp, c_vp, c_vp, c_vp, c_vp,
                                       c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]),
@@ -152,6 +156,20 @@ def selkv_workspace_error(workspace, stream=None):
 
 def selkv_compress_workspace_size(shape: selkv_shape) -> int:
     return int(library().selkv_compress_workspace_size(ctypes.byref(shape)))
+
+
+def selkv_layer_average_workspace_size(shape: selkv_shape) -> int:
+    return library().selkv_layer_average_workspace_size(ctypes.byref(shape))
+
+
+def selkv_layer_average_bias(shape: selkv_shape, params: selkv_params, kept_idx, bias, lengths,
+                             workspace, workspace_bytes: int, stream=None) -> int:
+    """kept_idx, bias: sequences of per-layer tensors (or device addresses)."""
+    L = len(kept_idx)
+    kept_arr = (c_vp * L)(*[_ptr(k) for k in kept_idx])
+    bias_arr = (c_vp * L)(*[_ptr(b) for b in bias])
+    return library().selkv_layer_average_bias(ctypes.byref(shape), ctypes.byref(params), L, kept_arr, bias_arr,
+                                              _ptr(lengths), _ptr(workspace), workspace_bytes, _stream(stream))
 
 
 def selkv_decode_workspace_size(shape: selkv_shape) -> int:

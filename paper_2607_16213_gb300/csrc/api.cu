@@ -328,6 +328,49 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 
+size_t selkv_layer_average_workspace_size(const selkv_shape* shape) {
+  if (!shape_ok(shape)) return 0;
+  return sizeof(WsHeader) + round256((size_t)shape->batch * shape->num_kv_heads * shape->n_cap * sizeof(float));
+}
+
+selkv_status selkv_layer_average_bias(const selkv_shape* shape, const selkv_params* params, int32_t num_layers,
+                                      const int32_t* const* kept_idx, float* const* bias,
+                                      const int32_t* lengths, void* workspace, size_t workspace_bytes,
+                                      selkv_stream_t stream) {
+  if (!shape_ok(shape) || params == nullptr || kept_idx == nullptr || bias == nullptr || lengths == nullptr)
+    return SELKV_ERR_INVALID_ARG;
+  if (num_layers < 1 || num_layers > kMaxLayers) return SELKV_ERR_INVALID_ARG;
+  const selkv_params& p = *params;
+  if (!std::isfinite(p.alpha) || p.select_mode < 0 || p.select_mode > 1 || p.bias_mode < 0 || p.bias_mode > 1)
+    return SELKV_ERR_INVALID_ARG;
+  if (!aligned(lengths, 4)) return SELKV_ERR_INVALID_ARG;
+  LayerPtrs P{};
+  for (int l = 0; l < num_layers; ++l) {
+    if (kept_idx[l] == nullptr || bias[l] == nullptr || !aligned(kept_idx[l], 16) || !aligned(bias[l], 16))
+      return SELKV_ERR_INVALID_ARG;
+    P.kept[l] = kept_idx[l];
+    P.bias[l] = bias[l];
+  }
+  const selkv_shape& s = *shape;
+  if (workspace == nullptr || !aligned(workspace, 256)) return SELKV_ERR_WORKSPACE;
+  if (workspace_bytes < selkv_layer_average_workspace_size(shape)) return SELKV_ERR_WORKSPACE;
+  if (p.alpha == 0.f || s.m_cap < 1) return SELKV_OK;  // every bias is 0 and stays 0
+  LayerAvgArgs a{};
+  a.B = s.batch;
+  a.Hkv = s.num_kv_heads;
+  a.m_cap = s.m_cap;
+  a.n_cap = s.n_cap;
+  a.per_head = p.select_mode == SELKV_SELECT_PER_HEAD ? 1 : 0;
+  a.L = num_layers;
+  a.alpha = p.alpha;
+  a.lengths = lengths;
+  a.flags = at<uint32_t>(workspace, 0);
+  a.acc = at<float>(workspace, sizeof(WsHeader));
+  const cudaError_t e = launch_layer_average(a, P, reinterpret_cast<cudaStream_t>(stream));
+  g_launches += (uint64_t)num_layers + 1;
+  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+}
+
 size_t selkv_decode_workspace_size(const selkv_shape* shape) {
   if (!shape_ok(shape)) return 0;
   return plan_decode(*shape).total;

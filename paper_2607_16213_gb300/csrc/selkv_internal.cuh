@@ -242,6 +242,20 @@ int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms);  // pass-1 k
 cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
+// Compensation averaged across layers (layer_average.cu).
+constexpr int kMaxLayers = 128;
+struct LayerPtrs {
+  const int32_t* kept[kMaxLayers];  // each layer's kept positions [B][units per b][m_cap]
+  float* bias[kMaxLayers];          // each layer's bias [B][Hkv][m_cap], read and rewritten
+};
+struct LayerAvgArgs {
+  int B, Hkv, m_cap, n_cap, per_head, L;
+  float alpha;
+  const int32_t* lengths;  // [B] compressed lengths
+  float* acc;              // [B][units per b][n_cap] sum over layers of expm1(bias / alpha)
+  uint32_t* flags;
+};
+cudaError_t launch_layer_average(const LayerAvgArgs& a, const LayerPtrs& P, cudaStream_t s);
 // Full cosine routing after the kept rows are in place: argmax, gate, grouping and merge.
 cudaError_t launch_route_cosine(const CompressArgs& a, cudaStream_t s);
 int cosine_kernels(int dtype, int D);  // kernels launch_route_cosine enqueues

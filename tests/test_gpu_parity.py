@@ -10,7 +10,7 @@ from oracle import selkv_oracle as O
 from paper_2607_16213_gb300 import api
 import paper_2607_16213_gb300 as S
 
-from parity import (Stats, check_decode, check_sequence, params_of, run_compress, to_dev)
+from parity import (BIAS_ATOL, Stats, check_decode, check_sequence, params_of, run_compress, to_dev)
 
 pytestmark = pytest.mark.gpu
 
@@ -395,3 +395,64 @@ def test_cosine_routing_hub_and_zero_rows():
     st = Stats()
     check_sequence(wl, x, host, 0, p, stats=st)
     print(dict(st))
+
+
+# ---------------------------------------------------------------- compensation averaged across layers
+@pytest.mark.parametrize("name,mode,bias_mode,alpha", [
+    ("bf16_ragged", O.SELECT_SHARED, O.BIAS_RATIO, 0.5),
+    ("tiny", O.SELECT_SHARED, O.BIAS_COUNT, 1.0),
+    ("bf16_mha", O.SELECT_PER_HEAD, O.BIAS_RATIO, 0.5),
+    ("bf16_d64_g4", O.SELECT_SHARED, O.BIAS_RATIO, 0.0),
+])
+def test_layer_average_bias(name, mode, bias_mode, alpha):
+    """Three layers compressed on the GPU (each checked against the oracle), then the biases
+    replaced by their cross-layer average (R21) through the C ABI, against the oracle's average
+    of the oracle's per-layer values."""
+    wl = SMALL.get(name) or PER_HEAD[name]
+    p = O.Params(select_mode=mode, bias_mode=bias_mode, alpha=alpha)
+    L = 3
+    caches, refs = [], []
+    for layer in range(L):
+        x = synth.gen_layer(wl, layer)
+        cache, host, _ = run_compress(wl, x, p)
+        caches.append(cache)
+        refs.append([check_sequence(wl, x, host, b, p) for b in range(wl.batch)])
+    shape = caches[0].shape
+    ws = api.Workspace(S.selkv_layer_average_workspace_size(shape))
+    S.check(S.selkv_layer_average_bias(shape, params_of(p), [c.debug["kept_idx"] for c in caches],
+                                       [c.bias for c in caches], caches[0].lengths, ws.buf, ws.nbytes),
+            "selkv_layer_average_bias")
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    count = bias_mode == O.BIAS_COUNT
+    for b in range(wl.batch):
+        m, n = refs[0][b]["m"], refs[0][b]["n"]
+        if alpha == 0.0:
+            for c in caches:
+                np.testing.assert_array_equal(c.bias[b, :, :m].cpu().numpy(), 0.0)
+            continue
+        # the oracle's per-slot quantity of each layer: R (ratio bias) or M (count bias)
+        x_l = [np.expm1(r[b]["bias"] / alpha) for r in refs]
+        q_l = [x if count else 1.0 + x for x in x_l]
+        want = O.layer_average_bias(q_l, [r[b]["kept_idx"] for r in refs], n, alpha, count)
+        for layer in range(L):
+            got = caches[layer].bias[b, :, :m].cpu().numpy().astype(np.float64)
+            exp = want[layer] if mode == O.SELECT_PER_HEAD else np.broadcast_to(want[layer], got.shape)
+            err = np.abs(got - exp).max()
+            assert err <= BIAS_ATOL, "layer %d seq %d: bias err %.3g" % (layer, b, err)
+
+
+def test_layer_average_one_layer_is_identity():
+    wl = SMALL["bf16_ragged"]
+    x = synth.gen_layer(wl, 0)
+    p = O.Params()
+    cache, host, _ = run_compress(wl, x, p)
+    before = cache.bias.clone()
+    ws = api.Workspace(S.selkv_layer_average_workspace_size(cache.shape))
+    S.check(S.selkv_layer_average_bias(cache.shape, params_of(p), [cache.debug["kept_idx"]], [cache.bias],
+                                       cache.lengths, ws.buf, ws.nbytes), "selkv_layer_average_bias")
+    torch.cuda.synchronize()
+    for b in range(wl.batch):
+        m = int(host["lengths"][b])
+        np.testing.assert_allclose(cache.bias[b, :, :m].cpu().numpy(), before[b, :, :m].cpu().numpy(),
+                                   rtol=0, atol=2e-6)
