@@ -37,6 +37,12 @@ namespace {
 #ifndef SELKV_DEC_PDL
 #define SELKV_DEC_PDL 1        // launch with programmatic dependent launch
 #endif
+#ifndef SELKV_DEC_PF_ROWS
+#define SELKV_DEC_PF_ROWS 128  // rows of the slice prefetched into L2 before griddepcontrol.wait
+#endif
+#ifndef SELKV_DEC_PF_AHEAD
+#define SELKV_DEC_PF_AHEAD 0   // >0: while streaming, prefetch into L2 the tile this far ahead
+#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif
@@ -253,6 +259,23 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
   if (warp == kConsumers && lane == 0) {
     prefetch_tensormap(&tmK);
     prefetch_tensormap(&tmV);
+#if SELKV_DEC_PF_ROWS > 0
+    // Warm L2 with the first rows of this CTA's slice while the previous kernel of the stream
+    // finishes (its CTAs' split combines leave HBM idle).  The slice comes from a length read
+    // before griddepcontrol.wait, which may be stale: it only steers a prefetch, and every
+    // result below is computed from data read after the wait.
+    const int Lg = min(max(ld_relaxed_gpu(a.lengths + b), 0), a.m_cap);
+    const int chk = ((Lg + S - 1) / S + kBoxRows - 1) / kBoxRows * kBoxRows;
+    const int plo = min(Lg, s * chk);
+    const int prow = min(min(Lg, plo + chk) - plo, SELKV_DEC_PF_ROWS);
+    const char* kp = static_cast<const char*>(a.Kc) + (bk * a.m_cap + plo) * (size_t)(D * 2);
+    const char* vp = static_cast<const char*>(a.Vc) + (bk * a.m_cap + plo) * (size_t)(D * 2);
+    for (int r = 0; r < prow; r += kBoxRows) {
+      const uint32_t bytes = (uint32_t)(min(kBoxRows, prow - r) * D * 2);
+      bulk_prefetch_l2(kp + (size_t)r * D * 2, bytes);
+      bulk_prefetch_l2(vp + (size_t)r * D * 2, bytes);
+    }
+#endif
   }
   // Everything above touches only this CTA's shared memory; everything below may read what
   // the previous kernel in the stream wrote (lengths, the cache, the workspace).
@@ -308,6 +331,17 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
             tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &full[st]);
         }
         issued = t + 1;
+#if SELKV_DEC_PF_AHEAD > 0
+        {
+          const int pr0 = (t + SELKV_DEC_PF_AHEAD) * kTile;  // first row of the tile ahead
+          if (pr0 >= SELKV_DEC_PF_ROWS && pr0 < hi - lo) {
+            const uint32_t bytes = (uint32_t)(min(kTile, hi - lo - pr0) * D * 2);
+            const size_t off = ((size_t)row0 + pr0) * (size_t)(D * 2);
+            bulk_prefetch_l2(static_cast<const char*>(a.Kc) + off, bytes);
+            bulk_prefetch_l2(static_cast<const char*>(a.Vc) + off, bytes);
+          }
+        }
+#endif
       }
       // every issued copy must have landed before the ring is reused or the CTA exits
       for (int t = max(0, issued - kStages); t < issued; ++t) mbar_wait(&full[t % kStages], (t / kStages) & 1);
