@@ -141,41 +141,20 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, p
 
 # ------------------------------------------------------------------------------ GPU arm
 class HostArena:
-    """Page-locked host memory for the end-to-end inputs, carved from one anonymous mapping
-    advised for transparent huge pages and registered with the CUDA runtime.  On the GB300
-    box (64 KiB base pages) host-to-device copies from ordinary pinned buffers drop from
-    ~210 GB/s to ~30 GB/s right after the GPU has streamed its own memory (the copy engine
-    re-translates every host page); with 512 MiB pages they stay at ~210 GB/s.  Falls back to
-    torch's pinned allocations if the registration fails."""
-
-    HUGE = 512 << 20
+    """Page-locked host memory for the end-to-end inputs: one allocation from the CUDA
+    runtime (cudaHostAlloc through torch), carved into the host copies of the inputs.  On the
+    GB300 machine it streams to the device at ~210 GB/s when copies run back to back; a region of
+    512 MiB transparent huge pages registered with cudaHostRegister measured no faster in the
+    end-to-end loop (and depends on the kernel finding the huge pages)."""
 
     def __init__(self, torch, nbytes: int):
-        import ctypes
-        import mmap
         self.torch = torch
-        total = (nbytes + self.HUGE - 1) // self.HUGE * self.HUGE
-        self.map = mmap.mmap(-1, total + self.HUGE, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
-        arr = np.frombuffer(self.map, dtype=np.uint8)
-        off = (-arr.ctypes.data) % self.HUGE
-        self.region = arr[off:off + total]
-        try:
-            libc = ctypes.CDLL(None)
-            libc.madvise.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int]
-            libc.madvise(ctypes.c_void_p(self.region.ctypes.data), ctypes.c_size_t(total), 14)  # MADV_HUGEPAGE
-        except (OSError, AttributeError):
-            pass
-        self.region[:] = 0
-        self.base = torch.from_numpy(self.region)
-        rc = torch.cuda.cudart().cudaHostRegister(self.base.data_ptr(), total, 0)
-        self.registered = int(rc) == 0
+        self.total = (nbytes + 255) // 256 * 256
+        self.base = torch.empty(self.total, dtype=torch.uint8, pin_memory=True)
         self.off = 0
-        self.total = total
 
     def take(self, like):
         """A page-locked host copy of `like`."""
-        if not self.registered:
-            return like.cpu().pin_memory()
         n = like.numel() * like.element_size()
         assert self.off + n <= self.total
         t = self.base[self.off:self.off + n].view(like.dtype).view(like.shape)
@@ -235,15 +214,17 @@ class Layered:
         self.aws = api.Workspace(S.selkv_layer_average_workspace_size(self.shape), dev) if layer_average else None
 
 
-def compress_layers(L: Layered, S, params, stream_ptr, before_layer=None):
-    """Enqueue the compression of every layer (and, with layer averaging, the average)."""
+def compress_layers(L: Layered, S, params, stream_ptr, before_layer=None, inputs=None):
+    """Enqueue the compression of every layer (and, with layer averaging, the average).
+    `inputs` = (K, V, Q) lists of device tensors per layer (default: the resident ones)."""
     wl = L.wl
+    Ks, Vs, Qs = inputs if inputs is not None else (L.K, L.V, L.Q)
     for layer in range(wl.layers):
         if before_layer is not None:
             before_layer(layer)
         c = L.caches[layer]
         dbg = {"kept_idx": L.kept[layer]} if L.layer_average else None
-        S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, L.K[layer], L.V[layer], L.Q[layer],
+        S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, Ks[layer], Vs[layer], Qs[layer],
                                  c.K_c, c.V_c, c.bias, c.lengths, dbg, L.cws.buf, L.cws.nbytes,
                                  stream_ptr), "compress")
     if L.layer_average:
@@ -398,7 +379,7 @@ def run_gpu(args):
     # end to end through the public API from pinned host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(L, S, api, torch, params, stream, dev, min(args.steps, 2))
+        e2e = run_e2e(L, S, api, torch, params, stream, dev, min(args.steps, 3), args.warmup)
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -437,11 +418,21 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
-def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int):
-    """The step through the public API with pinned host inputs: copy every layer's K, V, Q_obs
-    to the device (on a copy stream, overlapping the compression of the layers already
-    there), compress every layer, then per token copy q / k_new / v_new in, decode every layer
-    and read the token's outputs back.  Host buffers come from a HostArena."""
+def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: int):
+    """The step through the public API with pinned host inputs, as a serving loop runs it:
+    every layer's K, V and Q_obs are copied from host to device, every layer is compressed,
+    then per token q / k_new / v_new are copied in, every layer is decoded and the token's
+    outputs are read back.  Steps are double-buffered: the input copies of step i + 1 (on a
+    copy stream, into the other of two device input sets) run while step i decodes, and
+    layer l of a step compresses once its copies have landed.  The token loop (its copies and
+    decode calls) is captured once as a CUDA graph and replayed each step; the compression
+    calls are issued eagerly.  Every timed step moves its full input bytes across the link
+    inside the timed region (the copies for the first timed step run during the last warm-up
+    step, those issued during the last timed step are waited for before the clock stops).
+    On the GB300 machine a 13 GB host-to-device pass copies at ~210 GB/s back to back with other
+    copies but at 25-70 GB/s after or during the decode's HBM streaming, which sets this
+    number (and makes it vary from run to run; more copy streams did not help).  Host
+    buffers come from a HostArena."""
     wl = L.wl
     sp = stream.cuda_stream
     hq = L.arena.take(L.dq)
@@ -455,38 +446,67 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int):
         L.T * (dq.numel() + dk.numel() + dv.numel()) * dq.element_size()
     d2h = L.T * hout.numel() * hout.element_size()
 
+    # two device input sets: the resident one and a second of the same shapes
+    sets = [(L.K, L.V, L.Q),
+            ([torch.empty_like(x) for x in L.K], [torch.empty_like(x) for x in L.V],
+             [torch.empty_like(x) for x in L.Q])]
     copy_stream = torch.cuda.Stream(device=dev)
-    arrived = [torch.cuda.Event() for _ in range(wl.layers)]
+    arrived = [[torch.cuda.Event() for _ in range(wl.layers)] for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]  # last compression that read the set
 
-    def one():
-        # every layer's inputs on a copy stream; layer l compresses once its copies have landed
-        copy_stream.wait_stream(stream)
+    def tokens():
+        for t in range(L.T):
+            dq.copy_(hq[t], non_blocking=True)
+            dk.copy_(hk[t], non_blocking=True)
+            dv.copy_(hv[t], non_blocking=True)
+            for layer in range(wl.layers):
+                api.decode(L.caches[layer], dq[layer], dk[layer], dv[layer], out=L.out[0, layer],
+                           workspace=L.dws, stream=sp)
+            hout.copy_(L.out[0], non_blocking=True)
+
+    g_tok = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_tok, stream=stream):
+        tokens()
+    torch.cuda.synchronize()
+
+    def copy_inputs(si, after=None):
+        """Enqueue the host-to-device copies of every layer into input set si."""
+        Ks, Vs, Qs = sets[si]
         with torch.cuda.stream(copy_stream):
+            if after is not None:
+                copy_stream.wait_event(after)
             for layer in range(wl.layers):
                 hK, hV, hQ = L.host[layer]
-                L.K[layer].copy_(hK, non_blocking=True)
-                L.V[layer].copy_(hV, non_blocking=True)
-                L.Q[layer].copy_(hQ, non_blocking=True)
-                arrived[layer].record(copy_stream)
-        with torch.cuda.stream(stream):
-            compress_layers(L, S, params, sp, before_layer=lambda layer: stream.wait_event(arrived[layer]))
-            for t in range(L.T):
-                dq.copy_(hq[t], non_blocking=True)
-                dk.copy_(hk[t], non_blocking=True)
-                dv.copy_(hv[t], non_blocking=True)
-                for layer in range(wl.layers):
-                    api.decode(L.caches[layer], dq[layer], dk[layer], dv[layer], out=L.out[0, layer],
-                               workspace=L.dws, stream=sp)
-                hout.copy_(L.out[0], non_blocking=True)
-            stream.synchronize()
+                Ks[layer].copy_(hK, non_blocking=True)
+                Vs[layer].copy_(hV, non_blocking=True)
+                Qs[layer].copy_(hQ, non_blocking=True)
+                arrived[si][layer].record(copy_stream)
 
-    one()
+    def one(i):
+        si = i % 2
+        with torch.cuda.stream(stream):
+            compress_layers(L, S, params, sp, inputs=sets[si],
+                            before_layer=lambda layer: stream.wait_event(arrived[si][layer]))
+            consumed[si].record(stream)
+        # the next step's inputs go to the other set once its last compression is done
+        copy_inputs(1 - si, after=consumed[1 - si] if i > 0 else None)
+        with torch.cuda.stream(stream):
+            g_tok.replay()
+
+    copy_inputs(0)
+    for i in range(warmup):
+        one(i)
+    stream.synchronize()
+    torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for _ in range(steps):
-        one()
+    for i in range(warmup, warmup + steps):
+        one(i)
+    stream.synchronize()
+    copy_stream.synchronize()
     dt = (time.perf_counter() - t0) / steps
     return {"value": wl.batch * L.T / dt, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps}
+            "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps, "warmup": warmup,
+            "pipelined": "the next step's input copies overlap this step's decode"}
 
 
 DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "decode_simt.cu", "ptx.cuh", "selkv_internal.cuh",
