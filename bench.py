@@ -320,6 +320,14 @@ def run_gpu(args):
     torch.cuda.synchronize()
     wall = time.perf_counter() - t_wall
     clk = clocks.stop()
+    # every replayed step must have left the caches where one eager step leaves them: each
+    # layer's lengths at m_b + T (compression resets them, each token appends one row), and no
+    # device error flag raised
+    want = [int(math.floor(wl.rho * n)) + L.T for n in L.n_len]
+    for layer, c in enumerate(L.caches):
+        got = c.lengths.cpu().tolist()
+        assert got == want, "layer %d lengths %s after the timed steps, expected %s" % (layer, got[:4], want[:4])
+    assert L.cws.errors(sp) == 0 and L.dws.errors(sp) == 0, "device error flags after the timed steps"
     comp_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
     dec_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
     step_ms_total = ev[0][0].elapsed_time(ev[-1][2])
