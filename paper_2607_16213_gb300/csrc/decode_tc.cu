@@ -40,9 +40,6 @@ namespace {
 #ifndef SELKV_DEC_PF_ROWS
 #define SELKV_DEC_PF_ROWS 128  // rows of the slice prefetched into L2 before griddepcontrol.wait
 #endif
-#ifndef SELKV_DEC_PF_AHEAD
-#define SELKV_DEC_PF_AHEAD 0   // >0: while streaming, prefetch into L2 the tile this far ahead
-#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif
@@ -331,17 +328,6 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
             tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &full[st]);
         }
         issued = t + 1;
-#if SELKV_DEC_PF_AHEAD > 0
-        {
-          const int pr0 = (t + SELKV_DEC_PF_AHEAD) * kTile;  // first row of the tile ahead
-          if (pr0 >= SELKV_DEC_PF_ROWS && pr0 < hi - lo) {
-            const uint32_t bytes = (uint32_t)(min(kTile, hi - lo - pr0) * D * 2);
-            const size_t off = ((size_t)row0 + pr0) * (size_t)(D * 2);
-            bulk_prefetch_l2(static_cast<const char*>(a.Kc) + off, bytes);
-            bulk_prefetch_l2(static_cast<const char*>(a.Vc) + off, bytes);
-          }
-        }
-#endif
       }
       // every issued copy must have landed before the ring is reused or the CTA exits
       for (int t = max(0, issued - kStages); t < issued; ++t) mbar_wait(&full[t % kStages], (t / kStages) & 1);

@@ -219,6 +219,51 @@ def test_decode_edge_lengths():
     check_decode(out[1], want, "fp32")
 
 
+def test_decode_back_to_back_appends_sweep_the_split_slices():
+    """bf16 decode calls enqueued back to back on one cache, each appending a row, while the
+    lengths sweep through every point where the per-split row slices move.  Each launch reads
+    the length before waiting for the previous launch (to prefetch and to issue its first tile
+    early), so that read is often one row stale: both the kept and the discarded early first
+    tile are exercised.  Every step must match exact attention over the rows present then
+    (bias per row, 0 for appended rows)."""
+    B, Hq, Hkv, d, m_cap = 2, 8, 2, 128, 4224
+    L0 = [1, 700]
+    T, burst = 3500, 25
+    shape = api.make_shape("bf16", B, Hq, Hkv, d, 32, m_cap, m_cap)
+    g = torch.Generator().manual_seed(21)
+    cache = api.alloc_compressed(shape)
+    cache.K_c.copy_(torch.randn(cache.K_c.shape, generator=g))
+    cache.V_c.copy_(torch.randn(cache.V_c.shape, generator=g))
+    cache.bias.copy_(0.5 * torch.rand(cache.bias.shape, generator=g))
+    cache.lengths.copy_(torch.tensor(L0, dtype=torch.int32))
+    qs = torch.randn((T, B, Hq, d), generator=g).to(torch.bfloat16).cuda()
+    ks = torch.randn((T, B, Hkv, d), generator=g).to(torch.bfloat16).cuda()
+    vs = torch.randn((T, B, Hkv, d), generator=g).to(torch.bfloat16).cuda()
+    outs = torch.empty((burst, B, Hq, d), dtype=torch.bfloat16, device="cuda")
+    Kh = cache.K_c.double().cpu().numpy()
+    Vh = cache.V_c.double().cpu().numpy()
+    bh = cache.bias.double().cpu().numpy()
+    qh, kh, vh = (x.double().cpu().numpy() for x in (qs, ks, vs))
+    ws = api.Workspace(S.selkv_decode_workspace_size(shape))
+    for t0 in range(0, T, burst):
+        for i in range(burst):
+            t = t0 + i
+            api.decode(cache, qs[t], ks[t], vs[t], out=outs[i], workspace=ws)
+        got = outs.float().cpu().numpy()
+        for i in range(burst):
+            t = t0 + i
+            for b in range(B):
+                L = L0[b] + t
+                Kh[b, :, L] = kh[t, b]
+                Vh[b, :, L] = vh[t, b]
+                bh[b, :, L] = 0.0
+                want = O.decode(qh[t, b], Kh[b], Vh[b], bh[b], L + 1)
+                check_decode(got[i, b], want, "bf16", "step %d seq %d" % (t, b))
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    np.testing.assert_array_equal(cache.lengths.cpu().numpy(), np.array(L0) + T)
+
+
 def test_repeat_runs_are_bitwise_identical():
     wl = SMALL["bf16_ragged"]
     x = synth.gen_layer(wl, 5)
