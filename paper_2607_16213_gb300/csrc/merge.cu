@@ -277,6 +277,69 @@ __device__ __forceinline__ float transpose_reduce16(const float (&p)[kBatch], in
   return t + __shfl_xor_sync(0xffffffffu, t, 1);
 }
 
+#ifndef SELKV_MERGE_COPY
+#define SELKV_MERGE_COPY 1  // bucket routing without repositioning: the merge warps copy the kept rows
+#endif
+template <int BYTES>
+struct RawOf;
+template <>
+struct RawOf<4> { using type = uint32_t; };
+template <>
+struct RawOf<8> { using type = uint2; };
+template <>
+struct RawOf<16> { using type = uint4; };
+
+// Copy of bucket X's kept rows into their slots: every key row, and every value row but the
+// merge target's (written merged by the caller); ratio 1 and count 0 for the slots other
+// than the target's.  Loads of up to 8 kept positions are issued before their stores.  The
+// same work as copy_kernel does for every slot, done by the warp that owns the bucket.
+template <typename T, int D>
+__device__ __forceinline__ void copy_kept_rows(const CompressArgs& a, size_t bk, int base, bool keptX, int slotX,
+                                               int tau, int lane) {
+  constexpr int PER = D / 32;
+  using Raw = typename RawOf<PER * (int)sizeof(T)>::type;
+  const T* Kb = static_cast<const T*>(a.K) + bk * a.n_cap * D;
+  const T* Vb = static_cast<const T*>(a.V) + bk * a.n_cap * D;
+  T* Kc = static_cast<T*>(a.Kc) + bk * a.m_cap * D;
+  T* Vc = static_cast<T*>(a.Vc) + bk * a.m_cap * D;
+  if (keptX) {
+    if (slotX < 0 || slotX >= a.m_cap) {
+      raise_flag(a.flags, SELKV_DEVERR_COUNT);
+    } else if (base + lane != tau) {
+      a.ratio[bk * a.m_cap + slotX] = 1.f;
+      a.mcount[bk * a.m_cap + slotX] = 0.f;
+      if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slotX] = 1.f;
+    }
+    const size_t o = bk * a.n_cap + base + lane;
+    if (a.dbg_target) a.dbg_target[o] = -1;
+    if (a.dbg_gate) a.dbg_gate[o] = 0.f;
+    if (a.dbg_decision) a.dbg_decision[o] = 2;
+  }
+  uint32_t km = __ballot_sync(0xffffffffu, keptX && slotX >= 0 && slotX < a.m_cap);
+  while (km) {
+    constexpr int kN = 4;
+    int pos[kN], slot[kN];
+    Raw kr[kN], vr[kN];
+#pragma unroll
+    for (int i = 0; i < kN; ++i) {
+      const int bit = km ? __ffs(km) - 1 : -1;
+      km &= km ? km - 1u : 0u;
+      pos[i] = bit < 0 ? -1 : base + bit;
+      slot[i] = __shfl_sync(0xffffffffu, slotX, bit < 0 ? 0 : bit);
+      if (pos[i] >= 0) {
+        kr[i] = *reinterpret_cast<const Raw*>(Kb + (size_t)pos[i] * D + lane * PER);
+        if (pos[i] != tau) vr[i] = *reinterpret_cast<const Raw*>(Vb + (size_t)pos[i] * D + lane * PER);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kN; ++i) {
+      if (pos[i] < 0) continue;
+      *reinterpret_cast<Raw*>(Kc + (size_t)slot[i] * D + lane * PER) = kr[i];
+      if (pos[i] != tau) *reinterpret_cast<Raw*>(Vc + (size_t)slot[i] * D + lane * PER) = vr[i];
+    }
+  }
+}
+
 template <typename T, int D>
 __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   constexpr int PER = D / 32;  // elements of a row per lane
@@ -307,7 +370,9 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
   const float* vn = a.vnorm + bk * a.n_cap;
   const float AX = inX ? A[base + lane] : 0.f;
   const float NX = inX ? vn[base + lane] : 0.f;
-  if (tau < 0) {
+  const bool fuse_copy = SELKV_MERGE_COPY && a.rope == SELKV_ROPE_OFF;
+  const int slotX = (fuse_copy && inX) ? a.slot_of[su * a.n_cap + base + lane] : -1;
+  if (tau < 0) {  // (then X keeps no token: nothing to copy)
     // Empty bucket: under EXPAND a neighbour's warp owns these tokens; under DROP (or with
     // nothing kept at all) they stay without target.
     if (a.empty_bucket == SELKV_EMPTY_DROP || a.seq_m[b] == 0) {
@@ -465,6 +530,7 @@ __global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
     a.mcount[bk * a.m_cap + slot] = (float)merged;
     if (a.dbg_ratio) a.dbg_ratio[bk * a.m_cap + slot] = R_tau;
   }
+  if (fuse_copy) copy_kept_rows<T, D>(a, bk, base, keptX, slotX, tau, lane);
 }
 
 // bias[b][kv][slot] = alpha * ln(mean over KV heads of R[b][kv][slot])   (Sec. 3.6, GQA);
@@ -493,7 +559,9 @@ template <typename T, int D>
 void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
   constexpr int kPieces = D * (int)sizeof(T) / 16;
   const size_t copy_threads = (size_t)a.Hkv * a.m_cap * 2 * kPieces;
-  copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
+  // with the bucket routing and no repositioning the merge warps copy the kept rows themselves
+  if (!(SELKV_MERGE_COPY && a.routing == SELKV_ROUTE_BUCKET && a.rope == SELKV_ROPE_OFF))
+    copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
   if (a.routing == SELKV_ROUTE_BUCKET) merge_kernel<T, D><<<dim3(a.nbk, a.B * a.Hkv), 32, 0, s>>>(a);
 }
 
