@@ -16,7 +16,6 @@ namespace {
 
 // Kernels enqueued by each call (diagnostic count, see selkv_kernel_launches).
 std::atomic<uint64_t> g_launches{0};
-constexpr int kCompressKernels = 18;  // with the tensor-core scoring (20 with the CUDA-core one)
 constexpr int kDecodeKernels = 1;
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -144,6 +143,24 @@ T* at(void* ws, size_t off) {
 }  // namespace
 
 void note_launches(int kernels) { g_launches += (uint64_t)kernels; }
+
+// Kernels one selkv_compress call enqueues, mirroring the launch code: set-up and value norms;
+// the scoring's two passes and the fold of the row statistics between them; the selection
+// (init, pooling with digit pass 0, digit passes 1-2 and the tie step of each KV head's
+// top-k, then, in the shared mode only, the union with the trim's pass 0, its passes 1-2 and
+// tie step; finally the compaction's count and write); the RoPE tables when repositioning;
+// the routing and merge (bucket: route and merge, plus the kept-row copy unless the merge
+// does it; cosine: the copy and the cosine kernels); the bias.
+int compress_kernel_count(const CompressArgs& a) {
+  int k = 2 + 3;
+  k += a.per_head ? 7 : 11;
+  if (a.rope != SELKV_ROPE_OFF) k += 1;
+  if (a.routing == SELKV_ROUTE_COSINE)
+    k += 1 + (a.m_cap > 0 ? cosine_kernels(a.dtype, a.D) : 0);
+  else
+    k += 2 + (merge_copies_kept_rows(a) ? 0 : 1);
+  return k + 1;
+}
 
 }  // namespace selkv
 
@@ -322,9 +339,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   if (e == cudaSuccess)
     e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
   if (e == cudaSuccess) e = launch_merge(a, st);
-  g_launches += (score_uses_tc(a.dtype, a.D, a.R) ? kCompressKernels : kCompressKernels + 2) -
-                (a.per_head ? 4 : 0) + (a.rope ? 1 : 0) +  // no union / trim in per-head mode
-                (a.routing == SELKV_ROUTE_COSINE ? (s.m_cap > 0 ? cosine_kernels(a.dtype, a.D) : 0) - 2 : 0);
+  g_launches += (uint64_t)compress_kernel_count(a);
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

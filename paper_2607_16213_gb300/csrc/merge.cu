@@ -560,12 +560,16 @@ void launch_merge_t(const CompressArgs& a, cudaStream_t s) {
   constexpr int kPieces = D * (int)sizeof(T) / 16;
   const size_t copy_threads = (size_t)a.Hkv * a.m_cap * 2 * kPieces;
   // with the bucket routing and no repositioning the merge warps copy the kept rows themselves
-  if (!(SELKV_MERGE_COPY && a.routing == SELKV_ROUTE_BUCKET && a.rope == SELKV_ROPE_OFF))
+  if (!merge_copies_kept_rows(a))
     copy_kernel<T, D><<<dim3((unsigned)((copy_threads + 255) / 256), a.B), 256, 0, s>>>(a);
   if (a.routing == SELKV_ROUTE_BUCKET) merge_kernel<T, D><<<dim3(a.nbk, a.B * a.Hkv), 32, 0, s>>>(a);
 }
 
 }  // namespace
+
+bool merge_copies_kept_rows(const CompressArgs& a) {
+  return SELKV_MERGE_COPY && a.routing == SELKV_ROUTE_BUCKET && a.rope == SELKV_ROPE_OFF;
+}
 
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s) {
   if (a.rope != SELKV_ROPE_OFF) {

@@ -308,6 +308,10 @@ cudaError_t set_smem_once(int bytes) {
   return e;
 }
 
+// True when the merge kernel copies the kept rows itself (bucket routing, no repositioning),
+// so the separate copy kernel is not launched.
+bool merge_copies_kept_rows(const CompressArgs& a);
+
 int decode_splits(int B, int Hkv, int m_cap, int num_sms);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);     // dispatch by dtype
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);  // bf16: TMA + tensor cores
