@@ -8,7 +8,7 @@
 #include "selkv_internal.cuh"
 
 namespace selkv {
-cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
+cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, const SelectWs& w, cudaStream_t s);
 cudaError_t launch_vnorm(const CompressArgs& a, cudaStream_t s);
 cudaError_t launch_merge(const CompressArgs& a, cudaStream_t s);
 
@@ -146,14 +146,14 @@ void note_launches(int kernels) { g_launches += (uint64_t)kernels; }
 
 // Kernels one selkv_compress call enqueues, mirroring the launch code: set-up and value norms;
 // the scoring's two passes and the fold of the row statistics between them; the selection
-// (init, pooling with digit pass 0, digit passes 1-2 and the tie step of each KV head's
-// top-k, then, in the shared mode only, the union with the trim's pass 0, its passes 1-2 and
-// tie step; finally the compaction's count and write); the RoPE tables when repositioning;
+// (pooling with digit pass 0 and digit passes 1-2 of each KV head's top-k, then, in the
+// shared mode only, the union with the trim's pass 0 and its passes 1-2; finally the
+// compaction's count and write); the RoPE tables when repositioning;
 // the routing and merge (bucket: route and merge, plus the kept-row copy unless the merge
 // does it; cosine: the copy and the cosine kernels); the bias.
 int compress_kernel_count(const CompressArgs& a) {
   int k = 2 + 3;
-  k += a.per_head ? 7 : 11;
+  k += a.per_head ? 5 : 8;
   if (a.rope != SELKV_ROPE_OFF) k += 1;
   if (a.routing == SELKV_ROUTE_COSINE)
     k += 1 + (a.m_cap > 0 ? cosine_kernels(a.dtype, a.D) : 0);
@@ -322,7 +322,8 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     a.dbg_ratio = debug->ratio;
   }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = launch_setup(a, tab, st);
+  const SelectWs sw = carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap);
+  cudaError_t e = launch_setup(a, tab, sw, st);
   {
     // value norms on the side stream (they need seq_n from the set-up; selection needs them)
     std::lock_guard<std::mutex> lock(g_side_mu);
@@ -337,7 +338,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     if (e == cudaSuccess) e = side != nullptr ? cudaStreamWaitEvent(st, side->join, 0) : launch_vnorm(a, st);
   }
   if (e == cudaSuccess)
-    e = launch_select_grid(a, carve_select_ws(at<char>(workspace, plan.select), s.batch, s.num_kv_heads, s.n_cap), st);
+    e = launch_select_grid(a, sw, st);
   if (e == cudaSuccess) e = launch_merge(a, st);
   g_launches += (uint64_t)compress_kernel_count(a);
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;

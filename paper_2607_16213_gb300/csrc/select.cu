@@ -6,11 +6,17 @@
 namespace selkv {
 namespace {
 
-__global__ void setup_kernel(SeqTable tab, int B, int32_t* seq_n, int32_t* seq_m, int32_t* lengths) {
-  for (int b = threadIdx.x; b < B; b += blockDim.x) {
-    seq_n[b] = tab.n[b];
-    seq_m[b] = tab.m[b];
-    lengths[b] = tab.m[b];
+// Sequence table, output lengths and the selection's initial radix states.
+__global__ void setup_kernel(SeqTable tab, CompressArgs a, SelectWs w) {
+  for (int b = threadIdx.x; b < a.B; b += blockDim.x) {
+    a.seq_n[b] = tab.n[b];
+    a.seq_m[b] = tab.m[b];
+    a.lengths[b] = tab.m[b];
+  }
+  const int units = a.B * a.Hkv;
+  for (int i = threadIdx.x; i < units + a.B; i += blockDim.x) {
+    const int b = i >= units ? i - units : i / a.Hkv;
+    select_init_state(a, w, i, tab.n[b], tab.m[b]);
   }
 }
 
@@ -57,8 +63,8 @@ void launch_norms(const CompressArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s) {
-  setup_kernel<<<1, 256, 0, s>>>(tab, a.B, a.seq_n, a.seq_m, a.lengths);
+cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, const SelectWs& w, cudaStream_t s) {
+  setup_kernel<<<1, 256, 0, s>>>(tab, a, w);
   return cudaGetLastError();
 }
 

@@ -124,6 +124,55 @@ __global__ __launch_bounds__(kBlock) void pool_hist0_kernel(CompressArgs a, Sele
   if (active) flush_and_select(sh, w.topk_hist + (size_t)u * 3 * kBins, st, 0, gridDim.x, &s_last);
 }
 
+// After the last pass: when more entries equal the threshold than are still needed, find the
+// position of the last one taken (lowest positions first).  Run by the CTA that picked the
+// last digit of unit u, right after picking it.
+__device__ __noinline__ void resolve_tie(const CompressArgs& a, RadixState* st, const float* key, const uint8_t* member, int u,
+                            int per_seq) {
+  __shared__ uint32_t wcnt[32];
+  __shared__ uint32_t s_total;
+  __shared__ int s_jcut;
+  const int b = u / per_seq;
+  __syncthreads();
+  const uint32_t T = __ldcg(&st->prefix), krem = __ldcg(&st->krem);
+  if (__ldcg(&st->count_eq) == krem) {
+    if (threadIdx.x == 0) st->jcut = INT_MAX;
+    return;
+  }
+  const int ncand = a.seq_n[b] - a.recent;
+  const float* k = key + (size_t)u * a.n_cap;
+  const uint8_t* mb = member != nullptr ? member + (size_t)u * a.n_cap : nullptr;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  if (threadIdx.x == 0) s_jcut = INT_MAX;
+  uint32_t base = 0;
+  for (int j0 = 0; j0 < ncand; j0 += blockDim.x) {
+    const int j = j0 + threadIdx.x;
+    const bool f = j < ncand && (mb == nullptr || mb[j]) && __float_as_uint(k[j]) == T;
+    const unsigned bal = __ballot_sync(0xffffffffu, f);
+    if (lane == 0) wcnt[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t v = lane < nwarps ? wcnt[lane] : 0u;
+      uint32_t incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      if (lane < nwarps) wcnt[lane] = incl - v;
+      if (lane == 31) s_total = incl;
+    }
+    __syncthreads();
+    const uint32_t rank = base + wcnt[warp] + __popc(bal & ((1u << lane) - 1u)) + 1u;
+    if (f && rank == krem) s_jcut = j;
+    base += s_total;
+    __syncthreads();
+    if (base >= krem) break;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) st->jcut = s_jcut;
+}
+
 // Digit pass `pass` (1 or 2) of a set of units.  Unit u's keys are key[u * stride + j] for
 // j < len(u); member (optional) filters them.  Grid (position blocks, units).
 __global__ __launch_bounds__(kBlock) void hist_kernel(CompressArgs a, RadixState* states, uint32_t* hist,
@@ -151,55 +200,10 @@ __global__ __launch_bounds__(kBlock) void hist_kernel(CompressArgs a, RadixState
     if ((x & mask) == prefix) atomicAdd(&sh[(x >> shift) & dmask], 1u);
   }
   flush_and_select(sh, hist + ((size_t)u * 3 + pass) * kBins, st, pass, gridDim.x, &s_last);
-}
-
-// After the last pass: when more entries equal the threshold than are still needed, find the
-// position of the last one taken (lowest positions first).  One CTA per unit.
-__global__ __launch_bounds__(1024) void tie_kernel(CompressArgs a, RadixState* states, const float* key,
-                                                   const uint8_t* member, int per_seq) {
-  __shared__ uint32_t wcnt[32];
-  __shared__ uint32_t s_total;
-  __shared__ int s_jcut;
-  const int u = blockIdx.x, b = u / per_seq;
-  RadixState* st = &states[u];
-  if (st->active == 0u) return;
-  const uint32_t T = st->prefix, krem = st->krem;
-  if (st->count_eq == krem) {
-    if (threadIdx.x == 0) st->jcut = INT_MAX;
-    return;
+  if (pass == 2 && s_last) {
+    __threadfence();
+    resolve_tie(a, st, key, member, u, per_seq);
   }
-  const int ncand = a.seq_n[b] - a.recent;
-  const float* k = key + (size_t)u * a.n_cap;
-  const uint8_t* mb = member != nullptr ? member + (size_t)u * a.n_cap : nullptr;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) s_jcut = INT_MAX;
-  uint32_t base = 0;
-  for (int j0 = 0; j0 < ncand; j0 += blockDim.x) {
-    const int j = j0 + threadIdx.x;
-    const bool f = j < ncand && (mb == nullptr || mb[j]) && __float_as_uint(k[j]) == T;
-    const unsigned bal = __ballot_sync(0xffffffffu, f);
-    if (lane == 0) wcnt[warp] = __popc(bal);
-    __syncthreads();
-    if (warp == 0) {
-      const uint32_t v = wcnt[lane];
-      uint32_t incl = v;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
-      }
-      wcnt[lane] = incl - v;
-      if (lane == 31) s_total = incl;
-    }
-    __syncthreads();
-    const uint32_t rank = base + wcnt[warp] + __popc(bal & ((1u << lane) - 1u)) + 1u;
-    if (f && rank == krem) s_jcut = j;
-    base += s_total;
-    __syncthreads();
-    if (base >= krem) break;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) st->jcut = s_jcut;
 }
 
 // Union over KV heads, the trim key (score summed over KV heads), |U|, and digit pass 0 of
@@ -351,32 +355,6 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
   if (blk == (int)gridDim.x - 1 && threadIdx.x == 0 && (int)base != a.seq_m[b]) raise_flag(a.flags, SELKV_DEVERR_COUNT);
 }
 
-// Initial radix states: top-m_s per (b, kv) and the trim per b.
-__global__ void select_init_kernel(CompressArgs a, SelectWs w) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  const int units = a.B * a.Hkv;
-  if (i < units + a.B) {
-    const bool trim = i >= units;
-    const int b = trim ? i - units : i / a.Hkv;
-    const int k = a.seq_m[b] - a.recent;
-    const int ncand = a.seq_n[b] - a.recent;
-    RadixState s{};
-    s.krem = (uint32_t)max(k, 0);
-    s.jcut = INT_MAX;
-    if (trim) {
-      s.active = k > 0 ? 1u : 0u;  // the union kernel switches it off when |U| <= m_s
-    } else if (k <= 0) {
-      s.prefix = 0xffffffffu;  // select nothing
-      s.jcut = -1;
-    } else if (k >= ncand) {
-      s.prefix = 0u;  // select every candidate
-    } else {
-      s.active = 1u;
-    }
-    if (trim) w.trim[b] = s; else w.topk[i] = s;
-  }
-}
-
 }  // namespace
 
 size_t select_ws_bytes(int B, int Hkv, int n_cap) {
@@ -408,23 +386,20 @@ SelectWs carve_select_ws(void* base, int B, int Hkv, int n_cap) {
   return w;
 }
 
-// Pooling and the whole selection: 10 kernels (6 in the per-head mode) and one memset, all
-// on `s`, no host sync.
+// Pooling and the whole selection: 8 kernels (5 in the per-head mode) and one memset, all on
+// `s`, no host sync (the radix states are initialised by the set-up kernel).
 cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStream_t s) {
   const int units = a.B * a.Hkv;
   const int blocks = (a.n_cap + kSpan - 1) / kSpan;
   cudaError_t e = cudaMemsetAsync(w.topk_hist, 0, w.hist_bytes, s);
   if (e != cudaSuccess) return e;
-  select_init_kernel<<<(units + a.B + 255) / 256, 256, 0, s>>>(a, w);
   pool_hist0_kernel<<<dim3(blocks, units), kBlock, 0, s>>>(a, w);
   for (int pass = 1; pass < 3; ++pass)
     hist_kernel<<<dim3(blocks, units), kBlock, 0, s>>>(a, w.topk, w.topk_hist, a.score, nullptr, a.Hkv, pass);
-  tie_kernel<<<units, 1024, 0, s>>>(a, w.topk, a.score, nullptr, a.Hkv);
   if (!a.per_head) {  // union over KV heads and the trim (shared mode only)
     union_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w);
     for (int pass = 1; pass < 3; ++pass)
       hist_kernel<<<dim3(blocks, a.B), kBlock, 0, s>>>(a, w.trim, w.trim_hist, w.tkey, w.uflag, 1, pass);
-    tie_kernel<<<a.B, 1024, 0, s>>>(a, w.trim, w.tkey, w.uflag, 1);
   }
   const int sel_units = a.per_head ? units : a.B;
   compact_count_kernel<<<dim3(blocks, sel_units), kBlock, 0, s>>>(a, w);

@@ -232,6 +232,31 @@ struct SelectWs {
   float* tkey;          // [B][n_cap] score summed over KV heads
   uint8_t* uflag;       // [B][n_cap] member of the union
 };
+// Initial radix state i of units + B: top-m_s per (b, kv), then the trim per b.  Called by
+// the set-up kernel with seq_n and seq_m of this call.
+__device__ __forceinline__ void select_init_state(const CompressArgs& a, const SelectWs& w, int i, int n_b, int m_b) {
+  const int units = a.B * a.Hkv;
+  const bool trim = i >= units;
+  const int b = trim ? i - units : i / a.Hkv;
+  (void)b;
+  const int k = m_b - a.recent;
+  const int ncand = n_b - a.recent;
+  RadixState s{};
+  s.krem = (uint32_t)max(k, 0);
+  s.jcut = INT_MAX;
+  if (trim) {
+    s.active = k > 0 ? 1u : 0u;  // the union kernel switches it off when |U| <= m_s
+  } else if (k <= 0) {
+    s.prefix = 0xffffffffu;  // select nothing
+    s.jcut = -1;
+  } else if (k >= ncand) {
+    s.prefix = 0u;  // select every candidate
+  } else {
+    s.active = 1u;
+  }
+  if (trim) w.trim[i - units] = s; else w.topk[i] = s;
+}
+
 size_t select_ws_bytes(int B, int Hkv, int n_cap);
 SelectWs carve_select_ws(void* base, int B, int Hkv, int n_cap);
 cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStream_t s);

@@ -88,6 +88,33 @@ def test_compress_edge_cases(case):
         np.testing.assert_array_equal(host["bias"][0, :, :m], 0.0)
 
 
+@pytest.mark.parametrize("per_head", [False, True])
+def test_compress_exact_ties_take_the_lowest_positions(per_head):
+    """Every token of a sequence identical: the attention of all fully visible candidates, and
+    so their pooled scores, are exactly equal (bit-identical on the GPU as in the oracle), and
+    the top-m_s is decided by the position tie-break alone: lower positions first.  The kept
+    set must equal the oracle's exactly (no near-tie allowance)."""
+    wl = SMALL["bf16_ragged"].with_(batch=2, ragged=None)
+    x = synth.gen_layer(wl, 7)
+    x["K"][:] = x["K"][:, :, :1, :]
+    x["V"][:] = x["V"][:, :, :1, :]
+    p = O.Params(select_mode=O.SELECT_PER_HEAD if per_head else O.SELECT_SHARED)
+    _, host, _ = run_compress(wl, x, p)
+    for b in range(wl.batch):
+        n = int(x["n_len"][b])
+        ref = O.compress(x["K"][b].astype(np.float64), x["V"][b].astype(np.float64),
+                         x["Q_obs"][b].astype(np.float64), n, wl.rho, p)
+        m = int(host["lengths"][b])
+        assert m == ref.m
+        if per_head:
+            np.testing.assert_array_equal(host["kept_idx"][b, :, :m], ref.kept_idx)
+        else:
+            np.testing.assert_array_equal(host["kept_idx"][b, :m], ref.kept_idx)
+            # the tie really decided it: the kept candidates are a prefix of the tied run
+            kept = ref.kept_idx[ref.kept_idx < n - p.recent]
+            assert kept[-1] < n - wl.obs_window
+
+
 def test_window_equals_sequence():
     wl = SMALL["tiny"].with_(n=96, obs_window=96, rho=0.5)
     x = synth.gen_layer(wl, 0)
