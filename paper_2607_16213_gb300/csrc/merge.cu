@@ -341,7 +341,10 @@ __device__ __forceinline__ void copy_kept_rows(const CompressArgs& a, size_t bk,
 }
 
 template <typename T, int D>
-__global__ __launch_bounds__(32, 24) void merge_kernel(CompressArgs a) {
+#ifndef SELKV_MERGE_MINB
+#define SELKV_MERGE_MINB 32  // one-warp merge CTAs resident per SM (32: the most an SM holds)
+#endif
+__global__ __launch_bounds__(32, SELKV_MERGE_MINB) void merge_kernel(CompressArgs a) {
   constexpr int PER = D / 32;  // elements of a row per lane
   const int lane = threadIdx.x;
   const int X = blockIdx.x;
