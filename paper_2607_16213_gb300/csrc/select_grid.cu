@@ -19,6 +19,9 @@
 namespace selkv {
 namespace {
 
+#ifndef SELKV_SEL_MINB
+#define SELKV_SEL_MINB 4  // CTAs per SM the pooling and union kernels are compiled for (full occupancy)
+#endif
 constexpr int kBlock = 512;                 // threads per CTA
 constexpr int kPerThread = 2;               // positions per thread
 constexpr int kSpan = kBlock * kPerThread;  // positions per CTA
@@ -85,7 +88,7 @@ __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, 
 
 // Pooling of Eq. 1's score over the candidates, fused with digit pass 0 of each KV head's
 // top-m_s.  Grid (position blocks, B * Hkv).
-__global__ __launch_bounds__(kBlock) void pool_hist0_kernel(CompressArgs a, SelectWs w) {
+__global__ __launch_bounds__(kBlock, SELKV_SEL_MINB) void pool_hist0_kernel(CompressArgs a, SelectWs w) {
   __shared__ uint32_t sh[kBins];
   __shared__ bool s_last;
   const int u = blockIdx.y, b = u / a.Hkv;
@@ -208,7 +211,7 @@ __global__ __launch_bounds__(kBlock) void hist_kernel(CompressArgs a, RadixState
 
 // Union over KV heads, the trim key (score summed over KV heads), |U|, and digit pass 0 of
 // the trim.  Grid (position blocks, B).
-__global__ __launch_bounds__(kBlock) void union_kernel(CompressArgs a, SelectWs w) {
+__global__ __launch_bounds__(kBlock, SELKV_SEL_MINB) void union_kernel(CompressArgs a, SelectWs w) {
   __shared__ uint32_t sh[kBins];
   __shared__ uint32_t s_cnt;
   __shared__ bool s_last;
