@@ -139,6 +139,22 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, p
                 decode_s_per_layer_token=per_layer_tok, sample_wall_s=t_comp + t_dec)
 
 
+# ------------------------------------------------------------------------------ ranks
+def max_over_ranks(x: float, torch, dist, device) -> float:
+    """The largest x over all ranks (x itself without a process group of several ranks):
+    the job's time is that of its slowest rank."""
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() < 2:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, units_per_rank: float, seconds: float) -> float:
+    """Units processed by all ranks per second (weak scaling: every rank does the same work)."""
+    return world * units_per_rank / seconds
+
+
 # ------------------------------------------------------------------------------ GPU arm
 class HostArena:
     """Page-locked host memory for the end-to-end inputs: one allocation from the CUDA
@@ -335,15 +351,12 @@ def run_gpu(args):
     assert L.cws.errors(sp) == 0 and L.dws.errors(sp) == 0, "device error flags after the timed steps"
     comp_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
     dec_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
-    step_ms_total = ev[0][0].elapsed_time(ev[-1][2])
+    step_ms_total = max_over_ranks(ev[0][0].elapsed_time(ev[-1][2]), torch, dist, dev)
     if world > 1:
-        t = torch.tensor([step_ms_total], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        step_ms_total = float(t.item())
         dist.barrier()
     ms_per_step = step_ms_total / args.steps
     tokens_per_step = wl.batch * L.T
-    value = world * tokens_per_step * args.steps / (step_ms_total / 1e3)
+    value = whole_job_rate(world, tokens_per_step * args.steps, step_ms_total / 1e3)
     dec_ms_avg = sum(dec_ms) / len(dec_ms)
     comp_ms_avg = sum(comp_ms) / len(comp_ms)
     decode_tok_s = tokens_per_step / (dec_ms_avg / 1e3)
@@ -393,6 +406,8 @@ def run_gpu(args):
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(L, S, api, torch, params, stream, dev, min(args.steps, 3), args.warmup)
+        e2e["ms_per_step"] = max_over_ranks(e2e["ms_per_step"], torch, dist, dev)
+        e2e["value"] = whole_job_rate(world, wl.batch * L.T, e2e["ms_per_step"] / 1e3)
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,

@@ -1,0 +1,64 @@
+"""The multi-rank host logic of bench.py on CPU: two gloo ranks (one process each, launched
+as torchrun would, rendezvous on 127.0.0.1).  Every rank replays its own replica of the
+workload (weak scaling, no collective on the data path); the job's time is the slowest
+rank's, and the rate counts every rank's tokens."""
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+import bench
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank(rank, world, port, local, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world))
+    import torch
+    import torch.distributed as dist
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        out[rank] = bench.max_over_ranks(local[rank], torch, dist, "cpu")
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+def test_slowest_rank_sets_the_time_gloo_world_2():
+    import torch.multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as manager:
+        out = manager.dict()
+        mp.start_processes(_rank, args=(2, _free_port(), [183.0, 191.5], out), nprocs=2, join=True,
+                           start_method="spawn")
+        got = dict(out)
+    assert got == {0: 191.5, 1: 191.5}
+
+
+def test_single_process_time_is_local():
+    import torch
+    import torch.distributed as dist
+    assert bench.max_over_ranks(12.5, torch, dist, "cpu") == 12.5
+
+
+def test_whole_job_rate_counts_every_rank():
+    # 256 tokens per rank and step, 2 ranks, 5 steps in 0.5 s
+    assert bench.whole_job_rate(2, 256 * 5, 0.5) == pytest.approx(5120.0)
+    assert bench.whole_job_rate(1, 256 * 5, 0.5) == pytest.approx(2560.0)
+
+
+def test_reference_arm_prints_on_rank_0_only():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1"],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert r.stdout.strip() == ""
