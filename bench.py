@@ -182,8 +182,10 @@ class HostArena:
 class Layered:
     """Device-resident inputs and outputs of every layer."""
 
-    def __init__(self, wl, torch, api, S, dev, pinned_host: bool, layer_average: bool = False):
+    def __init__(self, wl, torch, api, S, dev, pinned_host: bool, layer_average: bool = False,
+                 compress_streams: int = 1):
         self.wl = wl
+        self.torch = torch
         B, Hq, Hkv, d, W = wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.obs_window
         tdt = api.torch_dtype(api.dtype_code(wl.dtype))
         self.n_len = [int(v) for v in synth.seq_lengths(wl)]
@@ -221,6 +223,11 @@ class Layered:
         self.dv = torch.from_numpy(np.stack(vs, 1)).to(dev).to(tdt)
         self.out = torch.empty((self.T, wl.layers, B, Hq, d), dtype=tdt, device=dev)
         self.cws = api.Workspace(S.selkv_compress_workspace_size(self.shape), dev)
+        # layers are compressed on `compress_streams` streams in turn (the caller's first), each
+        # with its own workspace; the extra streams fork from the caller's and join it again
+        self.comp_streams = [torch.cuda.Stream(device=dev) for _ in range(max(1, compress_streams) - 1)]
+        self.comp_ws = [api.Workspace(S.selkv_compress_workspace_size(self.shape), dev)
+                        for _ in self.comp_streams]
         self.dws = api.Workspace(S.selkv_decode_workspace_size(self.shape), dev)
         # compensation averaged across layers: each layer's kept positions are kept for it
         self.layer_average = layer_average
@@ -231,18 +238,32 @@ class Layered:
 
 
 def compress_layers(L: Layered, S, params, stream_ptr, before_layer=None, inputs=None):
-    """Enqueue the compression of every layer (and, with layer averaging, the average).
-    `inputs` = (K, V, Q) lists of device tensors per layer (default: the resident ones)."""
+    """Enqueue the compression of every layer (and, with layer averaging, the average) on the
+    current stream (`stream_ptr`), layer l on stream l mod (1 + extra streams) with that
+    stream's workspace: the compressions of a model's layers after prefill are independent, and
+    the latency-bound selection kernels of one layer leave room for another layer's work.
+    `inputs` = (K, V, Q) lists of device tensors per layer (default: the resident ones);
+    `before_layer(layer, stream)` may make the stream that compresses the layer wait."""
     wl = L.wl
+    torch = L.torch
+    main = torch.cuda.current_stream()
+    assert main.cuda_stream == stream_ptr, "compress_layers enqueues on the current stream"
+    streams = [main] + L.comp_streams
+    wss = [L.cws] + L.comp_ws
     Ks, Vs, Qs = inputs if inputs is not None else (L.K, L.V, L.Q)
+    for st in L.comp_streams:
+        st.wait_stream(main)
     for layer in range(wl.layers):
+        k = layer % len(streams)
         if before_layer is not None:
-            before_layer(layer)
+            before_layer(layer, streams[k])
         c = L.caches[layer]
         dbg = {"kept_idx": L.kept[layer]} if L.layer_average else None
         S.check(S.selkv_compress(L.shape, L.n_len, wl.rho, params, Ks[layer], Vs[layer], Qs[layer],
-                                 c.K_c, c.V_c, c.bias, c.lengths, dbg, L.cws.buf, L.cws.nbytes,
-                                 stream_ptr), "compress")
+                                 c.K_c, c.V_c, c.bias, c.lengths, dbg, wss[k].buf, wss[k].nbytes,
+                                 streams[k].cuda_stream), "compress")
+    for st in L.comp_streams:
+        main.wait_stream(st)
     if L.layer_average:
         S.check(S.selkv_layer_average_bias(L.shape, params, L.kept, [c.bias for c in L.caches],
                                            L.caches[0].lengths, L.aws.buf, L.aws.nbytes, stream_ptr),
@@ -290,7 +311,8 @@ def run_gpu(args):
         rope={"off": S.SELKV_ROPE_OFF, "half": S.SELKV_ROPE_HALF,
               "interleaved": S.SELKV_ROPE_INTERLEAVED}[args.rope], rope_theta=args.rope_theta,
         routing=S.SELKV_ROUTE_COSINE if args.routing == "cosine" else S.SELKV_ROUTE_BUCKET)
-    L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e, layer_average=args.layer_average)
+    L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e, layer_average=args.layer_average,
+                compress_streams=args.compress_streams)
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
     peaks, peak_src = load_peaks()
@@ -418,7 +440,7 @@ def run_gpu(args):
                    "head_dim": d, "obs_window": wl.obs_window, "select_mode": args.select_mode,
                    "rope": args.rope, "routing": args.routing,
                    "compensation": "averaged across layers" if args.layer_average else "per layer",
-                   "parallelism": "replicas",
+                   "parallelism": "replicas", "compress_streams": max(1, args.compress_streams),
                    "l2": "inputs larger than L2: every token streams all layers' compressed "
                          "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
                    "cuda_graph": True},
@@ -514,7 +536,7 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: 
         si = i % 2
         with torch.cuda.stream(stream):
             compress_layers(L, S, params, sp, inputs=sets[si],
-                            before_layer=lambda layer: stream.wait_event(arrived[si][layer]))
+                            before_layer=lambda layer, st: st.wait_event(arrived[si][layer]))
             consumed[si].record(stream)
         # the next step's inputs go to the other set once its last compression is done
         copy_inputs(1 - si, after=consumed[1 - si] if i > 0 else None)
@@ -602,6 +624,8 @@ def main():
     ap.add_argument("--routing", default="bucket", choices=["bucket", "cosine"],
                     help="routing of the evicted tokens: bucket (Eq. 3, the default) or the full "
                          "cosine routing of Sec. 3.4 (the oracle baseline is not sampled for it)")
+    ap.add_argument("--compress-streams", type=int, default=4,
+                    help="streams the layers' compressions are spread over (each with its own workspace)")
     ap.add_argument("--layer-average", action="store_true",
                     help="compensation averaged across layers instead of per layer (Sec. 3 overview)")
     args = ap.parse_args()
