@@ -158,10 +158,11 @@ def whole_job_rate(world: int, units_per_rank: float, seconds: float) -> float:
 # ------------------------------------------------------------------------------ GPU arm
 class HostArena:
     """Page-locked host memory for the end-to-end inputs: one allocation from the CUDA
-    runtime (cudaHostAlloc through torch), carved into the host copies of the inputs.  On the
-    GB300 machine it streams to the device at ~210 GB/s when copies run back to back; a region of
-    512 MiB transparent huge pages registered with cudaHostRegister measured no faster in the
-    end-to-end loop (and depends on the kernel finding the huge pages)."""
+    runtime (cudaHostAlloc through torch), carved into the host copies of the inputs.  On a
+    GB300 (Grace host, NVLink-C2C) it streams to the device at ~210 GB/s when copies run back
+    to back; a region of 512 MiB transparent huge pages registered with cudaHostRegister
+    measured no faster in the end-to-end loop (and depends on the kernel finding the huge
+    pages)."""
 
     def __init__(self, torch, nbytes: int):
         self.torch = torch
@@ -479,9 +480,9 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: 
     calls are issued eagerly.  Every timed step moves its full input bytes across the link
     inside the timed region (the copies for the first timed step run during the last warm-up
     step, those issued during the last timed step are waited for before the clock stops).
-    On the GB300 machine a 13 GB host-to-device pass copies at ~210 GB/s back to back with other
-    copies but at 25-70 GB/s after or during the decode's HBM streaming, which sets this
-    number (and makes it vary from run to run; more copy streams did not help).  Host
+    On a GB300 (Grace host) a 13 GB host-to-device pass copies at ~210 GB/s back to back with
+    other copies but at 25-70 GB/s after or during the decode's HBM streaming, which sets
+    this number (and makes it vary from run to run; more copy streams did not help).  Host
     buffers come from a HostArena."""
     wl = L.wl
     sp = stream.cuda_stream

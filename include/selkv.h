@@ -48,7 +48,7 @@ typedef struct CUstream_st* selkv_stream_t;
 typedef enum selkv_status {
   SELKV_OK = 0,
   SELKV_ERR_INVALID_ARG = 1, /* a pointer, size, shape or budget violates the contract */
-  SELKV_ERR_UNSUPPORTED = 2, /* a valid request this build does not implement          */
+  SELKV_ERR_UNSUPPORTED = 2, /* a valid request the library does not implement        */
   SELKV_ERR_WORKSPACE = 3,   /* workspace NULL, misaligned or smaller than required    */
   SELKV_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed                   */
   SELKV_ERR_DEVICE = 5       /* selkv_workspace_error found device error bits          */

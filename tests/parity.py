@@ -6,7 +6,7 @@ path: there either resolution is correct, the test checks that the GPU's choice 
 near-tied options, and the oracle then continues from the GPU's choice ("follow"), so the
 continuous outputs downstream are still compared element by element.
 
-Margins (derived from the arithmetic):
+Margins (derived from the arithmetic of the GPU path):
   DELTA      relative gap on scores / cumulative attention: the fp32 GPU values carry a
              relative error of a few 1e-6 (fp32 sums of exponentials whose arguments carry
              rounding error), so near-ties closer than 1e-4 relative may resolve either way.
