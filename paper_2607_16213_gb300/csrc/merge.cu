@@ -5,18 +5,20 @@
 //
 // Under Eq. 3 (argmax over the kept tokens of a bucket of the cumulative attention a) every
 // evicted token of a bucket routes to the same kept token tau_X, so the merge is a gather.
-// Four kernels, in stream order:
+// The kernels, in stream order:
 //   route  warp per (bucket X, sequence b): tau_X and a(tau_X) for every KV head (-1 / -inf
 //          for a bucket with no kept token);
-//   copy   every kept token's key and value row to its slot of K_c / V_c and ratio 1 for the
-//          slot; a thread per 16 bytes, coalesced.  Keys are unchanged, or, with RoPE
-//          repositioning (Eq. 7), turned by the shift from their position to their slot;
+//   copy   (only with RoPE repositioning or the cosine routing) every kept token's key and
+//          value row to its slot of K_c / V_c and ratio 1 for the slot; a thread per 16
+//          bytes, coalesced.  Keys are unchanged, or, with RoPE repositioning (Eq. 7),
+//          turned by the shift from their position to their slot;
 //   merge  one-warp CTA per (non-empty bucket X, KV head, sequence b): the evicted tokens of X and of
 //          the empty buckets that the nearest-ring rule gives to X, in ascending position
 //          order, 16 at a time: g_j = clamp(cos(v_j, v_tau), 0, 1) and
 //              v~_tau = (a_tau v_tau + sum g_j a_j v_j) / (a_tau + sum g_j a_j),
 //              R_tau  = (a_tau + sum g_j a_j) / a_tau,
-//          written over tau's slot;
+//          written over tau's slot; without the copy kernel the same warp then copies X's
+//          kept key rows and its other kept value rows to their slots (ratio 1);
 //   bias   bias = alpha * ln(mean over KV heads of R) for every slot (the same row for every
 //          KV head).
 // No floating-point atomics: every sum has a fixed order, so results are reproducible.
