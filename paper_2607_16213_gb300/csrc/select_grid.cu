@@ -10,8 +10,8 @@
 // digits in shared memory and add them to a per-unit global histogram; the last CTA of a unit
 // to arrive (one atomic add, no waiting) picks the digit and narrows the unit's prefix.  After
 // the last pass `count_eq` entries equal the threshold T; when more of them exist than are
-// still needed, a tie kernel finds the position of the last one taken.  A unit selects j iff
-// bits(key_j) > T or (bits(key_j) == T and j <= jcut).
+// still needed, the CTA that picked the last digit finds the position of the last one taken.
+// A unit selects j iff bits(key_j) > T or (bits(key_j) == T and j <= jcut).
 #include <climits>
 
 #include "selkv_internal.cuh"
