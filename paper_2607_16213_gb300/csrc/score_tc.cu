@@ -47,11 +47,6 @@ constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 colum
 __device__ __forceinline__ constexpr bool soft_exp(int i) { return (i & 15) < SELKV_SOFT_EXP; }
 __device__ __forceinline__ float ex2_mixed(float x, bool soft) { return soft ? ex2_poly(x) : ex2_approx(x); }
 
-// Pass 1 with the same pipelined loads measured slower (50.6 us against 49.1 us per
-// long-context layer: the running max then needs a correction every 16 keys), so it is off.
-#ifndef SELKV_P1_PIPE
-#define SELKV_P1_PIPE 0   // pass 1: pipelined 16-column TMEM loads on full, unmasked quarters
-#endif
 #ifndef SELKV_P2_PIPE
 #define SELKV_P2_PIPE 1   // pass 2: pipelined 16-column TMEM loads on full, unmasked tiles
 #endif
@@ -91,48 +86,6 @@ __device__ __forceinline__ float colsum64(uint32_t taddr, uint32_t rn, float sc)
   unpack_f2(a01, s0, s1);
   unpack_f2(a23, s2, s3);
   return (s0 + s1) + (s2 + s3);
-}
-
-// Pass 1, one thread's row over 64 keys of a tile (every key visible): the running max and
-// sum of 2^(v sc - max), updated every 16 keys; loads pipelined as in colsum64.
-__device__ __forceinline__ void rowstat_accum16(const float (&v)[16], float sc, int c0, float& m_run,
-                                                float& l_run) {
-  const float m01 = fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3]));
-  const float m23 = fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7]));
-  const float m45 = fmaxf(fmaxf(v[8], v[9]), fmaxf(v[10], v[11]));
-  const float m67 = fmaxf(fmaxf(v[12], v[13]), fmaxf(v[14], v[15]));
-  // the scale is positive, so max(v) * scale is the max of the scaled logits
-  const float mn = fmaxf(m_run, fmaxf(fmaxf(m01, m23), fmaxf(m45, m67)) * sc);
-  if (mn == -INFINITY) return;
-  const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
-  uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
-#pragma unroll
-  for (int i = 0; i < 16; i += 4) {
-    float x0, x1, x2, x3;
-    unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
-    unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
-    s01 = fadd2(s01, pack_f2(ex2_mixed(x0, soft_exp(c0 + i)), ex2_mixed(x1, soft_exp(c0 + i + 1))));
-    s23 = fadd2(s23, pack_f2(ex2_mixed(x2, soft_exp(c0 + i + 2)), ex2_mixed(x3, soft_exp(c0 + i + 3))));
-  }
-  float s0, s1, s2, s3;
-  unpack_f2(s01, s0, s1);
-  unpack_f2(s23, s2, s3);
-  l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
-  m_run = mn;
-}
-__device__ __forceinline__ void rowstat64(uint32_t taddr, float sc, float& m_run, float& l_run) {
-  float va[16], vb[16];
-  tmem_ld16_issue(taddr, va);
-  tmem_wait_ld16(va);
-#pragma unroll
-  for (int c = 0; c < 4; c += 2) {
-    tmem_ld16_issue(taddr + (c + 1) * 16, vb);
-    rowstat_accum16(va, sc, c * 16, m_run, l_run);
-    tmem_wait_ld16(vb);
-    if (c + 2 < 4) tmem_ld16_issue(taddr + (c + 2) * 16, va);
-    rowstat_accum16(vb, sc, (c + 1) * 16, m_run, l_run);
-    if (c + 2 < 4) tmem_wait_ld16(va);
-  }
 }
 
 template <int D, int PASS>
@@ -301,11 +254,9 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         tc_fence_after();
         const int key0 = (t_begin + t) * kKeys + part * 64;
         const bool full_quarter = key0 + 63 <= n - a.W;  // every row sees every key of the quarter
-        // warp-uniform: all 32 rows of this warp exist
-        const bool rows_full = h * 128 + q * 32 + 32 <= R;
-        if (ok && SELKV_P1_PIPE && SELKV_PACKED && full_quarter && rows_full) {
-          rowstat64(tmem + lane_base + buf * 256 + part * 64, sc, m_run, l_run);
-        } else if (ok) {
+        // (pass 1 keeps 32-column loads: 16-column pipelined loads, as in pass 2, measured
+        // slower here, the running max then needing a correction every 16 keys)
+        if (ok) {
 #pragma unroll 1
           for (int c = 0; c < 64; c += 32) {
             float v[32];
