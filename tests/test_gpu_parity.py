@@ -115,6 +115,42 @@ def test_compress_exact_ties_take_the_lowest_positions(per_head):
             assert kept[-1] < n - wl.obs_window
 
 
+def test_compress_on_concurrent_streams_matches_one_stream():
+    """Two layers compressed at once on two streams (a workspace each, as a caller compressing
+    a model's layers after prefill would) give bitwise the outputs of compressing them one
+    after the other on one stream."""
+    wl = SMALL["bf16_ragged"]
+    xs = [synth.gen_layer(wl, 20 + i) for i in range(2)]
+    n_len = [int(v) for v in xs[0]["n_len"]]
+    assert n_len == [int(v) for v in xs[1]["n_len"]]
+    m_cap = api.capacity(max(n_len), wl.rho)
+    shape = api.make_shape(wl.dtype, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                           wl.obs_window, wl.n, m_cap)
+    ins = [tuple(to_dev(x[k], wl.dtype) for k in ("K", "V", "Q_obs")) for x in xs]
+    torch.cuda.synchronize()  # the inputs exist before any other stream reads them
+
+    def run(streams):
+        outs = []
+        for i, st in enumerate(streams):
+            with torch.cuda.stream(st):
+                ws = api.Workspace(S.selkv_compress_workspace_size(shape), "cuda", st.cuda_stream)
+                outs.append((api.compress(shape, n_len, wl.rho, *ins[i], debug=True, workspace=ws,
+                                          stream=st.cuda_stream), ws))
+        torch.cuda.synchronize()
+        return outs
+
+    side = [torch.cuda.Stream(), torch.cuda.Stream()]
+    one = torch.cuda.Stream()
+    par = run(side)
+    seq = run([one, one])
+    for (a, wa), (b, wb) in zip(par, seq):
+        assert wa.errors() == 0 and wb.errors() == 0
+        for name in ("K_c", "V_c", "bias", "lengths"):
+            assert torch.equal(getattr(a, name), getattr(b, name)), name
+        for name in ("kept_idx", "target", "gate", "ratio"):
+            assert torch.equal(a.debug[name], b.debug[name]), name
+
+
 def test_window_equals_sequence():
     wl = SMALL["tiny"].with_(n=96, obs_window=96, rho=0.5)
     x = synth.gen_layer(wl, 0)
