@@ -1,7 +1,6 @@
 """The C-ABI library on the host: it loads, exports every function include/selkv.h declares,
 sizes workspaces, and rejects invalid arguments with a status code before any CUDA call (so
 these run without a GPU; no call here reaches a kernel launch)."""
-import ctypes
 import os
 import subprocess
 
