@@ -151,16 +151,21 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 #ifndef SELKV_DEC_CTAS_PER_SM
 #define SELKV_DEC_CTAS_PER_SM 1  // decode CTAs planned per SM when splitting the rows
 #endif
+#ifndef SELKV_DEC_FILL_ROWS
+#define SELKV_DEC_FILL_ROWS 512  // a CTA's fixed cost in the split model, in rows streamed
+#endif
 #ifndef SELKV_DEC_MAX_SPLITS
 #define SELKV_DEC_MAX_SPLITS 64  // most splits of one (sequence, KV head)
 #endif
 
 // Split count of each (sequence, KV head).  The B * Hkv * S CTAs run in waves of
 // CTAS_PER_SM * num_sms; a wave lasts about as long as streaming one CTA's rows plus a fixed
-// fill-and-fold cost worth kFillRows rows (about 2 us at one SM's share of HBM bandwidth).
-// S minimises waves * (rows per CTA + kFillRows) over the capacity m_cap, fewest splits on ties.
+// fill-and-fold cost worth kFillRows rows (about 5 us at one SM's share of HBM bandwidth, the
+// fixed cost measured per launch).  S minimises waves * (rows per CTA + kFillRows) over the
+// capacity m_cap, fewest splits on ties.  (Batch 4 x 8k compressed rows: 512 picks 4 splits,
+// 29.0 us per launch; 192 picked 9 splits in two waves, 31.2 us.  Batch 1 x 25k: 19 either way.)
 int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
-  constexpr long kFillRows = 192;
+  constexpr long kFillRows = SELKV_DEC_FILL_ROWS;
   const long units = (long)B * Hkv;
   const long slots = std::max(1L, (long)SELKV_DEC_CTAS_PER_SM * num_sms);
   const int smax = std::max(1, std::min(SELKV_DEC_MAX_SPLITS, (m_cap + 63) / 64));
