@@ -21,7 +21,9 @@
  *     bits in the workspace's error word (SELKV_DEVERR_*); the kernels never trap.  Read and
  *     clear them with selkv_workspace_error.
  *   - A workspace must be zeroed once before its first use (selkv_workspace_init).  Calls
- *     that share a workspace must not overlap on the GPU.
+ *     that share a workspace must not overlap on the GPU; calls with workspaces of their own
+ *     may run concurrently on different streams (for instance the compressions of a model's
+ *     layers after prefill).
  *   - Element types: dtype SELKV_BF16 (storage bf16, fp32 arithmetic) or SELKV_FP32.
  *   - Shapes: B sequences, Hq query heads, Hkv KV heads (Hkv divides Hq, G = Hq / Hkv; query
  *     head h reads KV head h / G), head dimension d in {64, 128}, observation window W.
