@@ -150,6 +150,20 @@ def max_over_ranks(x: float, torch, dist, device) -> float:
     return float(t.item())
 
 
+def decode_bytes_per_launch(wl, n_len, T: int) -> float:
+    """Algorithmic bytes of one decode launch (one layer, one token), averaged over T tokens:
+    each cached row of each KV head reads its K_c and V_c rows (d elements each) and one fp32
+    bias, the row appended at step t included (a sequence holds m_b + t + 1 rows at step t);
+    plus the queries and outputs of every query head and the appended key and value rows."""
+    esz = 2 if wl.dtype == "bf16" else 4
+    d, Hkv, Hq = wl.head_dim, wl.num_kv_heads, wl.num_q_heads
+    m_b = [int(math.floor(wl.rho * n)) for n in n_len]
+    per_row = Hkv * (2 * d * esz + 4)
+    rows_total = sum(sum(m + t + 1 for t in range(T)) for m in m_b)   # over the T steps
+    fixed = T * len(n_len) * (2 * Hq * d * esz + 2 * Hkv * d * esz)
+    return (rows_total * per_row + fixed) / T
+
+
 def whole_job_rate(world: int, units_per_rank: float, seconds: float) -> float:
     """Units processed by all ranks per second (weak scaling: every rank does the same work)."""
     return world * units_per_rank / seconds
@@ -384,15 +398,8 @@ def run_gpu(args):
     comp_ms_avg = sum(comp_ms) / len(comp_ms)
     decode_tok_s = tokens_per_step / (dec_ms_avg / 1e3)
 
-    # algorithmic bytes of the decode kernel per launch: each cached row of each KV head
-    # reads K_c and V_c (d elements each) and one fp32 bias; plus q, out, k_new, v_new.
-    esz = 2 if wl.dtype == "bf16" else 4
     d, Hkv, Hq, B = wl.head_dim, wl.num_kv_heads, wl.num_q_heads, wl.batch
-    m_b = [int(math.floor(wl.rho * n)) for n in L.n_len]
-    per_row = Hkv * (2 * d * esz + 4)
-    rows_total = sum(sum(m + t + 1 for t in range(L.T)) for m in m_b)   # over the T steps
-    fixed = L.T * B * (2 * Hq * d * esz + 2 * Hkv * d * esz)
-    dec_bytes_per_layer_step = (rows_total * per_row + fixed) / L.T
+    dec_bytes_per_layer_step = decode_bytes_per_launch(wl, L.n_len, L.T)
     dec_launch_us = dec_ms_avg * 1e3 / n_dec_launch
     achieved_gbs = dec_bytes_per_layer_step / (dec_launch_us * 1e-6) / 1e9
     peak_hbm = float(peaks["hbm_gbs"])

@@ -1,7 +1,8 @@
-"""The multi-rank host logic of bench.py on CPU: two gloo ranks (one process each, launched
-as torchrun would, rendezvous on 127.0.0.1).  Every rank replays its own replica of the
-workload (weak scaling, no collective on the data path); the job's time is the slowest
-rank's, and the rate counts every rank's tokens."""
+"""Host logic of bench.py on the CPU.  Ranks: two gloo ranks (one process each, launched as
+torchrun would, rendezvous on 127.0.0.1); every rank replays its own replica of the workload
+(weak scaling, no collective on the data path), the job's time is the slowest rank's, and the
+rate counts every rank's tokens.  Roofline: the decode kernel's algorithmic bytes per launch,
+checked against a count by hand."""
 import os
 import socket
 import subprocess
@@ -62,3 +63,15 @@ def test_reference_arm_prints_on_rank_0_only():
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     assert r.stdout.strip() == ""
+
+
+def test_decode_bytes_per_launch_by_hand():
+    """One launch of the 100k workload at token t: 8 KV heads x (25,000 + t + 1) rows of
+    K_c, V_c (256 bytes each, bf16 d = 128) and a 4-byte bias, plus q and out (32 heads x 256
+    bytes each) and the appended k and v (8 heads x 256 bytes each)."""
+    import synth
+    wl = synth.WORKLOADS["long_100k"]
+    T = 256
+    per_token = [8 * (25000 + t + 1) * 516 + 2 * 32 * 256 + 2 * 8 * 256 for t in range(T)]
+    assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(sum(per_token) / T)
+    assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(103750928.0)
