@@ -103,6 +103,7 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, p
     layers of sequence 0 and `decode_tokens` decode tokens over those layers; the rates are
     scaled to the whole step (all layers, all sequences, all decode steps)."""
     from oracle import selkv_oracle as O
+    cpu0 = os.times()
     t_comp = 0.0
     t_dec = 0.0
     ncomp = 0
@@ -129,6 +130,10 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, p
             ndec += 1
     per_layer_comp = t_comp / ncomp
     per_layer_tok = t_dec / ndec
+    cpu1 = os.times()
+    # the cores kept busy on average (process CPU time / wall time, data generation included):
+    # numpy's BLAS pool spreads the oracle's products over the host's cores
+    busy = ((cpu1.user - cpu0.user) + (cpu1.system - cpu0.system)) / max(1e-9, cpu1.elapsed - cpu0.elapsed)
     step_s = wl.batch * wl.layers * (per_layer_comp + wl.decode_steps * per_layer_tok)
     tokens = wl.batch * wl.decode_steps
     sample = ("fp64 oracle: compression of %d layer(s) x 1 sequence (n=%d) and %d decode token(s) "
@@ -136,7 +141,8 @@ def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, p
               % (layers, wl.n, decode_tokens, wl.layers, wl.batch, wl.decode_steps))
     return dict(value=tokens / step_s, unit="tokens/s", cores=os.cpu_count(), kind="oracle",
                 sample=sample, compress_s_per_layer=per_layer_comp,
-                decode_s_per_layer_token=per_layer_tok, sample_wall_s=t_comp + t_dec)
+                decode_s_per_layer_token=per_layer_tok, sample_wall_s=t_comp + t_dec,
+                cores_busy_avg=round(busy, 2))
 
 
 # ------------------------------------------------------------------------------ ranks
@@ -607,7 +613,7 @@ def run_reference(args):
             "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
                        "rho": wl.rho, "decode_steps": wl.decode_steps, "select_mode": args.select_mode},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
-                             "sample": info["sample"]},
+                             "sample": info["sample"], "cores_busy_avg": info["cores_busy_avg"]},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
