@@ -441,7 +441,7 @@ def run_gpu(args):
     # end to end through the public API from pinned host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(L, S, api, torch, params, stream, dev, min(args.steps, 3), args.warmup)
+        e2e = run_e2e(L, S, api, torch, params, stream, dev, args.e2e_steps, args.warmup)
         e2e["ms_per_step"] = max_over_ranks(e2e["ms_per_step"], torch, dist, dev)
         e2e["value"] = whole_job_rate(world, wl.batch * L.T, e2e["ms_per_step"] / 1e3)
 
@@ -573,6 +573,212 @@ def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: 
             "pipelined": "the next step's input copies overlap this step's decode"}
 
 
+# ------------------------------------------------------------------------------ serving sweep
+SWEEP_METRIC = "serving sweep point: compensated decode HBM GB/s per launch; compress ms/layer"
+L2_BYTES = 126 * 2 ** 20
+
+
+def parse_sweep(name: str):
+    """'sweep:B,n,rho' -> (B, n, rho)."""
+    b, n, r = name.split(":", 1)[1].split(",")
+    return int(b), int(n), float(r)
+
+
+def compress_bytes(wl, n_len) -> float:
+    """Algorithmic bytes of one layer's compression: every sequence reads its K and V rows and
+    its window queries once and writes its kept K_c and V_c rows and one fp32 bias per kept
+    position."""
+    esz = 2 if wl.dtype == "bf16" else 4
+    d, Hkv, Hq, W = wl.head_dim, wl.num_kv_heads, wl.num_q_heads, wl.obs_window
+    tot = 0
+    for n in n_len:
+        m = int(math.floor(wl.rho * n))
+        tot += 2 * Hkv * n * d * esz + Hq * W * d * esz + 2 * Hkv * m * d * esz + m * 4
+    return float(tot)
+
+
+def oracle_sweep_sample(wl, n_len, T: int) -> dict:
+    """The fp64 oracle on a bounded sample of one sweep point: compression of sequence 0 and
+    one decode token over its compressed cache, scaled to the layer (every sequence, by its
+    length) and to T decode tokens."""
+    from oracle import selkv_oracle as O
+    x = synth.gen_sequence(wl, 0, 0, threads=os.cpu_count() or 1)
+    n0 = x["n"]
+    K, V, Q = (x[k].astype(np.float64) for k in ("K", "V", "Q_obs"))
+    t0 = time.perf_counter()
+    r = O.compress(K, V, Q, n0, wl.rho)
+    t_comp = time.perf_counter() - t0
+    dec = synth.gen_decode(wl.with_(batch=1), 0, 1)
+    t0 = time.perf_counter()
+    O.decode(dec["q"][0, 0], r.K_c, r.V_c, r.bias, r.m)
+    t_dec = time.perf_counter() - t0
+    m0 = r.m
+    comp_layer = t_comp * sum(n_len) / n0
+    dec_layer = t_dec * sum(int(math.floor(wl.rho * n)) for n in n_len) / m0
+    return {"value": comp_layer * 1e3, "unit": "ms/layer (compression)", "cores": os.cpu_count(),
+            "kind": "oracle", "decode_ms_per_layer_token": dec_layer * 1e3,
+            "sample": "fp64 oracle: compression of sequence 0 (n=%d) and one decode token over its "
+                      "cache, scaled by length to the %d sequences of the layer" % (n0, len(n_len))}
+
+
+def sweep_point(args, point, torch, S, api, dev, peaks, peak_src) -> dict:
+    """One point of the batched serving sweep (ragged lengths, one layer): compression of the
+    layer timed from a cold L2 (an L2-sized buffer is written before each timed replay), then
+    decode over the compressed cache, T tokens each appending a row.  Decode runs over enough
+    copies of the compressed layer (up to 32, as a 32-layer model would hold) that one token's
+    caches exceed three times L2; if even 32 copies do not, the L2 is flushed before every
+    token and the flush's own time (measured alone) is subtracted."""
+    B, n, rho = point
+    wl = synth.sweep(B, n, rho)
+    T = wl.decode_steps
+    Hq, Hkv, d, W = wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.obs_window
+    n_len = [int(v) for v in synth.seq_lengths(wl)]
+    m_cap = api.capacity(max(n_len), rho, extra=T + 1)
+    shape = api.make_shape(wl.dtype, B, Hq, Hkv, d, W, n, m_cap)
+    bf = torch.bfloat16
+    K = torch.zeros((B, Hkv, n, d), dtype=bf, device=dev)
+    V = torch.zeros((B, Hkv, n, d), dtype=bf, device=dev)
+    Q = torch.empty((B, Hq, W, d), dtype=bf, device=dev)
+    for b in range(B):
+        x = synth.gen_sequence(wl, 0, b, threads=os.cpu_count() or 1)
+        nb = x["n"]
+        K[b, :, :nb].copy_(torch.from_numpy(x["K"]).to(bf))
+        V[b, :, :nb].copy_(torch.from_numpy(x["V"]).to(bf))
+        Q[b].copy_(torch.from_numpy(x["Q_obs"]).to(bf))
+        del x
+    params = S.selkv_params.defaults()
+    stream = torch.cuda.Stream(device=dev)
+    sp = stream.cuda_stream
+    cache = api.alloc_compressed(shape, dev)
+    ws = api.Workspace(S.selkv_compress_workspace_size(shape), dev)
+
+    def compress():
+        S.check(S.selkv_compress(shape, n_len, rho, params, K, V, Q, cache.K_c, cache.V_c, cache.bias,
+                                 cache.lengths, None, ws.buf, ws.nbytes, sp), "compress")
+
+    with torch.cuda.stream(stream):
+        compress()
+    torch.cuda.synchronize()
+    assert ws.errors(sp) == 0
+    g_comp = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_comp, stream=stream):
+        compress()
+    lengths0 = cache.lengths.clone()
+
+    dec_bytes = decode_bytes_per_launch(wl, n_len, T)
+    copies = max(1, min(32, int(math.ceil(3 * L2_BYTES / dec_bytes))))
+    flush_tokens = copies * dec_bytes < 2 * L2_BYTES
+    caches = [cache] + [api.CompressedCache(shape=shape, K_c=cache.K_c.clone(), V_c=cache.V_c.clone(),
+                                            bias=cache.bias.clone(), lengths=cache.lengths.clone())
+                        for _ in range(copies - 1)]
+    dd = synth.gen_decode(wl, 0, T)
+    dq, dk, dv = (torch.from_numpy(dd[k]).to(dev).to(bf) for k in ("q", "k_new", "v_new"))
+    out = torch.empty((T, B, Hq, d), dtype=bf, device=dev)
+    dws = api.Workspace(S.selkv_decode_workspace_size(shape), dev)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    g_dec, g_flush = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_dec, stream=stream):
+        for t in range(T):
+            if flush_tokens:
+                flush.zero_()
+            for c in caches:
+                S.check(S.selkv_decode_attn(shape, dq[t], c.K_c, c.V_c, c.bias, c.lengths, dk[t], dv[t], out[t],
+                                            dws.buf, dws.nbytes, sp), "decode")
+    with torch.cuda.graph(g_flush, stream=stream):
+        for t in range(T):
+            flush.zero_()
+
+    def reset_lengths():
+        for c in caches:
+            c.lengths.copy_(lengths0)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            flush.zero_()
+            g_comp.replay()
+            reset_lengths()
+            g_dec.replay()
+            g_flush.replay()
+    torch.cuda.synchronize()
+    steps = max(args.steps, 10)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
+    clocks = ClockSampler(torch.cuda.current_device() if not os.environ.get("CUDA_VISIBLE_DEVICES") else 0)
+    clocks.start()
+    time.sleep(0.3)
+    with torch.cuda.stream(stream):
+        for k in range(steps):
+            flush.zero_()
+            ev[k][0].record(stream)
+            g_comp.replay()
+            ev[k][1].record(stream)
+            reset_lengths()
+            ev[k][2].record(stream)
+            g_dec.replay()
+            ev[k][3].record(stream)
+            if flush_tokens:
+                ev[k][4].record(stream)
+                g_flush.replay()
+                ev[k][5].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    want = [int(math.floor(rho * v)) + T for v in n_len]
+    for c in caches:
+        assert c.lengths.cpu().tolist() == want, "lengths after the timed decode"
+    assert ws.errors(sp) == 0 and dws.errors(sp) == 0, "device error flags"
+    comp_ms = statistics.median(ev[k][0].elapsed_time(ev[k][1]) for k in range(steps))
+    dec_ms = statistics.median(ev[k][2].elapsed_time(ev[k][3]) for k in range(steps))
+    flush_ms = statistics.median(ev[k][4].elapsed_time(ev[k][5]) for k in range(steps)) if flush_tokens else 0.0
+    launch_us = (dec_ms - flush_ms) * 1e3 / (T * copies)
+    dec_gbs = dec_bytes / (launch_us * 1e-6) / 1e9
+    c_bytes = compress_bytes(wl, n_len)
+    comp_gbs = c_bytes / (comp_ms * 1e-3) / 1e9
+    peak_hbm = float(peaks["hbm_gbs"])
+    line = {
+        "metric": SWEEP_METRIC, "value": dec_gbs, "unit": "GB/s", "n_gpus": 1, "steps": steps,
+        "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "batch": B, "n": n, "rho": rho, "n_len_min": min(n_len),
+                   "n_len_max": max(n_len), "layers_timed": 1, "layers_reported": 32,
+                   "decode_steps": T, "q_heads": Hq, "kv_heads": Hkv, "head_dim": d, "obs_window": W,
+                   "decode_layer_copies": copies,
+                   "l2": ("compression: L2 flushed before each timed replay; decode: %s"
+                          % ("L2 flushed before each token, the flush time subtracted" if flush_tokens
+                             else "one token streams %.0f MB of caches (> 3x L2)" % (copies * dec_bytes / 1e6))),
+                   "cuda_graph": True},
+        "compress_ms_per_layer": comp_ms,
+        "compress_ms_x32": 32 * comp_ms,
+        "compress_gbs": comp_gbs,
+        "decode_launch_us": launch_us,
+        "decode_tok_s_x32": B / (32 * launch_us * 1e-6),
+        "roofline": {"kernel": "selkv decode (split-K, GQA, bias in softmax)", "bound": "hbm",
+                     "achieved": dec_gbs, "peak": peak_hbm, "unit": "GB/s", "frac": dec_gbs / peak_hbm,
+                     "peak_source": peak_src, "bytes_per_launch": dec_bytes, "launch_us": launch_us,
+                     "traffic": None},
+        "roofline_compress": {"bound": "hbm", "achieved": comp_gbs, "peak": peak_hbm, "unit": "GB/s",
+                              "frac": comp_gbs / peak_hbm, "bytes_per_layer": c_bytes},
+        "clocks": clk,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_sweep_sample(wl, n_len, T)
+    del K, V, Q, caches, cache, ws, dws, flush, g_comp, g_dec, g_flush
+    torch.cuda.empty_cache()
+    return line
+
+
+def run_sweep(args, points):
+    import torch
+    import paper_2607_16213_gb300 as S
+    from paper_2607_16213_gb300 import api, build as _build
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    _build.build()
+    S.library()
+    peaks, peak_src = load_peaks()
+    for pt in points:
+        print(json.dumps(sweep_point(args, pt, torch, S, api, dev, peaks, peak_src)), flush=True)
+
+
 DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "decode_simt.cu", "ptx.cuh", "selkv_internal.cuh",
                   "tma_host.cu")
 
@@ -624,10 +830,15 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="selkv", choices=["selkv", "reference"])
-    ap.add_argument("--workload", default="long_100k", choices=list(synth.WORKLOADS))
+    ap.add_argument("--workload", default="long_100k",
+                    help="one of %s, or sweep:B,n,rho (a point of the batched serving sweep)"
+                         % ", ".join(synth.WORKLOADS))
+    ap.add_argument("--sweep", default=None,
+                    help="serving-sweep points, 'all' or 'B,n,rho;B,n,rho;...': one JSON line each")
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--layers", type=int, default=None, help=argparse.SUPPRESS)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10, help="timed steps of the end-to-end measurement")
     ap.add_argument("--no-full", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--select-mode", default="shared", choices=["shared", "per_head"],
@@ -645,8 +856,14 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.sweep is not None:
+        pts = synth.SWEEP_POINTS if args.sweep == "all" else [
+            (int(b), int(n), float(r)) for b, n, r in (p.split(",") for p in args.sweep.split(";"))]
+        run_sweep(args, pts)
+    elif args.impl == "reference":
         run_reference(args)
+    elif args.workload.startswith("sweep:"):
+        run_sweep(args, [parse_sweep(args.workload)])
     else:
         run_gpu(args)
 

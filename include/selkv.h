@@ -166,7 +166,7 @@ SELKV_API selkv_status selkv_workspace_init(void* workspace, size_t workspace_by
 SELKV_API selkv_status selkv_workspace_error(void* workspace, selkv_stream_t stream, uint32_t* flags);
 
 /* ---------------------------------------------------------------------------------------
- * Compression (Algorithm 1, steps 1-6; step 7, RoPE repositioning, off as in Sec. 4.1).
+ * Compression (Algorithm 1; Sec. 3.1-3.6; RoPE repositioning, Eq. 7, off as in Sec. 4.1).
  *
  * For every sequence b (prefill length n_b = n_len[b]) and every KV head:
  *   a  = mean over the G query heads of the column sums of the causal observation-window
@@ -279,7 +279,9 @@ SELKV_API selkv_status selkv_decode_attn(const selkv_shape* shape, const void* q
  *     part that must start at zero before its kernel.  Calls that overlap on the GPU (on
  *     different streams or from different host threads) race on the array: serialise them.
  *   - The first call on a device looks up the array's device address with that device
- *     current; make that first call before any stream capture.
+ *     current, and a call made in another context than the one of the address it holds
+ *     (after cudaDeviceReset, for instance) looks it up again; make the first call on a
+ *     device, and the first call after a reset, before any stream capture.
  *   - flags_out: optional device uint32 that receives the SELKV_DEVERR_* bits (OR-ed in,
  *     never cleared); NULL drops them.
  * ------------------------------------------------------------------------------------- */

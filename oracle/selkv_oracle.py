@@ -430,8 +430,8 @@ class CompressResult:
 def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
              params: Params = Params(), follow_per_kv=None, follow_kept=None,
              follow_target=None) -> CompressResult:
-    """Algorithm 1 for one sequence of one layer (step 7, RoPE repositioning, only when
-    params.rope is set).  K, V: [Hkv][>=n][d]; Q: [Hq][W][d]; all float64.
+    """Compression of one sequence of one layer (Sec. 3.1-3.7; RoPE repositioning, Eq. 7,
+    only when params.rope is set).  K, V: [Hkv][>=n][d]; Q: [Hq][W][d]; all float64.
 
     follow_* replace a discrete choice of the oracle by a given one (per-KV-head top-k
     masks, final kept mask, merge targets), so that a test can compare the continuous
@@ -444,13 +444,13 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     if m_s < 0 or Q.shape[1] > n:
         raise ValueError("budget below the recent window, or window longer than the sequence")
     n_cand = n - params.recent
-    a = cumulative_attention(Q, K, n)                         # step 1 (re-pass)
+    a = cumulative_attention(Q, K, n)                         # Sec. 3.1 re-pass, Eq. 1 attention sum
     vn = value_norms(V, n)
     c = a * vn                                                # Eq. 1
     cp = pool_scores(c, n_cand, params.pool_kernel)           # smoothing
     if params.select_mode == SELECT_PER_HEAD:
         return _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target)
-    sel = select_shared(cp, n, m_s, params.recent, follow_per_kv, follow_kept)  # step 2
+    sel = select_shared(cp, n, m_s, params.recent, follow_per_kv, follow_kept)  # Eq. 2, Sec. 3.3 union and trim
     kept_idx = np.flatnonzero(sel.kept)
     target = np.full((Hkv, n), -1, dtype=np.int64)
     g = np.zeros((Hkv, n))
@@ -460,17 +460,17 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
     R = np.ones((Hkv, kept_idx.size))
     for kv in range(Hkv):
         t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
-             else _route(a[kv], V[kv], sel.kept, params))                      # step 3
+             else _route(a[kv], V[kv], sel.kept, params))                      # Eq. 3 (Sec. 3.4)
         target[kv] = t
-        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
-        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # steps 5, 6
+        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # Eq. 4
+        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx, t, g[kv])            # Eq. 5, Eq. 6
     if params.bias_mode == BIAS_COUNT:
         bias = count_bias(np.stack([merge_counts(kept_idx, target[kv], g[kv]) for kv in range(Hkv)]),
                           params.alpha, per_head=False)
     else:
         bias = gqa_bias(R, params.alpha)
     Kc = K[:, kept_idx].copy()
-    if params.rope != ROPE_OFF:                                         # step 7 (Eq. 7)
+    if params.rope != ROPE_OFF:                                         # Eq. 7 (Sec. 3.7)
         Kc = np.stack([reposition(Kc[kv], kept_idx, params.rope_theta, params.rope) for kv in range(Hkv)])
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=sel,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,
@@ -478,17 +478,17 @@ def compress(K: np.ndarray, V: np.ndarray, Q: np.ndarray, n: int, rho: float,
 
 
 def _route(a_kv, V_kv, kept, params):
-    """Step 3 of Algorithm 1 under the routing of params (Eq. 3 buckets, or R20 cosine)."""
+    """Merge targets under the routing of params (Eq. 3 buckets, or R20 cosine; Sec. 3.4)."""
     if params.routing == ROUTE_COSINE:
         return route_cosine(V_kv, kept)
     return route(a_kv, kept, params.bucket, params.empty_bucket)
 
 
 def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, follow_target):
-    """Algorithm 1 steps 2-6 with per-head selection (R17): every KV head has its own kept
-    set, targets, merged values and bias row."""
+    """Eq. 2-6 with per-head selection (R17; Sec. 3.3, Sec. 3.6): every KV head has its own
+    kept set, targets, merged values and bias row."""
     Hkv, _, d = K.shape
-    kept = select_per_head(cp, n, m_s, params.recent, follow_per_kv)      # step 2, per head
+    kept = select_per_head(cp, n, m_s, params.recent, follow_per_kv)      # Eq. 2 per head (Sec. 3.3)
     kept_idx = np.stack([np.flatnonzero(kept[kv]) for kv in range(Hkv)])  # [Hkv][m]
     target = np.full((Hkv, n), -1, dtype=np.int64)
     g = np.zeros((Hkv, n))
@@ -499,12 +499,12 @@ def _compress_per_head(K, V, n, m, m_s, a, vn, c, cp, params, follow_per_kv, fol
     R = np.ones((Hkv, m))
     for kv in range(Hkv):
         t = (np.asarray(follow_target[kv][:n], dtype=np.int64) if follow_target is not None
-             else _route(a[kv], V[kv], kept[kv], params))                      # step 3
+             else _route(a[kv], V[kv], kept[kv], params))                      # Eq. 3 (Sec. 3.4)
         target[kv] = t
-        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # step 4
-        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx[kv], t, g[kv])        # steps 5, 6
+        g[kv], sim[kv], decision[kv] = gate(V[kv, :n], t, params.gate_mode)     # Eq. 4
+        Vc[kv], R[kv] = merge(a[kv], V[kv, :n], kept_idx[kv], t, g[kv])        # Eq. 5, Eq. 6
         Kc[kv] = K[kv, kept_idx[kv]]
-        if params.rope != ROPE_OFF:                                     # step 7 (Eq. 7)
+        if params.rope != ROPE_OFF:                                     # Eq. 7 (Sec. 3.7)
             Kc[kv] = reposition(Kc[kv], kept_idx[kv], params.rope_theta, params.rope)
     return CompressResult(m=m, m_s=m_s, a=a, vnorm=vn, c=c, c_pooled=cp, sel=None,
                           kept_idx=kept_idx, target=target, g=g, sim=sim, decision=decision,

@@ -137,13 +137,16 @@ __device__ __forceinline__ void write_append_row(const DecodeArgs& a, size_t bk,
 // overlaps the combine; thread `owner` does both halves.  begin: reset the (b, kv) counter
 // and count this head on the sequence's counter; every CTA of the sequence has read
 // lengths[b] before its own arrival, so the last head to count may advance it.  end: that
-// head writes lengths[b] = L + 1 (the acquire on the counter keeps the write after the count).
+// head writes lengths[b] = L + 1.  The count is acquire-release: it acquires the heads that
+// counted before it and releases this head's own split CTAs' reads of lengths[b] (acquired
+// through their arrivals) to the head that writes it.  A CTA that leaves early (a timed-out
+// wait) still runs end, so the sequence's counter is reset for the next launch.
 __device__ __forceinline__ uint32_t finish_lengths_begin(const DecodeArgs& a, int b, size_t bk, bool app,
                                                          int owner = 0) {
   uint32_t old = 0u;
   if ((int)threadIdx.x == owner) {
     a.cnt_head[bk] = 0u;
-    if (app) old = atom_add_acquire_gpu(&a.cnt_seq[b], 1u);
+    if (app) old = atom_add_acq_rel_gpu(&a.cnt_seq[b], 1u);
   }
   return old;
 }

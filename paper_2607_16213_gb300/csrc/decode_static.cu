@@ -14,10 +14,14 @@
 //   * Every call reuses it and it keeps the previous call's contents; the counters that must
 //     start at zero are cleared by each call before its kernel runs.
 //   * Calls that overlap on the GPU (other streams, other host threads) race on it.
-//   * Its device address is looked up once per device, on the first call made with that
-//     device current; make that first call before any stream capture begins.
+//   * Its device address is looked up on the first call made with a device current, and
+//     again whenever that device's current context has changed since (after cudaDeviceReset
+//     the module is loaded anew, at a new address); make the first call on a device, and the
+//     first call after a reset, before any stream capture begins.
 #include <cmath>
 #include <mutex>
+
+#include <cudaTypedefs.h>
 
 #include "selkv_internal.cuh"
 
@@ -31,22 +35,44 @@ static __device__ __align__(256) unsigned char g_decode_scratch[SELKV_STATIC_SCR
 
 constexpr int kMaxDevices = 64;
 
-
 std::mutex g_mu;
 void* g_scratch_ptr[kMaxDevices] = {};
+CUcontext g_scratch_ctx[kMaxDevices] = {};
 
-// Device address of g_decode_scratch on the current device (looked up once per device).
+// cuCtxGetCurrent through the runtime's driver entry point (the library does not link libcuda).
+PFN_cuCtxGetCurrent_v4000 ctx_fn() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+  });
+  return fn;
+}
+
+// Device address of g_decode_scratch on the current device: looked up on the device's first
+// call and again when the thread's current context is not the one the address was taken in.
+// (If the context cannot be queried, the first address is kept.)
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  auto get_ctx = ctx_fn();
+  CUcontext ctx = nullptr;
+  if (get_ctx != nullptr && get_ctx(&ctx) != CUDA_SUCCESS) ctx = nullptr;
   std::lock_guard<std::mutex> lock(g_mu);
-  if (g_scratch_ptr[dev] == nullptr) {
+  const bool known = g_scratch_ptr[dev] != nullptr && (get_ctx == nullptr || (ctx != nullptr && ctx == g_scratch_ctx[dev]));
+  if (!known) {
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_decode_scratch);
+    e = cudaGetSymbolAddress(&p, g_decode_scratch);  // also makes the device's context current
     if (e != cudaSuccess) return e;
+    if (get_ctx != nullptr && get_ctx(&ctx) != CUDA_SUCCESS) ctx = nullptr;
     g_scratch_ptr[dev] = p;
+    g_scratch_ctx[dev] = ctx;
   }
   *out = g_scratch_ptr[dev];
   return cudaSuccess;

@@ -162,6 +162,7 @@ __device__ __forceinline__ void combine_record(const DecodeArgs& a, int b, int k
   if (!mbar_wait(bar, 0)) {
     if (tid == 0) raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
     mbar_wait(bar, 0);  // the copy must land before the CTA leaves
+    finish_lengths_end(a, b, L, app, seq_old, owner);  // the sequence counter must not stay raised
     return;
   }
   for (int g = warp; g < G; g += nwarps) {

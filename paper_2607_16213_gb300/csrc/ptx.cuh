@@ -101,11 +101,6 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* p, uint32_t v
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
 }
-__device__ __forceinline__ uint32_t atom_add_acquire_gpu(uint32_t* p, uint32_t v) {
-  uint32_t old;
-  asm volatile("atom.acquire.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
-}
 
 __device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
@@ -130,26 +125,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
-}
-
-// 2^x for x <= 0 on the FMA and integer pipes, leaving the special-function unit to other
-// work: x = n + f with n = round(x) (adding 1.5 * 2^23 rounds to an integer in the low
-// mantissa bits) and f in [-1/2, 1/2]; 2^f is a degree-5 polynomial (minimax in relative
-// error on [-1/2, 1/2], fitted by Remez exchange; 2.3e-7 relative in this fp32 Horner form,
-// about the error of ex2.approx) and n is added to its exponent field.  Inputs below -127
-// are clamped (the result is then below 2^-126).
-__device__ __forceinline__ float ex2_poly(float x) {
-  x = fmaxf(x, -127.f);
-  const float t = x + 12582912.f;
-  const float f = x - (t - 12582912.f);
-  float p = 1.3276472e-3f;
-  p = fmaf(p, f, 9.6755410e-3f);
-  p = fmaf(p, f, 5.5507131e-2f);
-  p = fmaf(p, f, 2.4022120e-1f);
-  p = fmaf(p, f, 6.9314694e-1f);
-  p = fmaf(p, f, 1.0000001f);
-  const int n = __float_as_int(t) - __float_as_int(12582912.f);
-  return __int_as_float(__float_as_int(p) + (n << 23));
 }
 
 // Packed pairs of fp32 (sm_100 and later): one instruction for two lanes' worth of work.

@@ -34,18 +34,9 @@ constexpr int kEpiWarps = 16;
 constexpr int kProducerWarp = 16, kMmaWarp = 17;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 columns
-#ifndef SELKV_SOFT_EXP
-#define SELKV_SOFT_EXP 0  // of every 16 exponentials, how many run as ex2_poly
-#endif
 #ifndef SELKV_PACKED
 #define SELKV_PACKED 1    // packed f32x2 arguments and sums in the epilogues
 #endif
-// Which exponentials of a 32-wide chunk run as ex2_poly on the FMA pipe instead of the
-// special-function unit.  On GB300 at these shapes the epilogues are bound by instruction
-// issue rather than by the special-function unit, and moving exponentials to the FMA pipe
-// (2 to 10 of 32) only slowed them, so the default is none.
-__device__ __forceinline__ constexpr bool soft_exp(int i) { return (i & 15) < SELKV_SOFT_EXP; }
-__device__ __forceinline__ float ex2_mixed(float x, bool soft) { return soft ? ex2_poly(x) : ex2_approx(x); }
 
 #ifndef SELKV_P2_PIPE
 #define SELKV_P2_PIPE 1   // pass 2: pipelined 16-column TMEM loads on full, unmasked tiles
@@ -55,7 +46,7 @@ __device__ __forceinline__ float ex2_mixed(float x, bool soft) { return soft ? e
 // 2^(v sc - M_r - log2(G Z_r)).  The accumulator is read 16 columns at a time, each load
 // issued before the arithmetic on the previous one so its latency overlaps that work; row
 // pairs are packed (f32x2) and summed in four interleaved partial sums.
-__device__ __forceinline__ void colsum_accum16(const float (&v)[16], uint32_t rn, uint64_t sc2, int c0,
+__device__ __forceinline__ void colsum_accum16(const float (&v)[16], uint32_t rn, uint64_t sc2,
                                                uint64_t& a01, uint64_t& a23) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
@@ -63,8 +54,8 @@ __device__ __forceinline__ void colsum_accum16(const float (&v)[16], uint32_t rn
     float x0, x1, x2, x3;
     unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, pack_f2(nm.x, nm.y)), x0, x1);
     unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, pack_f2(nm.z, nm.w)), x2, x3);
-    a01 = fadd2(a01, pack_f2(ex2_mixed(x0, soft_exp(c0 + i)), ex2_mixed(x1, soft_exp(c0 + i + 1))));
-    a23 = fadd2(a23, pack_f2(ex2_mixed(x2, soft_exp(c0 + i + 2)), ex2_mixed(x3, soft_exp(c0 + i + 3))));
+    a01 = fadd2(a01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
+    a23 = fadd2(a23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
   }
 }
 __device__ __forceinline__ float colsum64(uint32_t taddr, uint32_t rn, float sc) {
@@ -76,10 +67,10 @@ __device__ __forceinline__ float colsum64(uint32_t taddr, uint32_t rn, float sc)
 #pragma unroll
   for (int c = 0; c < 4; c += 2) {
     tmem_ld16_issue(taddr + (c + 1) * 16, vb);
-    colsum_accum16(va, rn + c * 64, sc2, c * 16, a01, a23);
+    colsum_accum16(va, rn + c * 64, sc2, a01, a23);
     tmem_wait_ld16(vb);
     if (c + 2 < 4) tmem_ld16_issue(taddr + (c + 2) * 16, va);
-    colsum_accum16(vb, rn + (c + 1) * 64, sc2, (c + 1) * 16, a01, a23);
+    colsum_accum16(vb, rn + (c + 1) * 64, sc2, a01, a23);
     if (c + 2 < 4) tmem_wait_ld16(va);
   }
   float s0, s1, s2, s3;
@@ -285,15 +276,15 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
                   float x0, x1, x2, x3;
                   unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
                   unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
-                  s01 = fadd2(s01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
-                  s23 = fadd2(s23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
+                  s01 = fadd2(s01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
+                  s23 = fadd2(s23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
                 }
                 unpack_f2(s01, s0, s1);
                 unpack_f2(s23, s2, s3);
               } else {
                 float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_mixed(fmaf(v[i], sc, -mn), soft_exp(i));
+                for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_approx(fmaf(v[i], sc, -mn));
                 s0 = s4[0];
                 s1 = s4[1];
                 s2 = s4[2];
@@ -358,8 +349,8 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
                   float x0, x1, x2, x3;
                   unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, pack_f2(nm.x, nm.y)), x0, x1);
                   unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, pack_f2(nm.z, nm.w)), x2, x3);
-                  a01 = fadd2(a01, pack_f2(ex2_mixed(x0, soft_exp(i)), ex2_mixed(x1, soft_exp(i + 1))));
-                  a23 = fadd2(a23, pack_f2(ex2_mixed(x2, soft_exp(i + 2)), ex2_mixed(x3, soft_exp(i + 3))));
+                  a01 = fadd2(a01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
+                  a23 = fadd2(a23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
                 }
                 unpack_f2(a01, s0, s1);
                 unpack_f2(a23, s2, s3);
@@ -368,10 +359,10 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
 #pragma unroll
                 for (int i = 0; i < 32; i += 4) {
                   const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);
-                  s4[0] += ex2_mixed(fmaf(v[i], sc, nm.x), soft_exp(i));
-                  s4[1] += ex2_mixed(fmaf(v[i + 1], sc, nm.y), soft_exp(i + 1));
-                  s4[2] += ex2_mixed(fmaf(v[i + 2], sc, nm.z), soft_exp(i + 2));
-                  s4[3] += ex2_mixed(fmaf(v[i + 3], sc, nm.w), soft_exp(i + 3));
+                  s4[0] += ex2_approx(fmaf(v[i], sc, nm.x));
+                  s4[1] += ex2_approx(fmaf(v[i + 1], sc, nm.y));
+                  s4[2] += ex2_approx(fmaf(v[i + 2], sc, nm.z));
+                  s4[3] += ex2_approx(fmaf(v[i + 3], sc, nm.w));
                 }
                 s0 = s4[0];
                 s1 = s4[1];

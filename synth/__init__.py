@@ -169,6 +169,38 @@ def _store(x: np.ndarray, dtype: str) -> np.ndarray:
     return round_bf16(x) if dtype == "bf16" else x
 
 
+def gen_sequence(wl: Workload, layer: int, b: int, threads: int = 1) -> dict:
+    """Sequence b of gen_layer(wl, layer) alone (the same values): K, V [Hkv][n_b][d] and
+    Q_obs [Hq][W][d] (fp32 arrays holding storage-dtype values) and its length n_b."""
+    Hq, Hkv, d, W = wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.obs_window
+    n_b = int(seq_lengths(wl)[b])
+    K = np.empty((Hkv, n_b, d), dtype=np.float32)
+    V = np.empty((Hkv, n_b, d), dtype=np.float32)
+    Q = np.empty((Hq, W, d), dtype=np.float32)
+    heavy = heavy_positions(wl, layer, b, n_b)
+
+    def kv_unit(kv):
+        k, v = _segmented(_rng(wl.seed, layer, b, kv, _KV), n_b, d, wl, pair=True)
+        k[heavy] *= 4.0
+        K[kv] = _store(k, wl.dtype)
+        V[kv] = _store(v, wl.dtype)
+
+    def q_unit(h):
+        (q,) = _segmented(_rng(wl.seed, layer, b, h, _Q), W, d, wl, pair=False)
+        Q[h] = _store(q, wl.dtype)
+
+    if threads > 1:
+        with ThreadPoolExecutor(threads) as ex:
+            list(ex.map(kv_unit, range(Hkv)))
+            list(ex.map(q_unit, range(Hq)))
+    else:
+        for kv in range(Hkv):
+            kv_unit(kv)
+        for h in range(Hq):
+            q_unit(h)
+    return dict(K=K, V=V, Q_obs=Q, n=n_b)
+
+
 def gen_layer(wl: Workload, layer: int, threads: int = 1) -> dict:
     """K, V [B][Hkv][n_cap][d], Q_obs [B][Hq][W][d] (fp32 arrays holding storage-dtype
     values; rows at or beyond n_b are zero) and n_len [B]."""

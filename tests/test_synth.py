@@ -71,3 +71,16 @@ def test_serving_sweep_points(b, n, r):
     n_len = synth.seq_lengths(wl)
     assert n_len.shape == (b,) and (n_len >= n // 2).all() and (n_len <= n).all()
     assert (b, n, r) in synth.SWEEP_POINTS
+
+
+def test_gen_sequence_equals_the_layers_sequence():
+    """A sequence generated alone holds exactly the values gen_layer gives it."""
+    wl = synth.sweep(3, 2048, 0.25)
+    x = synth.gen_layer(wl, 2, threads=4)
+    for b in range(wl.batch):
+        s = synth.gen_sequence(wl, 2, b, threads=2)
+        n = int(x["n_len"][b])
+        assert s["n"] == n
+        np.testing.assert_array_equal(s["K"], x["K"][b, :, :n])
+        np.testing.assert_array_equal(s["V"], x["V"][b, :, :n])
+        np.testing.assert_array_equal(s["Q_obs"], x["Q_obs"][b])
