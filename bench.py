@@ -98,51 +98,106 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------ oracle arm
-def oracle_sample(wl: synth.Workload, layers: int = 1, decode_tokens: int = 2, per_head: bool = False):
-    """Time the fp64 oracle on a bounded sample of one step of `wl`: compression of `layers`
-    layers of sequence 0 and `decode_tokens` decode tokens over those layers; the rates are
-    scaled to the whole step (all layers, all sequences, all decode steps)."""
+def _oracle_unit(job):
+    """One unit of the oracle baseline, run in a worker process: generate layer `layer` of
+    sequence 0, compress it with the fp64 oracle, then decode `tokens` tokens over the
+    compressed cache (each appending a row).  Returns the times and the process's CPU time."""
+    wl, layer, tokens, per_head = job
     from oracle import selkv_oracle as O
-    cpu0 = os.times()
-    t_comp = 0.0
+    cpu0 = time.process_time()
+    one = wl.with_(batch=1)
+    x = synth.gen_layer(one, layer)
+    n = int(x["n_len"][0])
+    K, V, Q = (x[k][0].astype(np.float64) for k in ("K", "V", "Q_obs"))
+    t0 = time.perf_counter()
+    r = O.compress(K, V, Q, n, wl.rho, O.Params(select_mode=O.SELECT_PER_HEAD if per_head else O.SELECT_SHARED))
+    t_comp = time.perf_counter() - t0
+    dec = synth.gen_decode(one, layer, tokens)
+    Kc, Vc, bias = r.K_c, r.V_c, r.bias
     t_dec = 0.0
-    ncomp = 0
-    ndec = 0
-    for layer in range(layers):
-        x = synth.gen_layer(wl.with_(batch=1), layer, threads=os.cpu_count() or 1)
-        n = int(x["n_len"][0])
-        K, V, Q = (x["K"][0].astype(np.float64), x["V"][0].astype(np.float64),
-                   x["Q_obs"][0].astype(np.float64))
+    for t in range(tokens):
+        Kc = np.concatenate([Kc, dec["k_new"][t, 0][:, None]], axis=1)
+        Vc = np.concatenate([Vc, dec["v_new"][t, 0][:, None]], axis=1)
+        bias = np.concatenate([bias, np.zeros(bias.shape[:-1] + (1,))], axis=-1)
         t0 = time.perf_counter()
-        r = O.compress(K, V, Q, n, wl.rho,
-                       O.Params(select_mode=O.SELECT_PER_HEAD if per_head else O.SELECT_SHARED))
-        t_comp += time.perf_counter() - t0
-        ncomp += 1
-        dec = synth.gen_decode(wl.with_(batch=1), layer, decode_tokens)
-        Kc, Vc, bias = r.K_c, r.V_c, r.bias
-        for t in range(decode_tokens):
-            Kc = np.concatenate([Kc, dec["k_new"][t, 0][:, None]], axis=1)
-            Vc = np.concatenate([Vc, dec["v_new"][t, 0][:, None]], axis=1)
-            bias = np.concatenate([bias, np.zeros(bias.shape[:-1] + (1,))], axis=-1)
+        O.decode(dec["q"][t, 0], Kc, Vc, bias, Kc.shape[1])
+        t_dec += time.perf_counter() - t0
+    return {"compress_s": t_comp, "decode_s_per_token": t_dec / max(1, tokens),
+            "cpu_s": time.process_time() - cpu0}
+
+
+def _single_threaded_blas():
+    """Environment for worker processes: one BLAS / OpenMP thread each (the pool supplies the
+    parallelism)."""
+    keys = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS")
+    old = {k: os.environ.get(k) for k in keys}
+    for k in keys:
+        os.environ[k] = "1"
+    return old
+
+
+def _restore_env(old):
+    for k, v in old.items():
+        if v is None:
+            os.environ.pop(k, None)
+        else:
+            os.environ[k] = v
+
+
+def oracle_sample(wl: synth.Workload, per_head: bool = False, decode_tokens: int = 2,
+                  single_thread_refs: bool = True) -> dict:
+    """The fp64 oracle on the host's cores, parallel over independent units: one worker process
+    per core (spawned, single-threaded BLAS), each compressing one layer of sequence 0 (layers
+    0 .. P-1) and decoding `decode_tokens` tokens over it; all P run at once, so each unit's
+    time is taken under the memory contention of a full machine.  The step estimate schedules
+    the step's B x L (sequence, layer) units on the P cores: ceil(B L / P) rounds of the mean
+    unit time (compression + decode_steps decode tokens).  With single_thread_refs, the tiny
+    and the 16k single-layer workloads are also timed alone on one core (compression and
+    decode per layer)."""
+    import multiprocessing as mp
+    P = os.cpu_count() or 1
+    jobs = [(wl, layer % wl.layers, decode_tokens, per_head) for layer in range(P)]
+    refs = [(synth.WORKLOADS["tiny"], 0, 16, False), (synth.WORKLOADS["llama_layer"], 0, 2, False)]
+    old = _single_threaded_blas()
+    try:
+        ctx = mp.get_context("spawn")   # no fork of a process that holds a CUDA context
+        with ctx.Pool(P) as pool:
             t0 = time.perf_counter()
-            O.decode(dec["q"][t, 0], Kc, Vc, bias, Kc.shape[1])
-            t_dec += time.perf_counter() - t0
-            ndec += 1
-    per_layer_comp = t_comp / ncomp
-    per_layer_tok = t_dec / ndec
-    cpu1 = os.times()
-    # the cores kept busy on average (process CPU time / wall time, data generation included):
-    # numpy's BLAS pool spreads the oracle's products over the host's cores
-    busy = ((cpu1.user - cpu0.user) + (cpu1.system - cpu0.system)) / max(1e-9, cpu1.elapsed - cpu0.elapsed)
-    step_s = wl.batch * wl.layers * (per_layer_comp + wl.decode_steps * per_layer_tok)
+            res = pool.map(_oracle_unit, jobs, chunksize=1)
+            wall = time.perf_counter() - t0
+            single = pool.map(_oracle_unit, refs, chunksize=1) if single_thread_refs else None
+    finally:
+        _restore_env(old)
+    unit_s = statistics.mean(r["compress_s"] + wl.decode_steps * r["decode_s_per_token"] for r in res)
+    rounds = math.ceil(wl.batch * wl.layers / P)
+    step_s = rounds * unit_s
     tokens = wl.batch * wl.decode_steps
-    sample = ("fp64 oracle: compression of %d layer(s) x 1 sequence (n=%d) and %d decode token(s) "
-              "per layer, scaled to %d layers x %d sequences x %d decode steps"
-              % (layers, wl.n, decode_tokens, wl.layers, wl.batch, wl.decode_steps))
-    return dict(value=tokens / step_s, unit="tokens/s", cores=os.cpu_count(), kind="oracle",
-                sample=sample, compress_s_per_layer=per_layer_comp,
-                decode_s_per_layer_token=per_layer_tok, sample_wall_s=t_comp + t_dec,
-                cores_busy_avg=round(busy, 2))
+    busy = sum(r["cpu_s"] for r in res) / wall
+    out = {"value": tokens / step_s, "unit": "tokens/s", "cores": P, "kind": "oracle",
+           "sample": ("fp64 oracle, %d worker processes (one per core, single-threaded BLAS) at once, "
+                      "each compressing one layer of one sequence (n=%d) and decoding %d token(s); "
+                      "the step's %d (sequence, layer) units scheduled as %d round(s) of the mean "
+                      "unit (compression + %d decode tokens)")
+           % (P, wl.n, decode_tokens, wl.batch * wl.layers, rounds, wl.decode_steps),
+           "compress_s_per_layer": statistics.mean(r["compress_s"] for r in res),
+           "decode_s_per_layer_token": statistics.mean(r["decode_s_per_token"] for r in res),
+           "sample_wall_s": wall, "cores_busy_avg": round(busy, 2)}
+    if single is not None:
+        out["single_thread"] = {
+            w.name: {"compress_s": r["compress_s"], "decode_s_per_token": r["decode_s_per_token"],
+                     "tokens_per_s": w.decode_steps / (w.layers * (r["compress_s"]
+                                                                   + w.decode_steps * r["decode_s_per_token"]))}
+            for (w, _, _, _), r in zip(refs, single)}
+    return out
+
+
+def oracle_step_sample(wl: synth.Workload, layer: int, decode_tokens: int, per_head: bool = False) -> dict:
+    """One bounded sample of the oracle in this process (BLAS on all cores): compression of
+    layer `layer` of sequence 0 and `decode_tokens` decode tokens, scaled to the step."""
+    r = _oracle_unit((wl, layer, decode_tokens, per_head))
+    step_s = wl.batch * wl.layers * (r["compress_s"] + wl.decode_steps * r["decode_s_per_token"])
+    return {"value": wl.batch * wl.decode_steps / step_s, "compress_s": r["compress_s"],
+            "decode_s_per_token": r["decode_s_per_token"]}
 
 
 # ------------------------------------------------------------------------------ ranks
@@ -417,6 +472,8 @@ def run_gpu(args):
         if pj.get("workload") == wl.name and pj.get("kernel_rev") == kernel_revision():
             traffic = pj.get("bytes_per_launch")
 
+    score = None if args.no_score else measure_scoring(L, S, api, torch, stream, dev, peaks, peak_src)
+
     # full-cache comparison (same kernel, bias = NULL, uncompressed cache, no append)
     full_tok_s = None
     if not args.no_full:
@@ -468,6 +525,7 @@ def run_gpu(args):
                      "frac": achieved_gbs / peak_hbm, "peak_source": peak_src,
                      "bytes_per_launch": dec_bytes_per_layer_step,
                      "launch_us": dec_launch_us, "traffic": traffic},
+        "roofline_score": score,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
         "wall_s_timed": wall,
@@ -480,6 +538,62 @@ def run_gpu(args):
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def score_flops_per_pass(wl, n_len) -> float:
+    """Flops of one pass of the scoring: the product of the G W window rows of every KV head
+    with all n_b keys (2 d flops per score), over every sequence; the causal corner is
+    computed and masked, so executed and algorithmic flops agree.  The method needs this one
+    product; the second pass repeats it (it needs the row normalisers of the first)."""
+    return float(sum(2.0 * wl.num_q_heads * wl.obs_window * n * wl.head_dim for n in n_len))
+
+
+def measure_scoring(L: Layered, S, api, torch, stream, dev, peaks, peak_src, reps: int = 3) -> dict:
+    """The scoring stage (selkv_score) of every layer, its two passes timed apart: first the
+    row-statistics pass of all layers back to back (each layer its own small workspace), then
+    the column-sum pass of all layers; CUDA events around each group, per-pass time = group
+    time / layers (median over `reps`).  Every layer reads its own K (205 MB at 100k context),
+    so nothing stays in L2 from one layer to the next."""
+    wl = L.wl
+    sp = stream.cuda_stream
+    wss = [api.Workspace(S.selkv_score_workspace_size(L.shape), dev) for _ in range(wl.layers)]
+    attn = torch.empty((wl.batch, wl.num_kv_heads, wl.n), dtype=torch.float32, device=dev)
+    rounds = []
+    with torch.cuda.stream(stream):
+        for r in range(reps + 1):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            e[0].record(stream)
+            for layer in range(wl.layers):
+                S.check(S.selkv_score(L.shape, L.n_len, L.K[layer], L.Q[layer], None, S.SELKV_SCORE_ROWSTATS,
+                                      wss[layer].buf, wss[layer].nbytes, sp), "score pass 1")
+            e[1].record(stream)
+            for layer in range(wl.layers):
+                S.check(S.selkv_score(L.shape, L.n_len, L.K[layer], L.Q[layer], attn, S.SELKV_SCORE_COLSUMS,
+                                      wss[layer].buf, wss[layer].nbytes, sp), "score pass 2")
+            e[2].record(stream)
+            if r > 0:   # the first round warms up
+                rounds.append(e)
+    torch.cuda.synchronize()
+    assert all(w.errors(sp) == 0 for w in wss), "device error flags in the scoring"
+    p1 = statistics.median(x[0].elapsed_time(x[1]) for x in rounds) * 1e3 / wl.layers
+    p2 = statistics.median(x[1].elapsed_time(x[2]) for x in rounds) * 1e3 / wl.layers
+    F = score_flops_per_pass(wl, L.n_len)
+    peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+    burst = float(peaks["bf16_tflops"])
+    r1, r2 = F / (p1 * 1e-6) / 1e12, F / (p2 * 1e-6) / 1e12
+    stage = F / ((p1 + p2) * 1e-6) / 1e12
+    return {"kernel": "selkv scoring (tcgen05, two passes over K)" if wl.dtype == "bf16" else "selkv scoring",
+            "bound": "tensor", "unit": "TFLOP/s", "peak": peak, "peak_burst": burst, "peak_source": peak_src,
+            "flops_per_pass": F, "pass1_us": p1, "pass2_us": p2,
+            "pass1_tflops": r1, "pass2_tflops": r2,
+            "pass1_frac": r1 / peak, "pass2_frac": r2 / peak,
+            "pass1_frac_burst": r1 / burst, "pass2_frac_burst": r2 / burst,
+            "achieved": 2 * F / ((p1 + p2) * 1e-6) / 1e12, "frac": 2 * F / ((p1 + p2) * 1e-6) / 1e12 / peak,
+            "useful_tflops_stage": stage, "useful_frac_stage": stage / peak,
+            "note": "pass 1 includes the sequence-table upload and the fold of the row statistics; "
+                    "achieved = executed flops of both passes over their time; useful = one product "
+                    "(what the method needs) over the stage's time; peaks: sustained, and burst beside",
+            "traffic": None}
 
 
 def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: int):
@@ -796,6 +910,9 @@ def kernel_revision() -> str:
 
 
 def run_reference(args):
+    """The oracle arm: each step is one bounded sample of the workload's step (compression of
+    one layer, a different layer each step, and 8 decode tokens over it), timed in this process
+    with BLAS on the host's cores and scaled to the step; the line reports the median."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if world > 1 and rank != 0:
@@ -803,23 +920,39 @@ def run_reference(args):
     wl = synth.WORKLOADS[args.workload]
     if args.decode_steps is not None:
         wl = wl.with_(decode_steps=args.decode_steps)
-    vals = []
-    for _ in range(args.warmup):
-        oracle_sample(wl, layers=1, decode_tokens=1, per_head=args.select_mode == "per_head")
-    info = None
-    for _ in range(args.steps):
-        info = oracle_sample(wl, layers=1, decode_tokens=1, per_head=args.select_mode == "per_head")
-        vals.append(info["value"])
+    per_head = args.select_mode == "per_head"
+    tokens_per_sample = 8
+    for i in range(args.warmup):
+        oracle_step_sample(wl, i % wl.layers, 1, per_head)
+    vals, comp, dec = [], [], []
+    cpu0, t0 = os.times(), time.perf_counter()
+    for k in range(args.steps):
+        r = oracle_step_sample(wl, (args.warmup + k) % wl.layers, tokens_per_sample, per_head)
+        vals.append(r["value"])
+        comp.append(r["compress_s"])
+        dec.append(r["decode_s_per_token"])
+    wall = time.perf_counter() - t0
+    cpu1 = os.times()
+    busy = ((cpu1.user - cpu0.user) + (cpu1.system - cpu0.system)) / max(1e-9, wall)
     v = statistics.median(vals)
     tokens = wl.batch * wl.decode_steps
+    sample = ("fp64 oracle, one process with BLAS on the host's cores: per step the compression of "
+              "one layer of one sequence (n=%d; layers %d..%d over the steps) and %d decode tokens "
+              "over it, scaled to %d layers x %d sequences x %d decode steps"
+              % (wl.n, args.warmup % wl.layers, (args.warmup + args.steps - 1) % wl.layers,
+                 tokens_per_sample, wl.layers, wl.batch, wl.decode_steps))
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": tokens / v * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
             "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "n": wl.n,
-                       "rho": wl.rho, "decode_steps": wl.decode_steps, "select_mode": args.select_mode},
-            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
-                             "sample": info["sample"], "cores_busy_avg": info["cores_busy_avg"]},
+                       "rho": wl.rho, "decode_steps": wl.decode_steps, "q_heads": wl.num_q_heads,
+                       "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim, "obs_window": wl.obs_window,
+                       "select_mode": args.select_mode},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample, "cores_busy_avg": round(busy, 2),
+                             "compress_s_per_layer": statistics.median(comp),
+                             "decode_s_per_layer_token": statistics.median(dec)},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -841,6 +974,7 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=10, help="timed steps of the end-to-end measurement")
     ap.add_argument("--no-full", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-score", action="store_true", help="skip the timing of the scoring passes")
     ap.add_argument("--select-mode", default="shared", choices=["shared", "per_head"],
                     help="token selection: shared (GQA union, the default) or per_head (MHA)")
     ap.add_argument("--rope", default="off", choices=["off", "half", "interleaved"],

@@ -205,6 +205,44 @@ SELKV_API selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n
                             void* workspace, size_t workspace_bytes, selkv_stream_t stream);
 
 /* ---------------------------------------------------------------------------------------
+ * Observation-window attention alone: the scoring stage of selkv_compress (Sec. 3.1 re-pass;
+ * the attention sums Eq. 1 weights by ||v|| and Eq. 5 calls a).  For every sequence b, KV
+ * head kv and position j < n_b:
+ *   attn[b][kv][j] = (1/G) sum over the G query heads h = kv G + g and the W window rows i
+ *                    of softmax_j(Q_obs[b][h][i] . K[b][kv][j] / sqrt(d)),
+ * causal: row i sits at position n_b - W + i and sees keys j <= n_b - W + i.  The values are
+ * bitwise those of selkv_compress's `attn` debug output for the same inputs.
+ *
+ * It runs as two passes over K: the first finds each window row's softmax normaliser (the
+ * maximum and the sum of the exponentials), the second sums the normalised probabilities
+ * over the rows.  `passes` selects what the call runs:
+ *   SELKV_SCORE_ALL       both passes: attn is written;
+ *   SELKV_SCORE_ROWSTATS  the first pass only: the normalisers stay in the workspace and
+ *                         attn is not touched (may be NULL);
+ *   SELKV_SCORE_COLSUMS   the second pass only, from the normalisers that the previous
+ *                         ROWSTATS call on this workspace left (same shape, n_len, K and
+ *                         Q_obs; this call reuses that call's sequence lengths).
+ *
+ * n_len   HOST array [B]: prefill lengths, W <= n_b <= n_cap.
+ * K       [B][Hkv][n_cap][d]; Q_obs [B][Hq][W][d]; attn [B][Hkv][n_cap] fp32 output
+ *         (entries j >= n_b untouched).
+ * Errors: SELKV_ERR_INVALID_ARG for a NULL or misaligned tensor, a bad shape or length or an
+ * unknown `passes`; SELKV_ERR_UNSUPPORTED for d not in {64, 128}; SELKV_ERR_WORKSPACE when
+ * workspace_bytes < selkv_score_workspace_size.
+ * ------------------------------------------------------------------------------------- */
+typedef enum selkv_score_passes {
+  SELKV_SCORE_ROWSTATS = 1,
+  SELKV_SCORE_COLSUMS = 2,
+  SELKV_SCORE_ALL = 3
+} selkv_score_passes;
+
+SELKV_API size_t selkv_score_workspace_size(const selkv_shape* shape);
+
+SELKV_API selkv_status selkv_score(const selkv_shape* shape, const int32_t* n_len, const void* K,
+                                   const void* Q_obs, float* attn, int32_t passes, void* workspace,
+                                   size_t workspace_bytes, selkv_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------
  * Compensation averaged across layers (the overview of Sec. 3 offers it next to the
  * per-layer bias of Sec. 3.6).  After the L layers of a model have been compressed with the
  * same params, every layer's bias is replaced by one value per position shared by all
@@ -254,6 +292,7 @@ SELKV_API selkv_status selkv_layer_average_bias(const selkv_shape* shape, const 
  * k_new, v_new  [B][Hkv][d] or both NULL.
  * An empty cache with no new row gives out = 0.  An append that would pass m_cap is skipped
  * and sets SELKV_DEVERR_CAPACITY.
+
  * ------------------------------------------------------------------------------------- */
 SELKV_API size_t selkv_decode_workspace_size(const selkv_shape* shape);
 

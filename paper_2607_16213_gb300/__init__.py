@@ -12,12 +12,14 @@ from ._binding import (  # noqa: F401
     SELKV_GATE_CLOSED, SELKV_EMPTY_EXPAND, SELKV_EMPTY_DROP, SELKV_SELECT_SHARED,
     SELKV_SELECT_PER_HEAD, SELKV_ROPE_OFF, SELKV_ROPE_HALF, SELKV_ROPE_INTERLEAVED,
     SELKV_BIAS_RATIO, SELKV_BIAS_COUNT, SELKV_ROUTE_BUCKET, SELKV_ROUTE_COSINE,
+    SELKV_SCORE_ROWSTATS, SELKV_SCORE_COLSUMS, SELKV_SCORE_ALL,
     SELKV_DEVERR_CAPACITY,
     SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT, SELKV_MAX_BATCH,
     SelKVError, selkv_shape, selkv_params, selkv_compress_debug, library, library_path,
     exported_symbols, check, selkv_status_string, selkv_kernel_launches, selkv_workspace_init,
     selkv_workspace_error, selkv_compress_workspace_size, selkv_compress,
     selkv_decode_workspace_size, selkv_decode_attn, selkv_decode_attn_static,
-    selkv_layer_average_workspace_size, selkv_layer_average_bias,
+    selkv_layer_average_workspace_size, selkv_layer_average_bias, selkv_score_workspace_size,
+    selkv_score,
     SELKV_STATIC_SCRATCH_BYTES,
 )

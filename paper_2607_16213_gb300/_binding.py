@@ -18,6 +18,7 @@ SELKV_SELECT_SHARED, SELKV_SELECT_PER_HEAD = 0, 1
 SELKV_ROPE_OFF, SELKV_ROPE_HALF, SELKV_ROPE_INTERLEAVED = 0, 1, 2
 SELKV_BIAS_RATIO, SELKV_BIAS_COUNT = 0, 1
 SELKV_ROUTE_BUCKET, SELKV_ROUTE_COSINE = 0, 1
+SELKV_SCORE_ROWSTATS, SELKV_SCORE_COLSUMS, SELKV_SCORE_ALL = 1, 2, 3
 SELKV_DEVERR_CAPACITY, SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT = 1, 2, 4, 8
 SELKV_MAX_BATCH = 1024
 SELKV_STATIC_SCRATCH_BYTES = 4 << 20
@@ -86,6 +87,9 @@ def library() -> ctypes.CDLL:
         "selkv_compress": (c_i32, [ctypes.POINTER(selkv_shape), ctypes.POINTER(c_i32), c_f64,
                                    ctypes.POINTER(selkv_params), c_vp, c_vp, c_vp, c_vp, c_vp, c_vp,
                                    c_vp, ctypes.POINTER(selkv_compress_debug), c_vp, c_sz, c_vp]),
+        "selkv_score_workspace_size": (c_sz, [ctypes.POINTER(selkv_shape)]),
+        "selkv_score": (c_i32, [ctypes.POINTER(selkv_shape), ctypes.POINTER(c_i32), c_vp, c_vp, c_vp, c_i32,
+                                c_vp, c_sz, c_vp]),
         "selkv_layer_average_workspace_size": (c_sz, [ctypes.POINTER(selkv_shape)]),
         "selkv_layer_average_bias": (c_i32, [ctypes.POINTER(selkv_shape), ctypes.POINTER(selkv_params), c_i32,
                                              ctypes.POINTER(c_vp), ctypes.POINTER(c_vp), c_vp, c_vp, c_sz,
@@ -156,6 +160,18 @@ def selkv_workspace_error(workspace, stream=None):
 
 def selkv_compress_workspace_size(shape: selkv_shape) -> int:
     return int(library().selkv_compress_workspace_size(ctypes.byref(shape)))
+
+
+def selkv_score_workspace_size(shape: selkv_shape) -> int:
+    return int(library().selkv_score_workspace_size(ctypes.byref(shape)))
+
+
+def selkv_score(shape: selkv_shape, n_len, K, Q_obs, attn, passes: int, workspace, workspace_bytes: int,
+                stream=None) -> int:
+    """See include/selkv.h.  n_len: host sequence of B ints."""
+    n_arr = (c_i32 * shape.batch)(*[int(x) for x in n_len])
+    return library().selkv_score(ctypes.byref(shape), n_arr, _ptr(K), _ptr(Q_obs), _ptr(attn), int(passes),
+                                 _ptr(workspace), int(workspace_bytes), _stream(stream))
 
 
 def selkv_layer_average_workspace_size(shape: selkv_shape) -> int:

@@ -62,8 +62,14 @@ SideStream* side_stream(cudaStream_t caller) {
   return x.ready ? &x : nullptr;
 }
 
+// Key slices of the scoring's first pass (one row-statistics partial per slice and row).
+int score_chunks(const selkv_shape& s, int R) {
+  return score_uses_tc(s.dtype, s.head_dim, R) ? score_tc_splits(s.batch, s.num_kv_heads, s.n_cap, R, kPlanSMs)
+                                               : (int)(((size_t)s.n_cap + kRowChunk - 1) / kRowChunk);
+}
+
 struct CompressPlan {
-  size_t seq_n, seq_m, rowpart, rowstat, attn, attn_part, vnorm, rope_tab, mcount, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
+  size_t seq_n, seq_m, rowpart, rowstat, attn, vnorm, rope_tab, mcount, score, kflag, slot, kept_pos, tau, atau, ratio, select, total;
   size_t ev_pos, cos_invn, cos_rank, cos_order, cos_cnt, cos_seg;
   int nchunks, R;
 };
@@ -78,14 +84,12 @@ CompressPlan plan_compress(const selkv_shape& s) {
   };
   const size_t B = s.batch, Hkv = s.num_kv_heads, n = s.n_cap;
   p.R = (s.num_q_heads / s.num_kv_heads) * s.obs_window;
-  p.nchunks = score_uses_tc(s.dtype, s.head_dim, p.R) ? score_tc_splits(s.batch, s.num_kv_heads, s.n_cap, p.R, kPlanSMs)
-                                                       : (int)((n + kRowChunk - 1) / kRowChunk);
+  p.nchunks = score_chunks(s, p.R);
   p.seq_n = take(B * 4);
   p.seq_m = take(B * 4);
   p.rowpart = take(B * Hkv * (size_t)p.nchunks * p.R * sizeof(float2));
   p.rowstat = take(B * Hkv * (size_t)p.R * sizeof(float2));
   p.attn = take(B * Hkv * n * 4);
-  p.attn_part = score_uses_tc(s.dtype, s.head_dim, p.R) ? take(4 * B * Hkv * n * 4) : 0;
   p.vnorm = take(B * Hkv * n * 4);
   p.score = take(B * Hkv * n * 4);
   // kept flags, slot maps: per sequence, or per KV head in the per-head mode (sized for that)
@@ -109,6 +113,30 @@ CompressPlan plan_compress(const selkv_shape& s) {
   p.cos_cnt = take(B * Hkv * (size_t)cos_chunks_for(s.n_cap) * s.m_cap * 4);
   p.cos_seg = take(B * Hkv * (size_t)s.m_cap * 8);
   p.select = take(select_ws_bytes(s.batch, s.num_kv_heads, s.n_cap));
+  p.total = off;
+  return p;
+}
+
+struct ScorePlan {
+  size_t seq_n, seq_m, rowpart, rowstat, total;
+  int nchunks, R;
+};
+
+ScorePlan plan_score(const selkv_shape& s) {
+  ScorePlan p{};
+  size_t off = sizeof(WsHeader);
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += round256(bytes);
+    return o;
+  };
+  const size_t B = s.batch, Hkv = s.num_kv_heads;
+  p.R = (s.num_q_heads / s.num_kv_heads) * s.obs_window;
+  p.nchunks = score_chunks(s, p.R);
+  p.seq_n = take(B * 4);
+  p.seq_m = take(B * 4);
+  p.rowpart = take(B * Hkv * (size_t)p.nchunks * p.R * sizeof(float2));
+  p.rowstat = take(B * Hkv * (size_t)p.R * sizeof(float2));
   p.total = off;
   return p;
 }
@@ -289,8 +317,6 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
   a.rowstat = at<float2>(workspace, plan.rowstat);
   a.attn = (debug && debug->attn) ? debug->attn : at<float>(workspace, plan.attn);
   a.vnorm = at<float>(workspace, plan.vnorm);
-  a.attn_parts = score_uses_tc(a.dtype, a.D, a.R) ? 4 : 1;
-  a.attn_part = a.attn_parts == 4 ? at<float>(workspace, plan.attn_part) : nullptr;
   a.score = (debug && debug->score) ? debug->score : at<float>(workspace, plan.score);
   a.kflag = at<uint8_t>(workspace, plan.kflag);
   a.slot_of = at<int32_t>(workspace, plan.slot);
@@ -341,6 +367,67 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     e = launch_select_grid(a, sw, st);
   if (e == cudaSuccess) e = launch_merge(a, st);
   g_launches += (uint64_t)compress_kernel_count(a);
+  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+}
+
+size_t selkv_score_workspace_size(const selkv_shape* shape) {
+  if (!shape_ok(shape)) return 0;
+  return plan_score(*shape).total;
+}
+
+selkv_status selkv_score(const selkv_shape* shape, const int32_t* n_len, const void* K, const void* Q_obs,
+                         float* attn, int32_t passes, void* workspace, size_t workspace_bytes,
+                         selkv_stream_t stream) {
+  if (!shape_ok(shape) || n_len == nullptr) return SELKV_ERR_INVALID_ARG;
+  const selkv_shape& s = *shape;
+  if (s.head_dim != 64 && s.head_dim != 128) return SELKV_ERR_UNSUPPORTED;
+  if (s.obs_window < 1 || s.n_cap < 1) return SELKV_ERR_INVALID_ARG;
+  if (passes != SELKV_SCORE_ROWSTATS && passes != SELKV_SCORE_COLSUMS && passes != SELKV_SCORE_ALL)
+    return SELKV_ERR_INVALID_ARG;
+  if (K == nullptr || Q_obs == nullptr || !aligned(K, 16) || !aligned(Q_obs, 16)) return SELKV_ERR_INVALID_ARG;
+  if ((passes & SELKV_SCORE_COLSUMS) && (attn == nullptr || !aligned(attn, 16))) return SELKV_ERR_INVALID_ARG;
+  static thread_local SeqTable tab;
+  for (int b = 0; b < s.batch; ++b) {
+    const int n = n_len[b];
+    if (n < s.obs_window || n > s.n_cap) return SELKV_ERR_INVALID_ARG;
+    tab.n[b] = n;
+    tab.m[b] = 0;
+  }
+  const ScorePlan plan = plan_score(s);
+  if (workspace == nullptr || !aligned(workspace, 256)) return SELKV_ERR_WORKSPACE;
+  if (workspace_bytes < plan.total) return SELKV_ERR_WORKSPACE;
+  CompressArgs a{};
+  a.dtype = s.dtype;
+  a.B = s.batch;
+  a.Hq = s.num_q_heads;
+  a.Hkv = s.num_kv_heads;
+  a.G = s.num_q_heads / s.num_kv_heads;
+  a.D = s.head_dim;
+  a.W = s.obs_window;
+  a.n_cap = s.n_cap;
+  a.m_cap = s.m_cap;
+  a.R = plan.R;
+  a.nchunks = plan.nchunks;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s.head_dim));
+  a.K = K;
+  a.Q = Q_obs;
+  a.attn = attn;
+  a.flags = at<uint32_t>(workspace, 0);
+  a.seq_n = at<int32_t>(workspace, plan.seq_n);
+  a.seq_m = at<int32_t>(workspace, plan.seq_m);
+  a.rowpart = at<float2>(workspace, plan.rowpart);
+  a.rowstat = at<float2>(workspace, plan.rowstat);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaSuccess;
+  int kernels = 0;
+  if (passes & SELKV_SCORE_ROWSTATS) {  // the column-sum pass reuses the table of its row-statistics call
+    e = launch_seq_setup(a, tab, st);
+    kernels += 3;
+  }
+  if (passes & SELKV_SCORE_COLSUMS) kernels += 1;
+  if (e == cudaSuccess)
+    e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st, passes) : launch_score_simt(a, st, passes);
+  g_launches += (uint64_t)kernels;
   return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
 }
 

@@ -190,11 +190,14 @@ __global__ __launch_bounds__(256) void colsum_kernel(CompressArgs a) {
 }
 
 template <typename T, int D>
-cudaError_t launch_score_t(const CompressArgs& a, cudaStream_t s) {
+cudaError_t launch_score_t(const CompressArgs& a, cudaStream_t s, int passes) {
   const int row_tiles = (a.R + kTile - 1) / kTile;
-  rowstats_kernel<T, D><<<dim3(a.nchunks, row_tiles, a.B * a.Hkv), 256, 0, s>>>(a);
-  launch_rowstat_reduce(a, s);
-  colsum_kernel<T, D><<<dim3((a.n_cap + kTile - 1) / kTile, a.B * a.Hkv), 256, 0, s>>>(a);
+  if (passes & kScoreRowstats) {
+    rowstats_kernel<T, D><<<dim3(a.nchunks, row_tiles, a.B * a.Hkv), 256, 0, s>>>(a);
+    launch_rowstat_reduce(a, s);
+  }
+  if (passes & kScoreColsums)
+    colsum_kernel<T, D><<<dim3((a.n_cap + kTile - 1) / kTile, a.B * a.Hkv), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -206,10 +209,10 @@ cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s) {
+cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s, int passes) {
   if (a.dtype == SELKV_BF16)
-    return a.D == 128 ? launch_score_t<__nv_bfloat16, 128>(a, s) : launch_score_t<__nv_bfloat16, 64>(a, s);
-  return a.D == 128 ? launch_score_t<float, 128>(a, s) : launch_score_t<float, 64>(a, s);
+    return a.D == 128 ? launch_score_t<__nv_bfloat16, 128>(a, s, passes) : launch_score_t<__nv_bfloat16, 64>(a, s, passes);
+  return a.D == 128 ? launch_score_t<float, 128>(a, s, passes) : launch_score_t<float, 64>(a, s, passes);
 }
 
 }  // namespace selkv

@@ -16,8 +16,8 @@
 // owns one half of the R rows; an epilogue thread owns a row and a quarter of each tile's
 // keys, and the four quarter states of a row are folded at the end.  Pass 2 puts 128 keys in
 // the lanes and the R rows in the columns; an epilogue thread owns a key and a quarter of the
-// rows and writes that quarter's column sum; the pooling kernel of the selection adds the four
-// quarters of a key in a fixed order.
+// rows, and the four quarters' column sums of a key are added in shared memory in a fixed
+// order before a_j is written.
 //
 // Every wait is bounded; on timeout the CTA raises SELKV_DEVERR_TIMEOUT, keeps the barrier
 // protocol of its epilogue warps, lets issued copies and MMAs finish (bounded) and frees its
@@ -113,7 +113,7 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* rneg = reinterpret_cast<float*>(misc + 256);               // pass 2: -(M + log2(G Z)) per row
-  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [4][128] float2
+  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [4][128] float2; pass 2: [2][4][128]
 
   const int kv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -381,8 +381,14 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
-        // this row quarter's column sum; the pooling kernel adds the four quarters in order
-        if (j < n) a.attn_part[((size_t)part * a.B * a.Hkv + bk) * a.n_cap + j] = acc;
+        // the four row quarters' column sums of key j meet in shared memory (one buffer per
+        // accumulator, so a tile's sums are read before the buffer comes round again); the
+        // warp of quarter 0 adds them in quarter order and writes a_j
+        float* cs = colpart + buf * 512;  // [4][128]
+        cs[part * 128 + klane] = acc;
+        named_bar_sync(1 + q, 4 * 32);
+        if (part == 0 && j < n)
+          a.attn[bk * a.n_cap + j] = ((cs[klane] + cs[128 + klane]) + cs[256 + klane]) + cs[384 + klane];
       }
     }
   }
@@ -405,7 +411,7 @@ int splits_for(int B, int Hkv, int n_cap, int num_sms, int row_parts, int keys) 
 }
 
 template <int D>
-cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st) {
+cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st, int passes) {
   using C1 = SCfg<D, 1>;
   using C2 = SCfg<D, 2>;
   CUtensorMap tq, tk1, tk2;
@@ -421,10 +427,12 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st) {
   cudaError_t e = set_smem_once<score_tc_kernel<D, 1>>(C1::kSmem);
   if (e == cudaSuccess) e = set_smem_once<score_tc_kernel<D, 2>>(C2::kSmem);
   if (e != cudaSuccess) return e;
-  k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
-  e = launch_rowstat_reduce(a, st);
-  if (e != cudaSuccess) return e;
-  k2<<<grid2, kThreads, C2::kSmem, st>>>(tq, tk2, a);
+  if (passes & kScoreRowstats) {
+    k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
+    e = launch_rowstat_reduce(a, st);
+    if (e != cudaSuccess) return e;
+  }
+  if (passes & kScoreColsums) k2<<<grid2, kThreads, C2::kSmem, st>>>(tq, tk2, a);
   return cudaGetLastError();
 }
 
@@ -436,8 +444,8 @@ int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms) {
   return splits_for(B, Hkv, n_cap, num_sms, (R + 127) / 128, SCfg<128, 1>::kKeys);
 }
 
-cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t st) {
-  return a.D == 128 ? launch_tc_t<128>(a, st) : launch_tc_t<64>(a, st);
+cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t st, int passes) {
+  return a.D == 128 ? launch_tc_t<128>(a, st, passes) : launch_tc_t<64>(a, st, passes);
 }
 
 }  // namespace selkv

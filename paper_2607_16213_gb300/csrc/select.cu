@@ -20,6 +20,14 @@ __global__ void setup_kernel(SeqTable tab, CompressArgs a, SelectWs w) {
   }
 }
 
+// Sequence table alone (the scoring entry point).
+__global__ void seq_setup_kernel(SeqTable tab, int32_t* seq_n, int32_t* seq_m, int B) {
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    seq_n[b] = tab.n[b];
+    seq_m[b] = tab.m[b];
+  }
+}
+
 // ||v_j|| per row: D / 8 lanes per row (at most 16), each loading 8 elements at a time.
 template <typename T, int D>
 __global__ void vnorm_kernel(CompressArgs a) {
@@ -65,6 +73,11 @@ void launch_norms(const CompressArgs& a, cudaStream_t s) {
 
 cudaError_t launch_setup(const CompressArgs& a, const SeqTable& tab, const SelectWs& w, cudaStream_t s) {
   setup_kernel<<<1, 256, 0, s>>>(tab, a, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s) {
+  seq_setup_kernel<<<1, 256, 0, s>>>(tab, a.seq_n, a.seq_m, a.B);
   return cudaGetLastError();
 }
 

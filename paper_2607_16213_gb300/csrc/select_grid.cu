@@ -98,26 +98,19 @@ __global__ __launch_bounds__(kBlock, SELKV_SEL_MINB) void pool_hist0_kernel(Comp
   for (int i = threadIdx.x; i < kBins; i += kBlock) sh[i] = 0u;
   __syncthreads();
   const int half = a.pool_kernel / 2;
-  float* at = a.attn + (size_t)u * a.n_cap;
+  const float* at = a.attn + (size_t)u * a.n_cap;
   const float* vn = a.vnorm + (size_t)u * a.n_cap;
   float* sc = a.score + (size_t)u * a.n_cap;
-  // a_j: final, or the sum of the scoring's four row-quarter column sums in quarter order
-  const size_t plane = (size_t)a.B * a.Hkv * a.n_cap;
-  const float* ap = a.attn_parts == 4 ? a.attn_part + (size_t)u * a.n_cap : nullptr;
-  auto attn_at = [&](int jj) -> float {
-    return ap != nullptr ? ((ap[jj] + ap[plane + jj]) + ap[2 * plane + jj]) + ap[3 * plane + jj] : at[jj];
-  };
   const int j0 = blockIdx.x * kSpan;
 #pragma unroll 1
   for (int e = 0; e < kPerThread; ++e) {
     const int j = j0 + e * kBlock + threadIdx.x;
     if (j >= n) continue;
-    if (ap != nullptr) at[j] = attn_at(j);  // the attention later kernels read
     float s = 0.f;
     if (j < ncand) {
       for (int t = -half; t <= half; ++t) {
         const int jj = j + t;
-        if (jj >= 0 && jj < ncand) s += attn_at(jj) * vn[jj];
+        if (jj >= 0 && jj < ncand) s += at[jj] * vn[jj];
       }
       s = s / (float)a.pool_kernel;
       if (active) atomicAdd(&sh[__float_as_uint(s) >> 21], 1u);

@@ -169,8 +169,6 @@ struct CompressArgs {
   float2* rowpart;   // [B][Hkv][nchunks][R] (max, sum) of 2^(s' - max) per column chunk
   float2* rowstat;   // [B][Hkv][R] (M, 1 / (G * Z))
   float* attn;       // [B][Hkv][n_cap]
-  float* attn_part;  // [4][B][Hkv][n_cap] column sums of four row quarters (tensor-core scoring)
-  int attn_parts;    // 4: attn is the sum of attn_part, formed by the pooling kernel; 1: attn is final
   float* vnorm;      // [B][Hkv][n_cap]
   float* score;      // [B][Hkv][n_cap]
   uint8_t* kflag;    // [units][n_cap] 1 = kept (units: B, or B * Hkv in per-head mode)
@@ -264,8 +262,11 @@ cudaError_t launch_select_grid(const CompressArgs& a, const SelectWs& w, cudaStr
 // Scoring: tensor-core path for bf16 with G W <= 256 rows, CUDA-core path otherwise.
 bool score_uses_tc(int dtype, int D, int R);
 int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms);  // pass-1 key splits
-cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s);
-cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s);
+// passes: bit 0 = row statistics (pass 1 and their fold), bit 1 = column sums (pass 2)
+constexpr int kScoreRowstats = 1, kScoreColsums = 2, kScoreAll = 3;
+cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t s, int passes = kScoreAll);
+cudaError_t launch_score_simt(const CompressArgs& a, cudaStream_t s, int passes = kScoreAll);
+cudaError_t launch_seq_setup(const CompressArgs& a, const SeqTable& tab, cudaStream_t s);
 cudaError_t launch_rowstat_reduce(const CompressArgs& a, cudaStream_t s);
 // Compensation averaged across layers (layer_average.cu).
 constexpr int kMaxLayers = 128;

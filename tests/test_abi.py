@@ -107,6 +107,30 @@ def test_decode_rejects_invalid_arguments(lib):
     assert dec(wsb=100) == S.SELKV_ERR_WORKSPACE
 
 
+def test_score_rejects_invalid_arguments(lib):
+    s = shape()
+    ws_size = S.selkv_score_workspace_size(s)
+    assert ws_size > 256 and ws_size % 256 == 0 and ws_size < S.selkv_compress_workspace_size(s)
+    assert S.selkv_score_workspace_size(shape(num_kv_heads=7)) == 0
+    sc = lambda **kw: S.selkv_score(kw.get("shape", s), kw.get("n_len", [16384]), kw.get("K", FAKE), FAKE,
+                                    kw.get("attn", FAKE), kw.get("passes", S.SELKV_SCORE_ALL),
+                                    kw.get("ws", FAKE), kw.get("wsb", 1 << 40), 0)
+    assert sc(passes=0) == S.SELKV_ERR_INVALID_ARG
+    assert sc(passes=4) == S.SELKV_ERR_INVALID_ARG
+    assert sc(n_len=[40]) == S.SELKV_ERR_INVALID_ARG           # W = 64 > n_b
+    assert sc(n_len=[20000]) == S.SELKV_ERR_INVALID_ARG        # n_b > n_cap
+    assert sc(K=0) == S.SELKV_ERR_INVALID_ARG
+    assert sc(K=FAKE + 8) == S.SELKV_ERR_INVALID_ARG
+    assert sc(attn=0) == S.SELKV_ERR_INVALID_ARG               # the column sums need an output
+    assert sc(attn=0, passes=S.SELKV_SCORE_COLSUMS) == S.SELKV_ERR_INVALID_ARG
+    assert sc(shape=shape(head_dim=96)) == S.SELKV_ERR_UNSUPPORTED
+    assert sc(ws=0) == S.SELKV_ERR_WORKSPACE
+    assert sc(wsb=ws_size - 256) == S.SELKV_ERR_WORKSPACE
+    # the row-statistics pass alone writes no attention: a NULL output passes validation
+    # (checked with a workspace too small, so that nothing is launched)
+    assert sc(attn=0, passes=S.SELKV_SCORE_ROWSTATS, wsb=16) == S.SELKV_ERR_WORKSPACE
+
+
 def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     import paper_2607_16213_gb300._binding as bind
     monkeypatch.setattr(bind, "_LIB", None)

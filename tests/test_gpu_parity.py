@@ -564,3 +564,37 @@ def test_layer_average_one_layer_is_identity():
         m = int(host["lengths"][b])
         np.testing.assert_allclose(cache.bias[b, :, :m].cpu().numpy(), before[b, :, :m].cpu().numpy(),
                                    rtol=0, atol=2e-6)
+
+
+# ---------------------------------------------------------------- scoring stage on its own
+@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4"])
+def test_score_entry_point(name):
+    """selkv_score (Sec. 3.1 re-pass, Eq. 1's attention sums): a within ATTN_RTOL of the
+    oracle; bitwise the `attn` of selkv_compress; the two passes run as separate calls
+    (row statistics, then column sums) give bitwise the one-call result."""
+    from parity import ATTN_RTOL
+    wl = SMALL[name]
+    x = synth.gen_layer(wl, 9)
+    n_len = [int(v) for v in x["n_len"]]
+    m_cap = api.capacity(max(n_len), wl.rho)
+    shape = api.make_shape(wl.dtype, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                           wl.obs_window, wl.n, m_cap)
+    K, Q = to_dev(x["K"], wl.dtype), to_dev(x["Q_obs"], wl.dtype)
+    ws = api.Workspace(S.selkv_score_workspace_size(shape))
+    a_all = torch.full((wl.batch, wl.num_kv_heads, wl.n), -1.0, device="cuda")
+    a_two = torch.full_like(a_all, -2.0)
+    S.check(S.selkv_score(shape, n_len, K, Q, a_all, S.SELKV_SCORE_ALL, ws.buf, ws.nbytes), "score")
+    S.check(S.selkv_score(shape, n_len, K, Q, None, S.SELKV_SCORE_ROWSTATS, ws.buf, ws.nbytes), "rowstats")
+    S.check(S.selkv_score(shape, n_len, K, Q, a_two, S.SELKV_SCORE_COLSUMS, ws.buf, ws.nbytes), "colsums")
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    _, host, _ = run_compress(wl, x, O.Params())
+    got, two = a_all.cpu().numpy(), a_two.cpu().numpy()
+    for b in range(wl.batch):
+        n = n_len[b]
+        want = O.cumulative_attention(x["Q_obs"][b].astype(np.float64), x["K"][b].astype(np.float64), n)
+        err = np.abs(got[b, :, :n] - want) / (np.abs(want) + 1e-30)
+        assert err.max() <= ATTN_RTOL, "attention rel err %.3g" % err.max()
+        np.testing.assert_array_equal(got[b, :, :n], host["attn"][b, :, :n])
+        np.testing.assert_array_equal(two[b, :, :n], got[b, :, :n])
+        assert (got[b, :, n:] == -1.0).all(), "entries past n_b were written"
