@@ -211,15 +211,18 @@ def max_over_ranks(x: float, torch, dist, device) -> float:
     return float(t.item())
 
 
-def decode_bytes_per_launch(wl, n_len, T: int) -> float:
+def decode_bytes_per_launch(wl, n_len, T: int, per_head: bool = False) -> float:
     """Algorithmic bytes of one decode launch (one layer, one token), averaged over T tokens:
-    each cached row of each KV head reads its K_c and V_c rows (d elements each) and one fp32
-    bias, the row appended at step t included (a sequence holds m_b + t + 1 rows at step t);
-    plus the queries and outputs of every query head and the appended key and value rows."""
+    each cached row of each KV head reads its K_c and V_c rows (d elements each), and each
+    cached position its fp32 bias (one value per position shared by the KV heads in the shared
+    selection mode, one per KV head in the per-head mode), the row appended at step t included
+    (a sequence holds m_b + t + 1 rows at step t); plus the queries and outputs of every query
+    head and the appended key and value rows.  (The kernel reads the shared-mode bias from
+    every KV head's copy of the row: 4 (Hkv - 1) bytes per position more than counted here.)"""
     esz = 2 if wl.dtype == "bf16" else 4
     d, Hkv, Hq = wl.head_dim, wl.num_kv_heads, wl.num_q_heads
     m_b = [int(math.floor(wl.rho * n)) for n in n_len]
-    per_row = Hkv * (2 * d * esz + 4)
+    per_row = Hkv * 2 * d * esz + 4 * (Hkv if per_head else 1)
     rows_total = sum(sum(m + t + 1 for t in range(T)) for m in m_b)   # over the T steps
     fixed = T * len(n_len) * (2 * Hq * d * esz + 2 * Hkv * d * esz)
     return (rows_total * per_row + fixed) / T
@@ -389,6 +392,9 @@ def run_gpu(args):
         routing=S.SELKV_ROUTE_COSINE if args.routing == "cosine" else S.SELKV_ROUTE_BUCKET)
     L = Layered(wl, torch, api, S, dev, pinned_host=not args.no_e2e, layer_average=args.layer_average,
                 compress_streams=args.compress_streams)
+    # inputs, caches and workspaces were initialised on the default stream; the work below runs
+    # on other streams, which do not wait for it
+    torch.cuda.synchronize()
     stream = torch.cuda.Stream(device=dev)
     sp = stream.cuda_stream
     peaks, peak_src = load_peaks()
@@ -460,7 +466,7 @@ def run_gpu(args):
     decode_tok_s = tokens_per_step / (dec_ms_avg / 1e3)
 
     d, Hkv, Hq, B = wl.head_dim, wl.num_kv_heads, wl.num_q_heads, wl.batch
-    dec_bytes_per_layer_step = decode_bytes_per_launch(wl, L.n_len, L.T)
+    dec_bytes_per_layer_step = decode_bytes_per_launch(wl, L.n_len, L.T, per_head=args.select_mode == "per_head")
     dec_launch_us = dec_ms_avg * 1e3 / n_dec_launch
     achieved_gbs = dec_bytes_per_layer_step / (dec_launch_us * 1e-6) / 1e9
     peak_hbm = float(peaks["hbm_gbs"])
@@ -480,6 +486,7 @@ def run_gpu(args):
         fshape = api.make_shape(wl.dtype, B, Hq, Hkv, d, wl.obs_window, wl.n, wl.n)
         flen = torch.tensor(L.n_len, dtype=torch.int32, device=dev)
         fws = api.Workspace(S.selkv_decode_workspace_size(fshape), dev)
+        torch.cuda.synchronize()   # flen and fws are ready before `stream` uses them
         nfull = max(2, min(16, L.T))
         def full_pass():
             for t in range(nfull):
@@ -512,8 +519,12 @@ def run_gpu(args):
                    "rope": args.rope, "routing": args.routing,
                    "compensation": "averaged across layers" if args.layer_average else "per layer",
                    "parallelism": "replicas", "compress_streams": max(1, args.compress_streams),
-                   "l2": "inputs larger than L2: every token streams all layers' compressed "
-                         "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9),
+                   "l2": (("inputs larger than L2: every token streams all layers' compressed "
+                           "caches (%.2f GB)" % (dec_bytes_per_layer_step * wl.layers / 1e9))
+                          if dec_bytes_per_layer_step * wl.layers > 2 * L2_BYTES else
+                          ("L2-resident: the workload's compressed caches (%.0f MB per token over all "
+                           "layers) fit in L2, so the decode figures are not HBM figures"
+                           % (dec_bytes_per_layer_step * wl.layers / 1e6))),
                    "cuda_graph": True},
         "decode_tok_s": decode_tok_s,
         "decode_gbs": achieved_gbs,
@@ -558,6 +569,7 @@ def measure_scoring(L: Layered, S, api, torch, stream, dev, peaks, peak_src, rep
     sp = stream.cuda_stream
     wss = [api.Workspace(S.selkv_score_workspace_size(L.shape), dev) for _ in range(wl.layers)]
     attn = torch.empty((wl.batch, wl.num_kv_heads, wl.n), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()   # the workspaces are zeroed before `stream` uses them
     rounds = []
     with torch.cuda.stream(stream):
         for r in range(reps + 1):
@@ -765,19 +777,24 @@ def sweep_point(args, point, torch, S, api, dev, peaks, peak_src) -> dict:
     sp = stream.cuda_stream
     cache = api.alloc_compressed(shape, dev)
     ws = api.Workspace(S.selkv_compress_workspace_size(shape), dev)
+    torch.cuda.synchronize()   # zeroed on the default stream; `stream` does not wait for it
 
     def compress():
         S.check(S.selkv_compress(shape, n_len, rho, params, K, V, Q, cache.K_c, cache.V_c, cache.bias,
                                  cache.lengths, None, ws.buf, ws.nbytes, sp), "compress")
 
+    m_b = [int(math.floor(rho * v)) for v in n_len]
     with torch.cuda.stream(stream):
         compress()
     torch.cuda.synchronize()
     assert ws.errors(sp) == 0
+    if cache.lengths.cpu().tolist() != m_b:
+        raise RuntimeError("lengths after the first compression: %s, expected %s"
+                           % (cache.lengths.cpu().tolist()[:8], m_b[:8]))
     g_comp = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_comp, stream=stream):
         compress()
-    lengths0 = cache.lengths.clone()
+    lengths0 = torch.tensor(m_b, dtype=torch.int32, device=dev)
 
     dec_bytes = decode_bytes_per_launch(wl, n_len, T)
     copies = max(1, min(32, int(math.ceil(3 * L2_BYTES / dec_bytes))))
@@ -790,6 +807,7 @@ def sweep_point(args, point, torch, S, api, dev, peaks, peak_src) -> dict:
     out = torch.empty((T, B, Hq, d), dtype=bf, device=dev)
     dws = api.Workspace(S.selkv_decode_workspace_size(shape), dev)
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    torch.cuda.synchronize()   # the copies, inputs and workspace are ready before `stream` uses them
     g_dec, g_flush = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_dec, stream=stream):
         for t in range(T):
@@ -807,13 +825,18 @@ def sweep_point(args, point, torch, S, api, dev, peaks, peak_src) -> dict:
             c.lengths.copy_(lengths0)
 
     with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
+        for i in range(args.warmup):
             flush.zero_()
             g_comp.replay()
+            if i == 0:
+                comp_len = cache.lengths.clone()
             reset_lengths()
             g_dec.replay()
             g_flush.replay()
     torch.cuda.synchronize()
+    if comp_len.cpu().tolist() != m_b:
+        raise RuntimeError("lengths after a replayed compression: %s, expected %s"
+                           % (comp_len.cpu().tolist()[:8], m_b[:8]))
     steps = max(args.steps, 10)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
     clocks = ClockSampler(torch.cuda.current_device() if not os.environ.get("CUDA_VISIBLE_DEVICES") else 0)
@@ -835,10 +858,16 @@ def sweep_point(args, point, torch, S, api, dev, peaks, peak_src) -> dict:
                 ev[k][5].record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
-    want = [int(math.floor(rho * v)) + T for v in n_len]
-    for c in caches:
-        assert c.lengths.cpu().tolist() == want, "lengths after the timed decode"
-    assert ws.errors(sp) == 0 and dws.errors(sp) == 0, "device error flags"
+    want = [m + T for m in m_b]
+    cflags, dflags = ws.errors(sp), dws.errors(sp)
+    for i, c in enumerate(caches):
+        got = c.lengths.cpu().tolist()
+        if got != want:
+            bad = [(b, got[b], want[b]) for b in range(B) if got[b] != want[b]]
+            raise RuntimeError("lengths after the timed decode (copy %d of %d; (seq, got, want) %s; "
+                               "device flags compress %#x decode %#x; m_cap %d)"
+                               % (i, copies, bad[:8], cflags, dflags, m_cap))
+    assert cflags == 0 and dflags == 0, "device error flags %#x %#x" % (cflags, dflags)
     comp_ms = statistics.median(ev[k][0].elapsed_time(ev[k][1]) for k in range(steps))
     dec_ms = statistics.median(ev[k][2].elapsed_time(ev[k][3]) for k in range(steps))
     flush_ms = statistics.median(ev[k][4].elapsed_time(ev[k][5]) for k in range(steps)) if flush_tokens else 0.0
@@ -889,8 +918,18 @@ def run_sweep(args, points):
     _build.build()
     S.library()
     peaks, peak_src = load_peaks()
+    failed = 0
     for pt in points:
-        print(json.dumps(sweep_point(args, pt, torch, S, api, dev, peaks, peak_src)), flush=True)
+        try:
+            line = sweep_point(args, pt, torch, S, api, dev, peaks, peak_src)
+        except (RuntimeError, AssertionError) as e:   # report the point and go on with the others
+            failed += 1
+            line = {"metric": SWEEP_METRIC, "config": {"workload": synth.sweep(*pt).name}, "error": str(e)}
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+        print(json.dumps(line), flush=True)
+    if failed:
+        sys.exit(1)
 
 
 DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "decode_simt.cu", "ptx.cuh", "selkv_internal.cuh",

@@ -87,20 +87,6 @@ __device__ __forceinline__ uint64_t fmul2(uint64_t x, uint64_t y) {
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(x), "l"(y));
   return d;
 }
-__device__ __forceinline__ float fmax3(float x, float y, float z) {
-  float d;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(x), "f"(y), "f"(z));
-  return d;
-}
-__device__ __forceinline__ float max32(const float (&x)[32]) {
-  float mx[11];
-#pragma unroll
-  for (int i = 0; i < 10; ++i) mx[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
-  mx[10] = fmaxf(x[30], x[31]);
-  const float m0 = fmax3(mx[0], mx[1], mx[2]), m1 = fmax3(mx[3], mx[4], mx[5]);
-  const float m2 = fmax3(mx[6], mx[7], mx[8]), m3 = fmax3(mx[9], mx[10], m0);
-  return fmax3(m1, m2, m3);
-}
 
 template <int D>
 __global__ __launch_bounds__(kThreads, 1) void cos_tc_kernel(const __grid_constant__ CUtensorMap tmB, CompressArgs a) {

@@ -34,9 +34,6 @@ constexpr int kEpiWarps = 16;
 constexpr int kProducerWarp = 16, kMmaWarp = 17;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 columns
-#ifndef SELKV_PACKED
-#define SELKV_PACKED 1    // packed f32x2 arguments and sums in the epilogues
-#endif
 
 #ifndef SELKV_P2_PIPE
 #define SELKV_P2_PIPE 1   // pass 2: pipelined 16-column TMEM loads on full, unmasked tiles
@@ -79,11 +76,15 @@ __device__ __forceinline__ float colsum64(uint32_t taddr, uint32_t rn, float sc)
   return (s0 + s1) + (s2 + s3);
 }
 
-template <int D, int PASS>
+// HALVES (pass 2): 1 when the R rows fit one accumulator of 256 columns, 2 when they take two
+// (R up to 512): each key tile is then multiplied by the two 256-row halves of Q in turn, the
+// halves alternating between the two accumulators, and the K ring is shortened to make room
+// for the 512 staged rows.
+template <int D, int PASS, int HALVES = 1>
 struct SCfg {
-  static constexpr int kKeys = PASS == 1 ? 256 : 128;    // keys per tile
-  static constexpr int kStages = PASS == 1 ? 2 : 4;      // K tiles in flight
-  static constexpr int kRows = PASS == 1 ? 128 : 256;    // Q rows staged per CTA
+  static constexpr int kKeys = PASS == 1 ? 256 : 128;                  // keys per tile
+  static constexpr int kStages = PASS == 1 ? 2 : (HALVES == 2 ? 2 : 4);  // K tiles in flight
+  static constexpr int kRows = PASS == 1 ? 128 : 256 * HALVES;          // Q rows staged per CTA
   static constexpr int kBoxes = D / 64;                  // 128-byte-wide boxes per row
   static constexpr int kKTile = kKeys * D * 2;           // one K tile
   static constexpr int kQBytes = kRows * D * 2;
@@ -92,11 +93,11 @@ struct SCfg {
   static constexpr int kSmem = 1024 + kQBytes + kRing + kMisc;
 };
 
-template <int D, int PASS>
+template <int D, int PASS, int HALVES>
 __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                                                                 const __grid_constant__ CUtensorMap tmK,
                                                                 CompressArgs a) {
-  using C = SCfg<D, PASS>;
+  using C = SCfg<D, PASS, HALVES>;
   constexpr int kKeys = C::kKeys, kStages = C::kStages;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
@@ -119,12 +120,12 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = a.seq_n[b];
   const int R = a.R;
-  const int Rp = (R + 15) & ~15;              // N of the pass-2 MMA
+  const int Rp = (R + 15) & ~15;              // N of the pass-2 MMAs over all halves
   const int MT = (R + 127) / 128;             // 128-row halves of the R rows
   const int h = PASS == 1 ? (int)blockIdx.x % MT : 0;           // pass 1: this CTA's rows
   const int split = PASS == 1 ? (int)blockIdx.x / MT : (int)blockIdx.x;
   const int nsplit = PASS == 1 ? (int)gridDim.x / MT : (int)gridDim.x;
-  const int Rq = PASS == 1 ? 128 : (R > 128 ? 256 : 128);     // rows of Q staged (whole TMA boxes)
+  const int Rq = PASS == 1 ? 128 : (HALVES == 2 ? 512 : (R > 128 ? 256 : 128));  // Q rows staged (whole boxes)
   const int ntiles_all = (n + kKeys - 1) / kKeys;
   const int per = (ntiles_all + nsplit - 1) / nsplit;
   const int t_begin = split * per;
@@ -149,7 +150,7 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   }
   if (warp == kMmaWarp) tmem_alloc(tmem_slot, kTmemCols);
   if (PASS == 2)
-    for (int r = threadIdx.x; r < 256; r += blockDim.x) {
+    for (int r = threadIdx.x; r < 256 * HALVES; r += blockDim.x) {
       // 2^(s' - M) / (G Z) = 2^(s' - (M + log2(G Z))): the normaliser joins the exponent
       const float2 st = r < R ? a.rowstat[bk * R + r] : make_float2(0.f, 0.f);
       rneg[r] = st.y > 0.f ? -(st.x - log2f(st.y)) : -INFINITY;
@@ -185,30 +186,37 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   } else if (warp == kMmaWarp) {
     if (lane == 0 && nt > 0) {
       bool ok = mbar_wait(qbar, 0);
-      const uint32_t idesc = PASS == 1 ? umma_idesc_bf16(128, kKeys) : umma_idesc_bf16(128, Rp);
       const uint32_t qbase = smem_u32(Qs);
-      int t = 0;
-      for (; ok && t < nt; ++t) {
-        const int st = t % kStages, buf = t & 1;
-        if (!mbar_wait(&full[st], (t / kStages) & 1) || !mbar_wait(&tempty[buf], ((t >> 1) & 1) ^ 1) ||
-            *abort_flag) {
+      int u = 0;  // accumulator use: one per (key tile, row half)
+      for (int t = 0; ok && t < nt; ++t) {
+        const int st = t % kStages;
+        if (!mbar_wait(&full[st], (t / kStages) & 1) || *abort_flag) {
           ok = false;
           break;
         }
-        tc_fence_after();
         const uint32_t kbase = smem_u32(Ks + st * C::kKTile);
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t koff = (ks >> 2) * (kKeys * 128) + (ks & 3) * 32;
-          const uint32_t qoff = (ks >> 2) * (Rq * 128) + (ks & 3) * 32;
-          if (PASS == 1) {
-            umma_bf16(tmem + buf * 256, umma_desc_sw128(qbase + qoff), umma_desc_sw128(kbase + koff), idesc, ks > 0);
-          } else {
-            umma_bf16(tmem + buf * 256, umma_desc_sw128(kbase + koff), umma_desc_sw128(qbase + qoff), idesc, ks > 0);
+        for (int ph = 0; ph < HALVES; ++ph, ++u) {
+          const int buf = u & 1;
+          if (!mbar_wait(&tempty[buf], ((u >> 1) & 1) ^ 1) || *abort_flag) {
+            ok = false;
+            break;
           }
+          tc_fence_after();
+          const uint32_t idesc = PASS == 1 ? umma_idesc_bf16(128, kKeys) : umma_idesc_bf16(128, min(256, Rp - ph * 256));
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint32_t koff = (ks >> 2) * (kKeys * 128) + (ks & 3) * 32;
+            const uint32_t qoff = (ks >> 2) * (Rq * 128) + (ks & 3) * 32 + ph * 256 * 128;
+            if (PASS == 1) {
+              umma_bf16(tmem + buf * 256, umma_desc_sw128(qbase + qoff), umma_desc_sw128(kbase + koff), idesc, ks > 0);
+            } else {
+              umma_bf16(tmem + buf * 256, umma_desc_sw128(kbase + koff), umma_desc_sw128(qbase + qoff), idesc, ks > 0);
+            }
+          }
+          umma_commit(&tfull[buf]);
         }
+        if (!ok) break;
         umma_commit(&empty[st]);
-        umma_commit(&tfull[buf]);
       }
       if (!ok) {
         *abort_flag = 1;
@@ -245,55 +253,44 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         tc_fence_after();
         const int key0 = (t_begin + t) * kKeys + part * 64;
         const bool full_quarter = key0 + 63 <= n - a.W;  // every row sees every key of the quarter
-        // (pass 1 keeps 32-column loads: 16-column pipelined loads, as in pass 2, measured
-        // slower here, the running max then needing a correction every 16 keys)
-        if (ok) {
-#pragma unroll 1
-          for (int c = 0; c < 64; c += 32) {
-            float v[32];
-            tmem_ld32(tmem + lane_base + buf * 256 + part * 64 + c, v);
-            float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (full_quarter && row_ok) {
+        // one 32-column chunk of this thread's row: masked where the row does not see the key
+        // (or the row does not exist), then the chunk's maximum and the running (max, sum)
+        auto row_chunk = [&](float (&v)[32], int c) {
+          if (!(full_quarter && row_ok)) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) cm[i & 3] = fmaxf(cm[i & 3], v[i]);
-            } else {
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                v[i] = (row_ok && key0 + c + i <= p) ? v[i] : -INFINITY;
-                cm[i & 3] = fmaxf(cm[i & 3], v[i]);
-              }
-            }
-            // the scale is positive, so max(v) * scale is the max of the scaled logits
-            const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])) * sc);
-            if (mn != -INFINITY) {
-              // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
-              float s0, s1, s2, s3;
-              if (SELKV_PACKED) {
-                const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
-                uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
-#pragma unroll
-                for (int i = 0; i < 32; i += 4) {
-                  float x0, x1, x2, x3;
-                  unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
-                  unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
-                  s01 = fadd2(s01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
-                  s23 = fadd2(s23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
-                }
-                unpack_f2(s01, s0, s1);
-                unpack_f2(s23, s2, s3);
-              } else {
-                float s4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_approx(fmaf(v[i], sc, -mn));
-                s0 = s4[0];
-                s1 = s4[1];
-                s2 = s4[2];
-                s3 = s4[3];
-              }
-              l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
-              m_run = mn;
-            }
+            for (int i = 0; i < 32; ++i) v[i] = (row_ok && key0 + c + i <= p) ? v[i] : -INFINITY;
           }
+          // the scale is positive, so max(v) * scale is the max of the scaled logits
+          const float mn = fmaxf(m_run, max32(v) * sc);
+          if (mn != -INFINITY) {
+            // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
+            const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
+            uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) {
+              float x0, x1, x2, x3;
+              unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
+              unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
+              s01 = fadd2(s01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
+              s23 = fadd2(s23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
+            }
+            float s0, s1, s2, s3;
+            unpack_f2(s01, s0, s1);
+            unpack_f2(s23, s2, s3);
+            l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
+            m_run = mn;
+          }
+        };
+        if (ok) {
+          // the second chunk's load is in flight while the first is reduced
+          const uint32_t ta = tmem + lane_base + buf * 256 + part * 64;
+          float va[32], vb[32];
+          tmem_ld32_issue(ta, va);
+          tmem_wait_ld32(va);
+          tmem_ld32_issue(ta + 32, vb);
+          row_chunk(va, 0);
+          tmem_wait_ld32(vb);
+          row_chunk(vb, 32);
         }
         tc_fence_before();
         __syncwarp();
@@ -318,29 +315,31 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
       }
     } else {
       const int klane = q * 32 + lane;   // key owned by this thread within the tile
-      const int r_lo = part * 64, r_hi = min(R, r_lo + 64);
+      int u = 0;                         // accumulator use, as counted by the MMA thread
       for (int t = 0; t < nt; ++t) {
-        const int buf = t & 1;
-        const bool ok = warp_wait(&tfull[buf], (t >> 1) & 1);
-        tc_fence_after();
         const int j = (t_begin + t) * kKeys + klane;
         const int jrel = j - (n - a.W);  // > 0: only rows with (r mod W) >= jrel see key j
-        float acc = 0.f;
         // every key of this warp is seen by every row: the whole tile is unmasked
         const bool unmasked = (t_begin + t) * kKeys + q * 32 + 31 <= n - a.W;
-        if (ok && SELKV_P2_PIPE && SELKV_PACKED && r_hi - r_lo == 64 && unmasked) {
-          acc = colsum64(tmem + lane_base + buf * 256 + r_lo, smem_u32(rneg + r_lo), sc);
-        } else if (ok) {
+        float acc = 0.f;
+        for (int ph = 0; ph < HALVES; ++ph, ++u) {
+          const int buf = u & 1;
+          const bool ok = warp_wait(&tfull[buf], (u >> 1) & 1);
+          tc_fence_after();
+          // this part's 64 rows of the half: accumulator columns from c0, rows from r_lo
+          const int c0 = part * 64, r_lo = ph * 256 + c0, r_hi = min(R, r_lo + 64);
+          const uint32_t tcol = tmem + lane_base + buf * 256 + c0;
+          if (ok && SELKV_P2_PIPE && r_hi - r_lo == 64 && unmasked) {
+            acc += colsum64(tcol, smem_u32(rneg + r_lo), sc);
+          } else if (ok) {
 #pragma unroll 1
-          for (int c = r_lo; c < r_hi; c += 32) {
-            float v[32];
-            tmem_ld32(tmem + lane_base + buf * 256 + c, v);
-            const int cnt = min(32, r_hi - c);
-            if (jrel <= 0 && cnt == 32) {
-              // sum over rows of 2^(v sc - M_r - log2(G Z_r)), pairs of rows packed; four
-              // interleaved partial sums as (0,1) and (2,3)
-              float s0, s1, s2, s3;
-              if (SELKV_PACKED) {
+            for (int c = r_lo; c < r_hi; c += 32) {
+              float v[32];
+              tmem_ld32(tcol + (c - r_lo), v);
+              const int cnt = min(32, r_hi - c);
+              if (jrel <= 0 && cnt == 32) {
+                // sum over rows of 2^(v sc - M_r - log2(G Z_r)), pairs of rows packed; four
+                // interleaved partial sums as (0,1) and (2,3)
                 const uint64_t sc2 = pack_f2(sc, sc);
                 uint64_t a01 = pack_f2(0.f, 0.f), a23 = a01;
 #pragma unroll
@@ -352,39 +351,26 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
                   a01 = fadd2(a01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
                   a23 = fadd2(a23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
                 }
+                float s0, s1, s2, s3;
                 unpack_f2(a01, s0, s1);
                 unpack_f2(a23, s2, s3);
+                acc += (s0 + s1) + (s2 + s3);
               } else {
-                float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                for (int i = 0; i < 32; i += 4) {
-                  const float4 nm = *reinterpret_cast<const float4*>(&rneg[c + i]);
-                  s4[0] += ex2_approx(fmaf(v[i], sc, nm.x));
-                  s4[1] += ex2_approx(fmaf(v[i + 1], sc, nm.y));
-                  s4[2] += ex2_approx(fmaf(v[i + 2], sc, nm.z));
-                  s4[3] += ex2_approx(fmaf(v[i + 3], sc, nm.w));
-                }
-                s0 = s4[0];
-                s1 = s4[1];
-                s2 = s4[2];
-                s3 = s4[3];
+                for (int i = 0; i < 32; ++i)
+                  if (i < cnt && (jrel <= 0 || (c + i) % a.W >= jrel))
+                    acc += ex2_approx(fmaf(v[i], sc, rneg[c + i]));
               }
-              acc += (s0 + s1) + (s2 + s3);
-            } else {
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (i < cnt && (jrel <= 0 || (c + i) % a.W >= jrel))
-                  acc += ex2_approx(fmaf(v[i], sc, rneg[c + i]));
             }
           }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty[buf]);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[buf]);
-        // the four row quarters' column sums of key j meet in shared memory (one buffer per
-        // accumulator, so a tile's sums are read before the buffer comes round again); the
-        // warp of quarter 0 adds them in quarter order and writes a_j
-        float* cs = colpart + buf * 512;  // [4][128]
+        // the four row quarters' column sums of key j meet in shared memory (two buffers,
+        // alternating by tile, so a tile's sums are read before its buffer comes round again);
+        // the warp of quarter 0 adds them in quarter order and writes a_j
+        float* cs = colpart + (t & 1) * 512;  // [4][128]
         cs[part * 128 + klane] = acc;
         named_bar_sync(1 + q, 4 * 32);
         if (part == 0 && j < n)
@@ -410,10 +396,10 @@ int splits_for(int B, int Hkv, int n_cap, int num_sms, int row_parts, int keys) 
   return s < 1 ? 1 : s;
 }
 
-template <int D>
+template <int D, int HALVES>
 cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st, int passes) {
   using C1 = SCfg<D, 1>;
-  using C2 = SCfg<D, 2>;
+  using C2 = SCfg<D, 2, HALVES>;
   CUtensorMap tq, tk1, tk2;
   if (!encode_rows_bf16(&tq, a.Q, (uint64_t)a.B * a.Hq * a.W, D, 128) ||
       !encode_rows_bf16(&tk1, a.K, (uint64_t)a.B * a.Hkv * a.n_cap, D, C1::kKeys) ||
@@ -422,10 +408,10 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st, int passes) {
   const int MT = (a.R + 127) / 128;
   const dim3 grid1(a.nchunks * MT, a.Hkv, a.B);
   const dim3 grid2(splits_for(a.B, a.Hkv, a.n_cap, kPlanSMs, 1, C2::kKeys), a.Hkv, a.B);
-  auto k1 = score_tc_kernel<D, 1>;
-  auto k2 = score_tc_kernel<D, 2>;
-  cudaError_t e = set_smem_once<score_tc_kernel<D, 1>>(C1::kSmem);
-  if (e == cudaSuccess) e = set_smem_once<score_tc_kernel<D, 2>>(C2::kSmem);
+  auto k1 = score_tc_kernel<D, 1, 1>;
+  auto k2 = score_tc_kernel<D, 2, HALVES>;
+  cudaError_t e = set_smem_once<score_tc_kernel<D, 1, 1>>(C1::kSmem);
+  if (e == cudaSuccess) e = set_smem_once<score_tc_kernel<D, 2, HALVES>>(C2::kSmem);
   if (e != cudaSuccess) return e;
   if (passes & kScoreRowstats) {
     k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
@@ -438,14 +424,17 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st, int passes) {
 
 }  // namespace
 
-bool score_uses_tc(int dtype, int D, int R) { return dtype == SELKV_BF16 && (D == 64 || D == 128) && R >= 1 && R <= 256; }
+// The window rows of a KV group, R = G W, go to the tensor cores up to 512 (two 256-row halves
+// in the column-sum pass); wider groups take the CUDA-core path.
+bool score_uses_tc(int dtype, int D, int R) { return dtype == SELKV_BF16 && (D == 64 || D == 128) && R >= 1 && R <= 512; }
 
 int score_tc_splits(int B, int Hkv, int n_cap, int R, int num_sms) {
   return splits_for(B, Hkv, n_cap, num_sms, (R + 127) / 128, SCfg<128, 1>::kKeys);
 }
 
 cudaError_t launch_score_tc(const CompressArgs& a, cudaStream_t st, int passes) {
-  return a.D == 128 ? launch_tc_t<128>(a, st, passes) : launch_tc_t<64>(a, st, passes);
+  if (a.R > 256) return a.D == 128 ? launch_tc_t<128, 2>(a, st, passes) : launch_tc_t<64, 2>(a, st, passes);
+  return a.D == 128 ? launch_tc_t<128, 1>(a, st, passes) : launch_tc_t<64, 1>(a, st, passes);
 }
 
 }  // namespace selkv

@@ -82,6 +82,14 @@ WORKLOADS = {
                              decode_steps=256, **_LLAMA),
     "long_100k": Workload(name="long_100k", batch=1, n=100000, layers=32, rho=0.25,
                           decode_steps=256, **_LLAMA),
+    # a wider GQA group (Llama-3-70B attention shape: 64 query heads over 8 KV heads, G = 8),
+    # one layer at 16k: G W = 512 window rows per KV head
+    "llama70b_layer": Workload(name="llama70b_layer", batch=1, n=16384, layers=1, rho=0.25,
+                               decode_steps=128, **dict(_LLAMA, num_q_heads=64)),
+    # the same G = 8 shape over 32 layers at 100k context (the long-context setting of the paper
+    # with the wider group)
+    "llama70b_100k": Workload(name="llama70b_100k", batch=1, n=100000, layers=32, rho=0.25,
+                              decode_steps=256, **dict(_LLAMA, num_q_heads=64)),
     # the paper's MHA setting (LongChat-7B-shaped: 32 query heads = 32 KV heads, 31,500-token
     # inputs, W = 32), for the per-head selection mode
     "longchat_mha_31k": Workload(name="longchat_mha_31k", batch=1, n=31500, layers=32, rho=0.25,

@@ -67,11 +67,14 @@ def test_reference_arm_prints_on_rank_0_only():
 
 def test_decode_bytes_per_launch_by_hand():
     """One launch of the 100k workload at token t: 8 KV heads x (25,000 + t + 1) rows of
-    K_c, V_c (256 bytes each, bf16 d = 128) and a 4-byte bias, plus q and out (32 heads x 256
-    bytes each) and the appended k and v (8 heads x 256 bytes each)."""
+    K_c, V_c (256 bytes each, bf16 d = 128), a 4-byte bias per position (shared by the KV
+    heads; per KV head in the per-head mode), plus q and out (32 heads x 256 bytes each) and the
+    appended k and v (8 heads x 256 bytes each)."""
     import synth
     wl = synth.WORKLOADS["long_100k"]
     T = 256
-    per_token = [8 * (25000 + t + 1) * 516 + 2 * 32 * 256 + 2 * 8 * 256 for t in range(T)]
+    per_token = [(25000 + t + 1) * (8 * 512 + 4) + 2 * 32 * 256 + 2 * 8 * 256 for t in range(T)]
     assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(sum(per_token) / T)
-    assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(103750928.0)
+    assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(103047330.0)
+    per_head = [8 * (25000 + t + 1) * 516 + 2 * 32 * 256 + 2 * 8 * 256 for t in range(T)]
+    assert bench.decode_bytes_per_launch(wl, [100000], T, per_head=True) == pytest.approx(sum(per_head) / T)

@@ -127,3 +127,17 @@ def test_long_100k_layer_rope_shifts():
     assert kept[-1] - (m - 1) > 50000
     for kv in range(wl.num_kv_heads):
         check_keys(host["K_c"][0, kv, :m], x["K"][0, kv][kept].astype(np.float64), kept, p, wl.dtype)
+
+
+def test_llama70b_layer_wide_group():
+    """One layer of the G = 8 workload (64 query heads over 8 KV heads, 16k, W = 64: G W = 512
+    window rows per KV head, scored on the tensor cores in two row halves): stage-by-stage
+    parity and decode."""
+    wl = synth.WORKLOADS["llama70b_layer"]
+    x = synth.gen_layer(wl, 0, threads=16)
+    p = O.Params()
+    cache, host, _ = run_compress(wl, x, p, extra=3)
+    st = Stats()
+    check_sequence(wl, x, host, 0, p, stats=st)
+    check_properties(wl, x, host, p)
+    _decode_sampled(wl, cache, 0, [0], steps=2)

@@ -33,6 +33,15 @@ SMALL = {
                                                         num_kv_heads=4, obs_window=40, seed=12),
     "fp32_d128": synth.WORKLOADS["tiny"].with_(name="fp32_d128", head_dim=128, n=1500, batch=2,
                                                ragged=(0.6, 1.0), seed=13),
+    # wide GQA groups: G W = 512 rows (two 256-row halves in the column-sum pass) and 384 rows
+    # (a half of 128), d 64
+    "bf16_g8_w64": synth.WORKLOADS["llama_layer"].with_(name="bf16_g8_w64", batch=2, n=2900,
+                                                        num_q_heads=16, num_kv_heads=2,
+                                                        ragged=(0.6, 1.0), seed=14),
+    "bf16_g16_w24_d64": synth.WORKLOADS["llama_layer"].with_(name="bf16_g16_w24_d64", batch=2, n=2100,
+                                                             head_dim=64, num_q_heads=32,
+                                                             num_kv_heads=2, obs_window=24,
+                                                             ragged=(0.7, 1.0), seed=15),
 }
 
 
@@ -215,7 +224,7 @@ def _decode_case(wl, layer, steps, use_bias=True, p=None):
     return worst
 
 
-@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4", "fp32_d128"])
+@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4", "fp32_d128", "bf16_g8_w64"])
 def test_decode_parity_small(name):
     worst = _decode_case(SMALL[name], 0, steps=4)
     print(name, "decode worst max/mean abs", worst)
@@ -567,7 +576,7 @@ def test_layer_average_one_layer_is_identity():
 
 
 # ---------------------------------------------------------------- scoring stage on its own
-@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4"])
+@pytest.mark.parametrize("name", ["tiny", "bf16_ragged", "bf16_d64_g4", "bf16_g8_w64", "bf16_g16_w24_d64"])
 def test_score_entry_point(name):
     """selkv_score (Sec. 3.1 re-pass, Eq. 1's attention sums): a within ATTN_RTOL of the
     oracle; bitwise the `attn` of selkv_compress; the two passes run as separate calls
