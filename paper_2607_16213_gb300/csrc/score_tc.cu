@@ -113,6 +113,10 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   uint64_t* done = qbar + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  // pass 2: per lane quarter and column-sum buffer, "the other three parts' sums are in" and
+  // "part 0 has read them"
+  uint64_t* cs_full = reinterpret_cast<uint64_t*>(misc + 128);  // [4][2]
+  uint64_t* cs_empty = cs_full + 8;                              // [4][2]
   float* rneg = reinterpret_cast<float*>(misc + 256);               // pass 2: -(M + log2(G Z)) per row
   float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [4][128] float2; pass 2: [2][4][128]
 
@@ -145,6 +149,10 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
     }
     mbar_init(qbar, 1);
     mbar_init(done, 1);
+    for (int i = 0; i < 8; ++i) {
+      mbar_init(&cs_full[i], 3 * 32);
+      mbar_init(&cs_empty[i], 32);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -253,44 +261,46 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         tc_fence_after();
         const int key0 = (t_begin + t) * kKeys + part * 64;
         const bool full_quarter = key0 + 63 <= n - a.W;  // every row sees every key of the quarter
-        // one 32-column chunk of this thread's row: masked where the row does not see the key
-        // (or the row does not exist), then the chunk's maximum and the running (max, sum)
-        auto row_chunk = [&](float (&v)[32], int c) {
-          if (!(full_quarter && row_ok)) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = (row_ok && key0 + c + i <= p) ? v[i] : -INFINITY;
-          }
-          // the scale is positive, so max(v) * scale is the max of the scaled logits
-          const float mn = fmaxf(m_run, max32(v) * sc);
-          if (mn != -INFINITY) {
-            // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
-            const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
-            uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
-#pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              float x0, x1, x2, x3;
-              unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
-              unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
-              s01 = fadd2(s01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
-              s23 = fadd2(s23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
-            }
-            float s0, s1, s2, s3;
-            unpack_f2(s01, s0, s1);
-            unpack_f2(s23, s2, s3);
-            l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
-            m_run = mn;
-          }
-        };
+        // (pass 1 reads the accumulator 32 columns at a time, each load waited for before its
+        // arithmetic: pipelined loads measured slower here, 16-column ones because the running
+        // max then needs a correction every 16 keys, 32-column ones by half a microsecond)
         if (ok) {
-          // the second chunk's load is in flight while the first is reduced
-          const uint32_t ta = tmem + lane_base + buf * 256 + part * 64;
-          float va[32], vb[32];
-          tmem_ld32_issue(ta, va);
-          tmem_wait_ld32(va);
-          tmem_ld32_issue(ta + 32, vb);
-          row_chunk(va, 0);
-          tmem_wait_ld32(vb);
-          row_chunk(vb, 32);
+#pragma unroll 1
+          for (int c = 0; c < 64; c += 32) {
+            float v[32];
+            tmem_ld32(tmem + lane_base + buf * 256 + part * 64 + c, v);
+            float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (full_quarter && row_ok) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) cm[i & 3] = fmaxf(cm[i & 3], v[i]);
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                v[i] = (row_ok && key0 + c + i <= p) ? v[i] : -INFINITY;
+                cm[i & 3] = fmaxf(cm[i & 3], v[i]);
+              }
+            }
+            // the scale is positive, so max(v) * scale is the max of the scaled logits
+            const float mn = fmaxf(m_run, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])) * sc);
+            if (mn != -INFINITY) {
+              // 2^(v sc - mn), pairs packed; sums in four interleaved lanes as (0,1) and (2,3)
+              const uint64_t sc2 = pack_f2(sc, sc), nm2 = pack_f2(-mn, -mn);
+              uint64_t s01 = pack_f2(0.f, 0.f), s23 = s01;
+#pragma unroll
+              for (int i = 0; i < 32; i += 4) {
+                float x0, x1, x2, x3;
+                unpack_f2(ffma2(pack_f2(v[i], v[i + 1]), sc2, nm2), x0, x1);
+                unpack_f2(ffma2(pack_f2(v[i + 2], v[i + 3]), sc2, nm2), x2, x3);
+                s01 = fadd2(s01, pack_f2(ex2_approx(x0), ex2_approx(x1)));
+                s23 = fadd2(s23, pack_f2(ex2_approx(x2), ex2_approx(x3)));
+              }
+              float s0, s1, s2, s3;
+              unpack_f2(s01, s0, s1);
+              unpack_f2(s23, s2, s3);
+              l_run = l_run * ex2_approx(m_run - mn) + ((s0 + s1) + (s2 + s3));
+              m_run = mn;
+            }
+          }
         }
         tc_fence_before();
         __syncwarp();
@@ -367,14 +377,31 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty[buf]);
         }
-        // the four row quarters' column sums of key j meet in shared memory (two buffers,
-        // alternating by tile, so a tile's sums are read before its buffer comes round again);
-        // the warp of quarter 0 adds them in quarter order and writes a_j
-        float* cs = colpart + (t & 1) * 512;  // [4][128]
-        cs[part * 128 + klane] = acc;
-        named_bar_sync(1 + q, 4 * 32);
-        if (part == 0 && j < n)
-          a.attn[bk * a.n_cap + j] = ((cs[klane] + cs[128 + klane]) + cs[256 + klane]) + cs[384 + klane];
+        // The four row quarters' column sums of key j meet in shared memory (two buffers,
+        // alternating by tile): parts 1-3 leave theirs and go on, part 0 adds them to its own in
+        // quarter order and writes a_j.  A part reuses a buffer only once part 0 has read it.
+        const int cb = t & 1;
+        float* cs = colpart + cb * 512;  // [4][128]
+        uint64_t* cfull = &cs_full[q * 2 + cb];
+        uint64_t* cempty = &cs_empty[q * 2 + cb];
+        // bounded wait of every lane (each lane acquires what it then reads or overwrites)
+        auto lane_wait = [&](uint64_t* bar, uint32_t parity) {
+          if (*abort_flag) return;
+          if (!mbar_wait(bar, parity)) {
+            *abort_flag = 1;
+            raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+          }
+        };
+        if (part > 0) {
+          if (t >= 2) lane_wait(cempty, ((t >> 1) - 1) & 1);
+          cs[part * 128 + klane] = acc;
+          mbar_arrive(cfull);
+        } else {
+          lane_wait(cfull, (t >> 1) & 1);
+          const float sum = ((acc + cs[128 + klane]) + cs[256 + klane]) + cs[384 + klane];
+          mbar_arrive(cempty);
+          if (j < n) a.attn[bk * a.n_cap + j] = sum;
+        }
       }
     }
   }
