@@ -30,10 +30,21 @@
 namespace selkv {
 namespace {
 
-constexpr int kEpiWarps = 16;
-constexpr int kProducerWarp = 16, kMmaWarp = 17;
-constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr uint32_t kTmemCols = 512;  // two accumulators of up to 256 fp32 columns
+#ifndef SELKV_P1_KEYS
+#define SELKV_P1_KEYS 256  // pass 1: keys per tile (the MMA's N), a multiple of 32
+#endif
+#ifndef SELKV_P1_CPW
+#define SELKV_P1_CPW 2     // pass 1: 32-column accumulator chunks per epilogue warp and tile
+#endif
+// Epilogue warps: pass 1 splits a tile's keys over the warps of each TMEM lane quarter (32
+// columns x SELKV_P1_CPW per warp), pass 2 splits the rows over four warps per lane quarter.
+// A TMA producer warp and an MMA warp follow them.
+constexpr int kP1Parts = SELKV_P1_KEYS / (32 * SELKV_P1_CPW);
+static_assert(kP1Parts * 32 * SELKV_P1_CPW == SELKV_P1_KEYS && kP1Parts >= 1, "pass-1 tile split");
+static_assert(4 * kP1Parts + 2 <= 32 && SELKV_P1_KEYS <= 256, "pass-1 warps per CTA");
+__host__ __device__ constexpr int epi_warps(int pass) { return pass == 1 ? 4 * kP1Parts : 16; }
+__host__ __device__ constexpr int cta_threads(int pass) { return (epi_warps(pass) + 2) * 32; }
 
 #ifndef SELKV_P2_PIPE
 #define SELKV_P2_PIPE 1   // pass 2: pipelined 16-column TMEM loads on full, unmasked tiles
@@ -82,22 +93,25 @@ __device__ __forceinline__ float colsum64(uint32_t taddr, uint32_t rn, float sc)
 // for the 512 staged rows.
 template <int D, int PASS, int HALVES = 1>
 struct SCfg {
-  static constexpr int kKeys = PASS == 1 ? 256 : 128;                  // keys per tile
+  static constexpr int kKeys = PASS == 1 ? SELKV_P1_KEYS : 128;        // keys per tile
   static constexpr int kStages = PASS == 1 ? 2 : (HALVES == 2 ? 2 : 4);  // K tiles in flight
   static constexpr int kRows = PASS == 1 ? 128 : 256 * HALVES;          // Q rows staged per CTA
   static constexpr int kBoxes = D / 64;                  // 128-byte-wide boxes per row
   static constexpr int kKTile = kKeys * D * 2;           // one K tile
   static constexpr int kQBytes = kRows * D * 2;
   static constexpr int kRing = kStages * kKTile;
-  static constexpr int kMisc = 256 + 256 * 8 + 2 * 4 * 128 * 4;
+  // barriers | -(M + log2(G Z)) of up to 512 rows | pass 1: [parts][128] float2, pass 2: [2][4][128] float
+  static constexpr int kMisc = 256 + 256 * 8 + (kP1Parts * 128 * 8 > 4096 ? kP1Parts * 128 * 8 : 4096);
   static constexpr int kSmem = 1024 + kQBytes + kRing + kMisc;
 };
 
 template <int D, int PASS, int HALVES>
-__global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
-                                                                const __grid_constant__ CUtensorMap tmK,
-                                                                CompressArgs a) {
+__global__ __launch_bounds__(cta_threads(PASS), 1) void score_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                                                                        const __grid_constant__ CUtensorMap tmK,
+                                                                        CompressArgs a) {
   using C = SCfg<D, PASS, HALVES>;
+  constexpr int kEpiWarps = epi_warps(PASS);
+  constexpr int kProducerWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
   constexpr int kKeys = C::kKeys, kStages = C::kStages;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
@@ -118,7 +132,7 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
   uint64_t* cs_full = reinterpret_cast<uint64_t*>(misc + 128);  // [4][2]
   uint64_t* cs_empty = cs_full + 8;                              // [4][2]
   float* rneg = reinterpret_cast<float*>(misc + 256);               // pass 2: -(M + log2(G Z)) per row
-  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [4][128] float2; pass 2: [2][4][128]
+  float* colpart = reinterpret_cast<float*>(misc + 256 + 256 * 8);  // pass 1: [parts][128] float2; pass 2: [2][4][128]
 
   const int kv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -259,16 +273,17 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         const int buf = t & 1;
         const bool ok = warp_wait(&tfull[buf], (t >> 1) & 1);
         tc_fence_after();
-        const int key0 = (t_begin + t) * kKeys + part * 64;
-        const bool full_quarter = key0 + 63 <= n - a.W;  // every row sees every key of the quarter
+        constexpr int kCols = 32 * SELKV_P1_CPW;           // this warp's keys of the tile
+        const int key0 = (t_begin + t) * kKeys + part * kCols;
+        const bool full_quarter = key0 + kCols - 1 <= n - a.W;  // every row sees every key of the part
         // (pass 1 reads the accumulator 32 columns at a time, each load waited for before its
         // arithmetic: pipelined loads measured slower here, 16-column ones because the running
         // max then needs a correction every 16 keys, 32-column ones by half a microsecond)
         if (ok) {
 #pragma unroll 1
-          for (int c = 0; c < 64; c += 32) {
+          for (int c = 0; c < kCols; c += 32) {
             float v[32];
-            tmem_ld32(tmem + lane_base + buf * 256 + part * 64 + c, v);
+            tmem_ld32(tmem + lane_base + buf * 256 + part * kCols + c, v);
             float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             if (full_quarter && row_ok) {
 #pragma unroll
@@ -306,20 +321,22 @@ __global__ __launch_bounds__(kThreads, 1) void score_tc_kernel(const __grid_cons
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
       }
-      // fold the four key quarters of each row in quarter order (quarters 1-3 via shared memory)
-      float2* st4 = reinterpret_cast<float2*>(colpart);  // [4][128]
+      // fold the key parts of each row in part order (parts 1.. via shared memory)
+      float2* st4 = reinterpret_cast<float2*>(colpart);  // [parts][128]
       if (part > 0) st4[part * 128 + q * 32 + lane] = make_float2(m_run, l_run);
       named_bar_sync(1, kEpiWarps * 32);
       if (part == 0 && row_ok) {
-        float2 o[4];
+        float2 o[kP1Parts];
         o[0] = make_float2(m_run, l_run);
 #pragma unroll
-        for (int k = 1; k < 4; ++k) o[k] = st4[k * 128 + q * 32 + lane];
-        const float M = fmaxf(fmaxf(o[0].x, o[1].x), fmaxf(o[2].x, o[3].x));
+        for (int k = 1; k < kP1Parts; ++k) o[k] = st4[k * 128 + q * 32 + lane];
+        float M = o[0].x;
+#pragma unroll
+        for (int k = 1; k < kP1Parts; ++k) M = fmaxf(M, o[k].x);
         float L = 0.f;
         if (M != -INFINITY) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k) L += o[k].y * ex2_approx(o[k].x - M);
+          for (int k = 0; k < kP1Parts; ++k) L += o[k].y * ex2_approx(o[k].x - M);
         }
         a.rowpart[(bk * a.nchunks + split) * R + r] = make_float2(M, L);
       }
@@ -441,11 +458,11 @@ cudaError_t launch_tc_t(const CompressArgs& a, cudaStream_t st, int passes) {
   if (e == cudaSuccess) e = set_smem_once<score_tc_kernel<D, 2, HALVES>>(C2::kSmem);
   if (e != cudaSuccess) return e;
   if (passes & kScoreRowstats) {
-    k1<<<grid1, kThreads, C1::kSmem, st>>>(tq, tk1, a);
+    k1<<<grid1, cta_threads(1), C1::kSmem, st>>>(tq, tk1, a);
     e = launch_rowstat_reduce(a, st);
     if (e != cudaSuccess) return e;
   }
-  if (passes & kScoreColsums) k2<<<grid2, kThreads, C2::kSmem, st>>>(tq, tk2, a);
+  if (passes & kScoreColsums) k2<<<grid2, cta_threads(2), C2::kSmem, st>>>(tq, tk2, a);
   return cudaGetLastError();
 }
 
