@@ -276,7 +276,8 @@ class Layered:
         if pinned_host:
             es = 2 if wl.dtype == "bf16" else 4
             per_layer = (2 * B * Hkv * wl.n * d + B * Hq * W * d) * es + 3 * 256
-            decode = wl.decode_steps * wl.layers * B * (Hq + 2 * Hkv) * d * es + wl.layers * B * Hq * d * es + 4 * 256
+            # every token's q, k_new, v_new and every token's outputs
+            decode = wl.decode_steps * wl.layers * B * (2 * Hq + 2 * Hkv) * d * es + 4 * 256
             self.arena = HostArena(torch, wl.layers * per_layer + decode)
         threads = os.cpu_count() or 1
         for layer in range(wl.layers):
@@ -609,94 +610,118 @@ def measure_scoring(L: Layered, S, api, torch, stream, dev, peaks, peak_src, rep
 
 
 def run_e2e(L: Layered, S, api, torch, params, stream, dev, steps: int, warmup: int):
-    """The step through the public API with pinned host inputs, as a serving loop runs it:
-    every layer's K, V and Q_obs are copied from host to device, every layer is compressed,
-    then per token q / k_new / v_new are copied in, every layer is decoded and the token's
-    outputs are read back.  Steps are double-buffered: the input copies of step i + 1 (on a
-    copy stream, into the other of two device input sets) run while step i decodes, and
-    layer l of a step compresses once its copies have landed.  The token loop (its copies and
-    decode calls) is captured once as a CUDA graph and replayed each step; the compression
-    calls are issued eagerly.  Every timed step moves its full input bytes across the link
-    inside the timed region (the copies for the first timed step run during the last warm-up
-    step, those issued during the last timed step are waited for before the clock stops).
-    On a GB300 (Grace host) a 13 GB host-to-device pass copies at ~210 GB/s back to back with
-    other copies but at 25-70 GB/s after or during the decode's HBM streaming, which sets
-    this number (and makes it vary from run to run; more copy streams did not help).  Host
-    buffers come from a HostArena."""
+    """The step through the public API with its inputs in pinned host memory: every layer's
+    K, V and Q_obs and every token's q, k_new and v_new are copied from host to device, every
+    layer is compressed, the tokens are decoded (each token every layer, appending), and every
+    token's outputs are read back to host memory.  Steps are double-buffered: the input
+    copies of step i + 1 (on a copy stream, into the other of two device input sets) run while
+    step i computes; layer l of a step compresses once its copies have landed and the token
+    loop starts once the token inputs have.  The token loop (the decode calls only) is
+    captured once per input set as a CUDA graph; the compression calls are issued eagerly; the
+    outputs go back on a third stream once the step's token loop is done.  Every timed step
+    moves its full input and output bytes across the link inside the timed region (the input
+    copies for the first timed step run during the last warm-up step; those issued during the
+    last timed step, and the last outputs, are waited for before the clock stops).  The
+    per-token inputs travel with the step's other inputs rather than token by token: a small
+    copy queued behind the layers' bulk copies on the host link would stall its token for the
+    length of the bulk transfer.  Host buffers come from a HostArena."""
     wl = L.wl
     sp = stream.cuda_stream
     hq = L.arena.take(L.dq)
     hk = L.arena.take(L.dk)
     hv = L.arena.take(L.dv)
-    hout = L.arena.take(torch.empty(L.out.shape[1:], dtype=L.out.dtype))
-    dq = torch.empty_like(L.dq[0])
-    dk = torch.empty_like(L.dk[0])
-    dv = torch.empty_like(L.dv[0])
+    hout = L.arena.take(torch.empty(L.out.shape, dtype=L.out.dtype))
     h2d = sum(t.numel() * t.element_size() for trip in L.host for t in trip) + \
-        L.T * (dq.numel() + dk.numel() + dv.numel()) * dq.element_size()
-    d2h = L.T * hout.numel() * hout.element_size()
+        sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+    d2h = hout.numel() * hout.element_size()
 
     # two device input sets: the resident one and a second of the same shapes
-    sets = [(L.K, L.V, L.Q),
+    sets = [(L.K, L.V, L.Q, L.dq, L.dk, L.dv),
             ([torch.empty_like(x) for x in L.K], [torch.empty_like(x) for x in L.V],
-             [torch.empty_like(x) for x in L.Q])]
+             [torch.empty_like(x) for x in L.Q], torch.empty_like(L.dq), torch.empty_like(L.dk),
+             torch.empty_like(L.dv))]
     copy_stream = torch.cuda.Stream(device=dev)
+    out_stream = torch.cuda.Stream(device=dev)
     arrived = [[torch.cuda.Event() for _ in range(wl.layers)] for _ in range(2)]
-    consumed = [torch.cuda.Event() for _ in range(2)]  # last compression that read the set
-
-    def tokens():
-        for t in range(L.T):
-            dq.copy_(hq[t], non_blocking=True)
-            dk.copy_(hk[t], non_blocking=True)
-            dv.copy_(hv[t], non_blocking=True)
-            for layer in range(wl.layers):
-                api.decode(L.caches[layer], dq[layer], dk[layer], dv[layer], out=L.out[0, layer],
-                           workspace=L.dws, stream=sp)
-            hout.copy_(L.out[0], non_blocking=True)
-
-    g_tok = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_tok, stream=stream):
-        tokens()
+    tok_arrived = [torch.cuda.Event() for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]  # last kernel of a step that read the set
+    decoded = torch.cuda.Event()
     torch.cuda.synchronize()
 
+    def tokens(si):
+        _, _, _, dq, dk, dv = sets[si]
+        for t in range(L.T):
+            for layer in range(wl.layers):
+                api.decode(L.caches[layer], dq[t, layer], dk[t, layer], dv[t, layer], out=L.out[t, layer],
+                           workspace=L.dws, stream=sp)
+
+    g_tok = []
+    for si in range(2):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            tokens(si)
+        g_tok.append(g)
+    torch.cuda.synchronize()
+
+    copy_marks = []   # (start, end) events around each step's input copies
+
     def copy_inputs(si, after=None):
-        """Enqueue the host-to-device copies of every layer into input set si."""
-        Ks, Vs, Qs = sets[si]
+        """Enqueue the host-to-device copies of a step's inputs into input set si."""
+        Ks, Vs, Qs, dq, dk, dv = sets[si]
         with torch.cuda.stream(copy_stream):
             if after is not None:
                 copy_stream.wait_event(after)
+            m0, m1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            m0.record(copy_stream)
             for layer in range(wl.layers):
                 hK, hV, hQ = L.host[layer]
                 Ks[layer].copy_(hK, non_blocking=True)
                 Vs[layer].copy_(hV, non_blocking=True)
                 Qs[layer].copy_(hQ, non_blocking=True)
                 arrived[si][layer].record(copy_stream)
+            dq.copy_(hq, non_blocking=True)
+            dk.copy_(hk, non_blocking=True)
+            dv.copy_(hv, non_blocking=True)
+            tok_arrived[si].record(copy_stream)
+            m1.record(copy_stream)
+            copy_marks.append((m0, m1))
 
     def one(i):
         si = i % 2
         with torch.cuda.stream(stream):
-            compress_layers(L, S, params, sp, inputs=sets[si],
+            compress_layers(L, S, params, sp, inputs=sets[si][:3],
                             before_layer=lambda layer, st: st.wait_event(arrived[si][layer]))
+            stream.wait_event(tok_arrived[si])
+            stream.wait_event(decoded)     # the previous step's outputs have been read back
+            g_tok[si].replay()
             consumed[si].record(stream)
-        # the next step's inputs go to the other set once its last compression is done
+        # the step's outputs go back once its tokens are decoded
+        with torch.cuda.stream(out_stream):
+            out_stream.wait_event(consumed[si])
+            hout.copy_(L.out, non_blocking=True)
+            decoded.record(out_stream)
+        # the next step's inputs go to the other set once the step that last read it is done
         copy_inputs(1 - si, after=consumed[1 - si] if i > 0 else None)
-        with torch.cuda.stream(stream):
-            g_tok.replay()
 
     copy_inputs(0)
     for i in range(warmup):
         one(i)
-    stream.synchronize()
     torch.cuda.synchronize()
+    first = len(copy_marks)
     t0 = time.perf_counter()
     for i in range(warmup, warmup + steps):
         one(i)
     stream.synchronize()
+    out_stream.synchronize()
     copy_stream.synchronize()
     dt = (time.perf_counter() - t0) / steps
+    bulk = sum(t.numel() * t.element_size() for trip in L.host for t in trip) + \
+        sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+    copy_ms = [a.elapsed_time(b) for a, b in copy_marks[first:]]
     return {"value": wl.batch * L.T / dt, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": dt * 1e3, "steps": steps, "warmup": warmup,
-            "pipelined": "the next step's input copies overlap this step's decode"}
+            "pipelined": "the next step's input copies overlap this step's compute",
+            "input_copy_gbs": [round(bulk / (ms * 1e-3) / 1e9, 1) for ms in copy_ms]}
 
 
 # ------------------------------------------------------------------------------ serving sweep
