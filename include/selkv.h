@@ -292,7 +292,17 @@ SELKV_API selkv_status selkv_layer_average_bias(const selkv_shape* shape, const 
  * k_new, v_new  [B][Hkv][d] or both NULL.
  * An empty cache with no new row gives out = 0.  An append that would pass m_cap is skipped
  * and sets SELKV_DEVERR_CAPACITY.
-
+ *
+ * Overlap with the previous kernel (bf16 caches): the decode is launched with programmatic
+ * dependent launch and may start loading cache rows below lengths[b] - 1 while the kernel
+ * enqueued just before it on the same stream is still running.  That kernel must therefore
+ * not write those rows of K_c and V_c (it may write q, k_new, v_new, the bias, lengths, and
+ * row lengths[b] - 1 onwards).  The library's own calls never do: a decode appends only at
+ * lengths[b], and a compression writes K_c and V_c before its last kernel.  A caller kernel
+ * that rewrites cached rows must be separated from the decode by another stream operation
+ * (any other kernel, a copy or an event).  Everything the result is computed from is read
+ * after the previous kernel has completed: rows loaded early are used only where the slice
+ * planned from the final lengths[b] starts at the same row and covers them.
  * ------------------------------------------------------------------------------------- */
 SELKV_API size_t selkv_decode_workspace_size(const selkv_shape* shape);
 

@@ -17,8 +17,12 @@
 //
 // Every mbarrier wait is bounded: on timeout the CTA raises SELKV_DEVERR_TIMEOUT, stops, and
 // waits (bounded again) for the copies it has issued before leaving.  Launched with
-// programmatic dependent launch: the barrier set-up overlaps the previous kernel's tail, and
-// nothing another kernel may have written is read before griddepcontrol.wait.
+// programmatic dependent launch: while the previous kernel of the stream finishes, the CTA
+// sets up its barriers and loads the first tiles of its slice, planned from a length read
+// without ordering, into the ring (only rows that no kernel still running can be writing:
+// below that length minus one).  After griddepcontrol.wait the slice is planned again from
+// the length read in order, and an early tile is kept only where the two plans agree; the
+// query, the bias and the lengths used for the result are all read after the wait.
 #include <algorithm>
 
 #include "decode_common.cuh"
@@ -38,7 +42,16 @@ namespace {
 #define SELKV_DEC_PDL 1        // launch with programmatic dependent launch
 #endif
 #ifndef SELKV_DEC_PF_ROWS
-#define SELKV_DEC_PF_ROWS 128  // rows of the slice prefetched into L2 before griddepcontrol.wait
+#define SELKV_DEC_PF_ROWS 128  // rows prefetched into L2 before griddepcontrol.wait when no tile is preloaded
+#endif
+#ifndef SELKV_DEC_PRELOAD
+#define SELKV_DEC_PRELOAD 2    // tiles of the slice loaded into the ring before griddepcontrol.wait
+#endif
+#ifndef SELKV_DEC_PRELOAD_WAVE
+#define SELKV_DEC_PRELOAD_WAVE 1  // only CTAs of the grid's first wave load early
+#endif
+#ifndef SELKV_DEC_PRELOAD_MIN
+#define SELKV_DEC_PRELOAD_MIN 8  // ... on slices of at least this many tiles
 #endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
@@ -60,8 +73,9 @@ struct Cfg {
   static constexpr int kTileBytes = kTile * D * 2;     // K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  // after the ring: full[kStages], empty[kStages], comb, abort flag (8 bytes), warp states
-  static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + (2 * kStages + 2) * 8 + 2 * kConsumers * 16 * 4;
+  // after the ring: full[kStages], empty[kStages], pre[kStages], comb, abort flag (8 bytes),
+  // warp states
+  static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + (3 * kStages + 2) * 8 + 2 * kConsumers * 16 * 4;
   static constexpr int kFoldLd = D + 8;                // fold row stride (floats): conflict-free float2 stores
   static_assert(kConsumers * 16 * kFoldLd * 4 <= kRingBytes, "fold scratch fits");
 };
@@ -234,38 +248,71 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kRingBytes);
   uint64_t* empty = full + kStages;
-  uint64_t* comb = empty + kStages;  // completion of the combine's bulk copy
+  uint64_t* pre = empty + kStages;   // completion of the tiles loaded before griddepcontrol.wait
+  uint64_t* comb = pre + kStages;    // completion of the combine's bulk copy
   volatile int* s_abort = reinterpret_cast<volatile int*>(comb + 1);
   float* wm = reinterpret_cast<float*>(comb + 2);  // [kConsumers][16] warp maxima (base 2)
   float* wl = wm + kConsumers * 16;                // [kConsumers][16] warp sums
   __shared__ bool s_last;
+  __shared__ int s_pre_lo, s_pre_n;  // slice start and tile count of the early loads
 
   const int s = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = a.G, S = a.splits;
   const size_t bk = (size_t)b * a.Hkv + kv;
 
-  if (tid == 0) {
+  if (warp == kConsumers && lane == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], kConsumers);
+      mbar_init(&pre[i], 1);
     }
     mbar_init(comb, 1);
     *s_abort = 0;
     fence_mbar_init();
-  }
-  if (warp == kConsumers && lane == 0) {
     prefetch_tensormap(&tmK);
     prefetch_tensormap(&tmV);
-#if SELKV_DEC_PF_ROWS > 0
-    // Warm L2 with the first rows of this CTA's slice while the previous kernel of the stream
-    // finishes (its CTAs' split combines leave HBM idle).  The slice comes from a length read
-    // before griddepcontrol.wait, which may be stale: it only steers a prefetch, and every
-    // result below is computed from data read after the wait.
+    // Before griddepcontrol.wait, while the previous kernel of the stream finishes (its split
+    // combines leave HBM idle), this CTA starts on its slice as planned from a length read
+    // without ordering, which may be stale.  Rows below that length minus one are rows no
+    // kernel that may still be running writes: the previous kernel is at most appending the
+    // row at the length it read (a decode of this cache), and anything before it has
+    // completed (the contract in selkv.h).  Whole tiles below that bound are loaded into the
+    // ring; after the wait they are used only if the slice, planned again from the true
+    // length, starts at the same row and covers them.  Only CTAs of the grid's first wave
+    // (later waves start while HBM is busy anyway) with slices of at least
+    // SELKV_DEC_PRELOAD_MIN tiles load early: on short slices the early loads are a large
+    // share of the work and they compete with the previous kernel's last CTAs; such slices
+    // prefetch their first rows into L2 instead.
     const int Lg = min(max(ld_relaxed_gpu(a.lengths + b), 0), a.m_cap);
     const int chk = ((Lg + S - 1) / S + kBoxRows - 1) / kBoxRows * kBoxRows;
-    const int plo = min(Lg, s * chk);
-    const int prow = min(min(Lg, plo + chk) - plo, SELKV_DEC_PF_ROWS);
+    const int plo = min(Lg, s * chk), phi = min(Lg, plo + chk);
+    int npre = 0;
+#if SELKV_DEC_PRELOAD
+    const int safe = min(phi, Lg - 1);
+    const bool first_wave = SELKV_DEC_PRELOAD_WAVE == 0 ||
+                            (int)(blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z)) < kPlanSMs;
+    const int max_pre = (first_wave && phi - plo >= SELKV_DEC_PRELOAD_MIN * kTile) ? min(kStages, SELKV_DEC_PRELOAD) : 0;
+    for (; npre < max_pre && plo + (npre + 1) * kTile <= safe; ++npre) {
+      unsigned char* base = smem + npre * C::kStageBytes;
+      mbar_arrive_expect_tx(&pre[npre], C::kStageBytes);
+      for (int h = 0; h < kHalves; ++h) {
+        const int y = (int)(bk * a.m_cap) + plo + npre * kTile + h * kBoxRows;
+#pragma unroll
+        for (int bx = 0; bx < C::kBoxes; ++bx)
+          tma_load_2d(base + bx * C::kBoxBytes + h * C::kPieceBytes, &tmK, bx * 64, y, &pre[npre]);
+#pragma unroll
+        for (int bx = 0; bx < C::kBoxes; ++bx)
+          tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &pre[npre]);
+      }
+    }
+#endif
+    s_pre_lo = plo;
+    s_pre_n = npre;
+#if SELKV_DEC_PF_ROWS > 0
+    // no tile loaded early: the slice's first rows go to L2 (a prefetch; nothing computed
+    // depends on it, so it may cover any row of the early plan)
+    const int prow = npre > 0 ? 0 : min(phi - plo, SELKV_DEC_PF_ROWS);
     const char* kp = static_cast<const char*>(a.Kc) + (bk * a.m_cap + plo) * (size_t)(D * 2);
     const char* vp = static_cast<const char*>(a.Vc) + (bk * a.m_cap + plo) * (size_t)(D * 2);
     for (int r = 0; r < prow; r += kBoxRows) {
@@ -307,6 +354,8 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
     // ---------------- producer ----------------
     if (lane == 0) {
       int issued = 0;
+      const int npre = s_pre_n;
+      uint32_t pre_seen = 0u;  // early loads known to have landed
       for (int t = 0; t < ntiles; ++t) {
         const int st = t % kStages;
         if (!mbar_wait(&empty[st], ((t / kStages) & 1) ^ 1)) {
@@ -315,6 +364,20 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
           break;
         }
         if (*s_abort) break;
+        if (t < npre) {
+          // the early load into this stage lands before the stage is released or reloaded
+          if (!mbar_wait(&pre[st], 0)) {
+            *s_abort = 1;
+            raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+            break;
+          }
+          pre_seen |= 1u << st;
+          if (lo == s_pre_lo && lo + (t + 1) * kTile <= hi) {
+            mbar_arrive(&full[st]);  // the tile is already in place
+            issued = t + 1;
+            continue;
+          }
+        }
         unsigned char* base = smem + st * C::kStageBytes;
         // a split's last tile may be cut at a box boundary: load only the boxes it covers
         const int nh = min(kHalves, (hi - lo - t * kTile + kBoxRows - 1) / kBoxRows);
@@ -332,6 +395,8 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       }
       // every issued copy must have landed before the ring is reused or the CTA exits
       for (int t = max(0, issued - kStages); t < issued; ++t) mbar_wait(&full[t % kStages], (t / kStages) & 1);
+      for (int st = 0; st < npre; ++st)
+        if (!(pre_seen & (1u << st))) mbar_wait(&pre[st], 0);
     }
   } else {
     // ---------------- consumers ----------------

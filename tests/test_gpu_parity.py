@@ -607,3 +607,32 @@ def test_score_entry_point(name):
         np.testing.assert_array_equal(got[b, :, :n], host["attn"][b, :, :n])
         np.testing.assert_array_equal(two[b, :, :n], got[b, :, :n])
         assert (got[b, :, n:] == -1.0).all(), "entries past n_b were written"
+
+
+def test_decode_after_a_kernel_that_rewrites_the_lengths():
+    """The decode starts on its slice before the kernel enqueued just before it has finished,
+    planning from a length it reads without ordering.  Here that previous kernel rewrites the
+    lengths (a torch fill on the same stream: shorter, then longer than the decode before it
+    left them), so the early plan is stale: every output must still equal exact attention over
+    the rows the new length names."""
+    B, Hq, Hkv, d, m_cap = 2, 8, 2, 128, 4096
+    shape = api.make_shape("bf16", B, Hq, Hkv, d, 32, m_cap, m_cap)
+    g = torch.Generator().manual_seed(5)
+    cache = api.alloc_compressed(shape)
+    cache.K_c.copy_(torch.randn(cache.K_c.shape, generator=g))
+    cache.V_c.copy_(torch.randn(cache.V_c.shape, generator=g))
+    cache.bias.copy_(0.3 * torch.rand(cache.bias.shape, generator=g))
+    ws = api.Workspace(S.selkv_decode_workspace_size(shape))
+    Kh = cache.K_c.double().cpu().numpy()
+    Vh = cache.V_c.double().cpu().numpy()
+    bh = cache.bias.double().cpu().numpy()
+    for L in (3000, 1100, 3900, 700, 2600):
+        cache.lengths.fill_(L)   # a kernel on the current stream, right before the decode
+        q = torch.randn((B, Hq, d), generator=g).to(torch.bfloat16).cuda()
+        out = api.decode(cache, q, workspace=ws).float().cpu().numpy()
+        qh = q.double().cpu().numpy()
+        for b in range(B):
+            want = O.decode(qh[b], Kh[b], Vh[b], bh[b], L)
+            check_decode(out[b], want, "bf16", "length %d seq %d" % (L, b))
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
