@@ -636,3 +636,37 @@ def test_decode_after_a_kernel_that_rewrites_the_lengths():
             check_decode(out[b], want, "bf16", "length %d seq %d" % (L, b))
     torch.cuda.synchronize()
     assert ws.errors() == 0
+
+
+def test_compress_and_decode_at_the_maximum_batch():
+    """SELKV_MAX_BATCH sequences of a few hundred tokens each (ragged, the smallest near the
+    window): every sequence passes the structural checks, eight spread over the batch are
+    checked against the oracle stage by stage, and one decode step of all of them against
+    exact attention over each one's compressed rows."""
+    from parity import check_properties
+    wl = synth.WORKLOADS["llama_layer"].with_(name="max_batch", batch=S.SELKV_MAX_BATCH, n=320,
+                                              num_q_heads=8, num_kv_heads=2, obs_window=24,
+                                              ragged=(0.3, 1.0), seed=17)
+    x = synth.gen_layer(wl, 0, threads=16)
+    p = O.Params()
+    cache, host, _ = run_compress(wl, x, p, extra=1)
+    check_properties(wl, x, host, p)
+    for b in np.linspace(0, wl.batch - 1, 8).astype(int):
+        check_sequence(wl, x, host, int(b), p)
+    dec = synth.gen_decode(wl, 0, 1)
+    Kc = cache.K_c.double().cpu().numpy()
+    Vc = cache.V_c.double().cpu().numpy()
+    bias = cache.bias.double().cpu().numpy()
+    lens = cache.lengths.cpu().numpy().copy()
+    ws = api.Workspace(S.selkv_decode_workspace_size(cache.shape))
+    out = api.decode(cache, to_dev(dec["q"][0], wl.dtype), to_dev(dec["k_new"][0], wl.dtype),
+                     to_dev(dec["v_new"][0], wl.dtype), workspace=ws).float().cpu().numpy()
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    np.testing.assert_array_equal(cache.lengths.cpu().numpy(), lens + 1)
+    for b in range(0, wl.batch, 37):
+        L = int(lens[b])
+        K1 = np.concatenate([Kc[b, :, :L], dec["k_new"][0, b][:, None]], axis=1)
+        V1 = np.concatenate([Vc[b, :, :L], dec["v_new"][0, b][:, None]], axis=1)
+        b1 = np.concatenate([bias[b, 0, :L], [0.0]])
+        check_decode(out[b], O.decode(dec["q"][0, b], K1, V1, b1, L + 1), wl.dtype, "seq %d" % b)
