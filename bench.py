@@ -99,14 +99,16 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ oracle arm
 def _oracle_unit(job):
-    """One unit of the oracle baseline, run in a worker process: generate layer `layer` of
-    sequence 0, compress it with the fp64 oracle, then decode `tokens` tokens over the
-    compressed cache (each appending a row).  Returns the times and the process's CPU time."""
-    wl, layer, tokens, per_head = job
+    """One unit of the oracle baseline: generate layer `layer` of sequence 0 (on job[4]
+    threads, default 1), compress it with the fp64 oracle, then decode `tokens` tokens over
+    the compressed cache (each appending a row).  Returns the times and the process's CPU
+    time."""
+    wl, layer, tokens, per_head = job[:4]
+    gen_threads = job[4] if len(job) > 4 else 1
     from oracle import selkv_oracle as O
     cpu0 = time.process_time()
     one = wl.with_(batch=1)
-    x = synth.gen_layer(one, layer)
+    x = synth.gen_layer(one, layer, threads=gen_threads)
     n = int(x["n_len"][0])
     K, V, Q = (x[k][0].astype(np.float64) for k in ("K", "V", "Q_obs"))
     t0 = time.perf_counter()
@@ -194,7 +196,7 @@ def oracle_sample(wl: synth.Workload, per_head: bool = False, decode_tokens: int
 def oracle_step_sample(wl: synth.Workload, layer: int, decode_tokens: int, per_head: bool = False) -> dict:
     """One bounded sample of the oracle in this process (BLAS on all cores): compression of
     layer `layer` of sequence 0 and `decode_tokens` decode tokens, scaled to the step."""
-    r = _oracle_unit((wl, layer, decode_tokens, per_head))
+    r = _oracle_unit((wl, layer, decode_tokens, per_head, os.cpu_count() or 1))
     step_s = wl.batch * wl.layers * (r["compress_s"] + wl.decode_steps * r["decode_s_per_token"])
     return {"value": wl.batch * wl.decode_steps / step_s, "compress_s": r["compress_s"],
             "decode_s_per_token": r["decode_s_per_token"]}
