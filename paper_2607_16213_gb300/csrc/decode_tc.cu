@@ -53,6 +53,9 @@ namespace {
 #ifndef SELKV_DEC_PRELOAD_MIN
 #define SELKV_DEC_PRELOAD_MIN 8  // ... on slices of at least this many tiles
 #endif
+#ifndef SELKV_DEC_PF_QB
+#define SELKV_DEC_PF_QB 2  // tiles of bias rows (and the group's queries) prefetched into L2 before the wait
+#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif
@@ -319,6 +322,24 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
       const uint32_t bytes = (uint32_t)(min(kBoxRows, prow - r) * D * 2);
       bulk_prefetch_l2(kp + (size_t)r * D * 2, bytes);
       bulk_prefetch_l2(vp + (size_t)r * D * 2, bytes);
+    }
+#endif
+#if SELKV_DEC_PF_QB > 0
+    // The group's queries and the bias of the slice's first rows go to L2 as well: the first
+    // tiles are then waiting on nothing but L2 hits after the wait.  The previous kernel may
+    // still write these (q, the bias): a prefetch only moves lines into L2, where its writes
+    // land, and the values used are loaded after the wait.
+    {
+      const char* qp = static_cast<const char*>(a.q) + ((size_t)b * a.Hq + (size_t)kv * G) * D * 2;
+      for (int off = 0; off < G * D * 2; off += 128) prefetch_l2(qp + off);
+      if (a.bias != nullptr) {
+        const char* bp = reinterpret_cast<const char*>(a.bias + bk * a.m_cap + plo);
+        const int nb = min(phi - plo, SELKV_DEC_PF_QB * kTile) * 4;  // bytes, inside row bk's bias
+        if (nb > 0) {
+          for (int off = 0; off < nb; off += 128) prefetch_l2(bp + off);
+          prefetch_l2(bp + nb - 1);
+        }
+      }
     }
 #endif
   }

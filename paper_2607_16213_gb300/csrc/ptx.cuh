@@ -78,6 +78,10 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
                "l"(src), "r"(bytes), "r"(smem_u32(bar))
                : "memory");
 }
+// Prefetch of the 128-byte line holding `p` into L2 (a hint: no data returned, no ordering).
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
 // Hint: bring `bytes` (a multiple of 16) of global memory starting at `src` (16-byte aligned)
 // into L2.  No completion, no effect on any result.
 __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
