@@ -36,9 +36,12 @@ __device__ __forceinline__ bool selected(uint32_t u, int j, const RadixState& s)
 
 // Add this CTA's shared histogram to the unit's global one, then arrive; the last CTA of the
 // unit (of `nblocks`) reads the unit's histogram back into `sh` (one round of loads), picks
-// the digit of `pass` and narrows the unit's state.
+// the digit of `pass` and narrows the unit's state.  The pick uses the whole CTA: thread t
+// sums `per` consecutive bins counted from the top digit down, a CTA-wide scan of those sums
+// finds the thread whose bins reach the krem-th entry, and that thread walks its bins.
 __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, int pass, int nblocks,
                                  bool* s_last) {
+  __shared__ uint32_t s_wsum[32];
   const int bins = pass == 2 ? 1024 : kBins;
   __syncthreads();
   for (int i = threadIdx.x; i < bins; i += blockDim.x)
@@ -51,38 +54,56 @@ __device__ void flush_and_select(uint32_t* sh, uint32_t* ghist, RadixState* st, 
   __threadfence();
   for (int i = threadIdx.x; i < bins; i += blockDim.x) sh[i] = __ldcg(&ghist[i]);
   __syncthreads();
-  if (threadIdx.x < 32) {
-    const int lane = threadIdx.x, per = bins / 32;
-    const int hi = bins - 1 - lane * per;  // this lane covers bins hi, hi-1, ..., hi-per+1
-    uint32_t tot = 0;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
+  const int per = bins >= (int)blockDim.x ? bins / (int)blockDim.x : 1;
+  const int owners = bins / per;             // threads that own bins (the rest own none)
+  const int hi = bins - 1 - tid * per;       // this thread's bins: hi, hi-1, ..., hi-per+1
+  uint32_t tot = 0;
+  if (tid < owners)
     for (int t = 0; t < per; ++t) tot += sh[hi - t];
-    uint32_t incl = tot;
+  uint32_t incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_wsum[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t v = lane < nwarps ? s_wsum[lane] : 0u;
+    uint32_t w = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
+      const uint32_t x = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += x;
     }
-    const uint32_t krem = st->krem;
-    const unsigned bal = __ballot_sync(0xffffffffu, incl >= krem);
-    const int L = bal ? __ffs(bal) - 1 : 31;
-    if (lane == L) {
-      uint32_t cum = incl - tot;
-      int dg = hi - per + 1;
-      uint32_t cnt = 0;
-      for (int t = 0; t < per; ++t) {
-        const uint32_t c = sh[hi - t];
-        if (cum + c >= krem) {
-          dg = hi - t;
-          cnt = c;
-          break;
-        }
-        cum += c;
+    if (lane < nwarps) s_wsum[lane] = w - v;  // entries in the bins of the warps before
+  }
+  __syncthreads();
+  incl += s_wsum[warp];
+  const uint32_t krem = st->krem;
+  const uint32_t excl = incl - tot;
+  // the owner of the krem-th entry; if fewer entries remain than krem, the owner of bin 0;
+  // with krem = 0, the owner of the top bin
+  const bool mine = tid < owners && ((excl < krem && incl >= krem) || (tid == owners - 1 && incl < krem) ||
+                                     (krem == 0u && tid == 0));
+  if (mine) {
+    uint32_t cum = excl;
+    int dg = hi - per + 1;
+    uint32_t cnt = 0;
+    for (int t = 0; t < per; ++t) {
+      const uint32_t c = sh[hi - t];
+      if (cum + c >= krem) {
+        dg = hi - t;
+        cnt = c;
+        break;
       }
-      st->prefix |= (uint32_t)dg << kShift[pass];
-      st->krem = krem - cum;
-      if (pass == 2) st->count_eq = cnt;
-      st->arrive = 0u;
+      cum += c;
     }
+    st->prefix |= (uint32_t)dg << kShift[pass];
+    st->krem = krem - cum;
+    if (pass == 2) st->count_eq = cnt;
+    st->arrive = 0u;
   }
 }
 
