@@ -377,8 +377,9 @@ __global__ __launch_bounds__(kBlock) void compact_write_kernel(CompressArgs a, S
 size_t select_ws_bytes(int B, int Hkv, int n_cap) {
   const size_t units = (size_t)B * Hkv;
   const size_t blocks = (size_t)(n_cap + kSpan - 1) / kSpan;
+  // seven regions, each start rounded up to 256 bytes
   return (units + B) * sizeof(RadixState) + (units + B) * 3 * kBins * 4 + units * blocks * 4 +
-         (size_t)B * n_cap * 5 + 4 * 256;
+         (size_t)B * n_cap * 5 + 7 * 256;
 }
 
 SelectWs carve_select_ws(void* base, int B, int Hkv, int n_cap) {
