@@ -153,6 +153,10 @@ typedef struct selkv_compress_debug {
 /* Human-readable name of a status code (static storage). */
 SELKV_API const char* selkv_status_string(selkv_status status);
 
+/* The CUDA runtime error behind the last SELKV_ERR_CUDA returned on the calling thread
+ * (cudaSuccess = 0 if none), and its name in *name when name is not NULL (static storage). */
+SELKV_API int selkv_last_cuda_error(const char** name);
+
 /* Number of kernels this library has enqueued since it was loaded, over all threads and
  * devices (a diagnostic counter; a captured CUDA graph counts its kernels once, at capture). */
 SELKV_API uint64_t selkv_kernel_launches(void);

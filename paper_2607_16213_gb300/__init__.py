@@ -16,7 +16,8 @@ from ._binding import (  # noqa: F401
     SELKV_DEVERR_CAPACITY,
     SELKV_DEVERR_TIMEOUT, SELKV_DEVERR_LENGTH, SELKV_DEVERR_COUNT, SELKV_MAX_BATCH,
     SelKVError, selkv_shape, selkv_params, selkv_compress_debug, library, library_path,
-    exported_symbols, check, selkv_status_string, selkv_kernel_launches, selkv_workspace_init,
+    exported_symbols, check, selkv_status_string, selkv_last_cuda_error, selkv_kernel_launches,
+    selkv_workspace_init,
     selkv_workspace_error, selkv_compress_workspace_size, selkv_compress,
     selkv_decode_workspace_size, selkv_decode_attn, selkv_decode_attn_static,
     selkv_layer_average_workspace_size, selkv_layer_average_bias, selkv_score_workspace_size,

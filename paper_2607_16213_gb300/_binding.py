@@ -31,7 +31,11 @@ c_i32, c_u32, c_u64, c_sz, c_vp, c_f32, c_f64 = (ctypes.c_int32, ctypes.c_uint32
 class SelKVError(RuntimeError):
     def __init__(self, status: int, what: str = ""):
         self.status = status
-        super().__init__("%s: %s (status %d)" % (what or "selkv", selkv_status_string(status), status))
+        detail = ""
+        if status == SELKV_ERR_CUDA:
+            code, name = selkv_last_cuda_error()
+            detail = "; %s (%d)" % (name, code)
+        super().__init__("%s: %s (status %d%s)" % (what or "selkv", selkv_status_string(status), status, detail))
 
 
 class selkv_shape(ctypes.Structure):
@@ -80,6 +84,7 @@ def library() -> ctypes.CDLL:
     lib = ctypes.CDLL(path)
     sig = {
         "selkv_status_string": (ctypes.c_char_p, [c_i32]),
+        "selkv_last_cuda_error": (c_i32, [ctypes.POINTER(ctypes.c_char_p)]),
         "selkv_kernel_launches": (c_u64, []),
         "selkv_workspace_init": (c_i32, [c_vp, c_sz, c_vp]),
         "selkv_workspace_error": (c_i32, [c_vp, c_vp, ctypes.POINTER(c_u32)]),
@@ -141,6 +146,16 @@ def selkv_status_string(status: int) -> str:
         return library().selkv_status_string(status).decode()
     except RuntimeError:
         return "status %d" % status
+
+
+def selkv_last_cuda_error():
+    """(code, name) of the CUDA error behind the last SELKV_ERR_CUDA on this thread."""
+    try:
+        name = ctypes.c_char_p()
+        code = int(library().selkv_last_cuda_error(ctypes.byref(name)))
+        return code, (name.value or b"").decode()
+    except RuntimeError:
+        return -1, "unknown"
 
 
 def selkv_kernel_launches() -> int:

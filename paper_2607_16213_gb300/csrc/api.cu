@@ -192,6 +192,16 @@ int compress_kernel_count(const CompressArgs& a) {
 
 }  // namespace selkv
 
+namespace selkv {
+namespace {
+thread_local cudaError_t g_last_cuda = cudaSuccess;
+}  // namespace
+selkv_status cuda_fail(cudaError_t e) {
+  g_last_cuda = e;
+  return SELKV_ERR_CUDA;
+}
+}  // namespace selkv
+
 using namespace selkv;
 
 extern "C" {
@@ -208,13 +218,19 @@ const char* selkv_status_string(selkv_status status) {
   return "unknown status";
 }
 
+int selkv_last_cuda_error(const char** name) {
+  const cudaError_t e = g_last_cuda;
+  if (name != nullptr) *name = cudaGetErrorName(e);
+  return (int)e;
+}
+
 uint64_t selkv_kernel_launches(void) { return g_launches.load(); }
 
 selkv_status selkv_workspace_init(void* workspace, size_t workspace_bytes, selkv_stream_t stream) {
   if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < sizeof(WsHeader))
     return SELKV_ERR_WORKSPACE;
-  if (cudaMemsetAsync(workspace, 0, workspace_bytes, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-    return SELKV_ERR_CUDA;
+  const cudaError_t e = cudaMemsetAsync(workspace, 0, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e);
   return SELKV_OK;
 }
 
@@ -222,12 +238,13 @@ selkv_status selkv_workspace_error(void* workspace, selkv_stream_t stream, uint3
   if (workspace == nullptr || flags == nullptr) return SELKV_ERR_INVALID_ARG;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   uint32_t f = 0;
-  if (cudaMemcpyAsync(&f, workspace, sizeof(f), cudaMemcpyDeviceToHost, st) != cudaSuccess) return SELKV_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return SELKV_ERR_CUDA;
+  if (const cudaError_t e = cudaMemcpyAsync(&f, workspace, sizeof(f), cudaMemcpyDeviceToHost, st); e != cudaSuccess)
+    return cuda_fail(e);
+  if (const cudaError_t e = cudaStreamSynchronize(st); e != cudaSuccess) return cuda_fail(e);
   *flags = f;
   if (f != 0) {
-    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), st) != cudaSuccess) return SELKV_ERR_CUDA;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return SELKV_ERR_CUDA;
+    if (const cudaError_t e = cudaMemsetAsync(workspace, 0, sizeof(uint32_t), st); e != cudaSuccess) return cuda_fail(e);
+    if (const cudaError_t e = cudaStreamSynchronize(st); e != cudaSuccess) return cuda_fail(e);
     return SELKV_ERR_DEVICE;
   }
   return SELKV_OK;
@@ -367,7 +384,7 @@ selkv_status selkv_compress(const selkv_shape* shape, const int32_t* n_len, doub
     e = launch_select_grid(a, sw, st);
   if (e == cudaSuccess) e = launch_merge(a, st);
   g_launches += (uint64_t)compress_kernel_count(a);
-  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+  return e == cudaSuccess ? SELKV_OK : cuda_fail(e);
 }
 
 size_t selkv_score_workspace_size(const selkv_shape* shape) {
@@ -428,7 +445,7 @@ selkv_status selkv_score(const selkv_shape* shape, const int32_t* n_len, const v
   if (e == cudaSuccess)
     e = score_uses_tc(a.dtype, a.D, a.R) ? launch_score_tc(a, st, passes) : launch_score_simt(a, st, passes);
   g_launches += (uint64_t)kernels;
-  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+  return e == cudaSuccess ? SELKV_OK : cuda_fail(e);
 }
 
 size_t selkv_layer_average_workspace_size(const selkv_shape* shape) {
@@ -471,7 +488,7 @@ selkv_status selkv_layer_average_bias(const selkv_shape* shape, const selkv_para
   a.acc = at<float>(workspace, sizeof(WsHeader));
   const cudaError_t e = launch_layer_average(a, P, reinterpret_cast<cudaStream_t>(stream));
   g_launches += (uint64_t)num_layers + 1;
-  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+  return e == cudaSuccess ? SELKV_OK : cuda_fail(e);
 }
 
 size_t selkv_decode_workspace_size(const selkv_shape* shape) {
@@ -520,7 +537,7 @@ selkv_status selkv_decode_attn(const selkv_shape* shape, const void* q, void* K_
   a.partial = at<float>(workspace, plan.partial);
   const cudaError_t e = launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
   g_launches += kDecodeKernels;
-  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+  return e == cudaSuccess ? SELKV_OK : cuda_fail(e);
 }
 
 }  // extern "C"

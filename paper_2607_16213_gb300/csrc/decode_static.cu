@@ -115,11 +115,11 @@ extern "C" SELKV_API selkv_status selkv_decode_attn_static(
   if (need > (size_t)SELKV_STATIC_SCRATCH_BYTES) return SELKV_ERR_WORKSPACE;
 
   void* base = nullptr;
-  if (scratch_address(&base) != cudaSuccess) return SELKV_ERR_CUDA;
+  if (const cudaError_t e = scratch_address(&base); e != cudaSuccess) return cuda_fail(e);
   char* sb = static_cast<char*>(base);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   // the counters must start at zero; the error word is cleared with them
-  if (cudaMemsetAsync(sb, 0, off_part, st) != cudaSuccess) return SELKV_ERR_CUDA;
+  if (const cudaError_t e = cudaMemsetAsync(sb, 0, off_part, st); e != cudaSuccess) return cuda_fail(e);
 
   DecodeArgs a{};
   a.dtype = s.dtype;
@@ -145,5 +145,5 @@ extern "C" SELKV_API selkv_status selkv_decode_attn_static(
   a.partial = reinterpret_cast<float*>(sb + off_part);
   const cudaError_t e = launch_decode(a, st);
   note_launches(1);
-  return e == cudaSuccess ? SELKV_OK : SELKV_ERR_CUDA;
+  return e == cudaSuccess ? SELKV_OK : cuda_fail(e);
 }

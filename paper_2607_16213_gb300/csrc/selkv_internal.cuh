@@ -338,6 +338,9 @@ cudaError_t set_smem_once(int bytes) {
 // so the separate copy kernel is not launched.
 bool merge_copies_kept_rows(const CompressArgs& a);
 
+// SELKV_ERR_CUDA, with `e` kept for selkv_last_cuda_error on this thread.
+selkv_status cuda_fail(cudaError_t e);
+
 int decode_splits(int B, int Hkv, int m_cap, int num_sms);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);     // dispatch by dtype
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);  // bf16: TMA + tensor cores

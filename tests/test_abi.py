@@ -47,6 +47,12 @@ def test_status_strings(lib):
     assert S.selkv_status_string(99) == "unknown status"
 
 
+def test_last_cuda_error_starts_clear(lib):
+    # nothing has failed on this thread: cudaSuccess, by its runtime name
+    code, name = S.selkv_last_cuda_error()
+    assert code == 0 and name == "cudaSuccess"
+
+
 def test_workspace_sizes(lib):
     s = shape()
     c = S.selkv_compress_workspace_size(s)
