@@ -252,7 +252,7 @@ __global__ __launch_bounds__(cta_threads(PASS), 1) void score_tc_kernel(const __
     const int q = warp & 3, part = warp >> 2;  // lane quarter of TMEM, and which part of the work
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const float sc = a.scale_log2;
-    // lane 0 waits, the warp follows its verdict (tcgen05.ld below needs the whole warp)
+    // lane 0 waits, the warp follows its outcome (tcgen05.ld below needs the whole warp)
     auto warp_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
       int ok = 0;
       if (lane == 0) {
