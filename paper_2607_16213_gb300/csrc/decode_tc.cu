@@ -257,6 +257,7 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
   float* wm = reinterpret_cast<float*>(comb + 2);  // [kConsumers][16] warp maxima (base 2)
   float* wl = wm + kConsumers * 16;                // [kConsumers][16] warp sums
   __shared__ bool s_last;
+  __shared__ float s_inv[16];  // one split: 1 / sum per query head of the group
   __shared__ int s_pre_lo, s_pre_n;  // slice start and tile count of the early loads
 
   const int s = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
@@ -620,7 +621,8 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
 #pragma unroll
           for (int w = 0; w < kConsumers; ++w) Ls = fmaf(wl[w * 16 + g], exp2f(wm[w * 16 + g] - M), Ls);
         }
-        *pv.ml(bk, g, s) = aborted ? make_float2(-INFINITY, 0.f) : make_float2(M, Ls);
+        if (S == 1) s_inv[g] = (Ls > 0.f && !aborted) ? 1.f / Ls : 0.f;
+        else *pv.ml(bk, g, s) = aborted ? make_float2(-INFINITY, 0.f) : make_float2(M, Ls);
       }
     }
   }
@@ -639,8 +641,23 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
         acc.w += v.w;
       }
       if (aborted) acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      reinterpret_cast<float4*>(pv.o(bk, g, s))[d4] = acc;
+      if (S == 1) {
+        // the CTA holds the whole of (b, kv): its fold is the output
+        const float iv = s_inv[g];
+        const float r[4] = {acc.x * iv, acc.y * iv, acc.z * iv, acc.w * iv};
+        store4(static_cast<__nv_bfloat16*>(a.out) + (bk * G + g) * D + d4 * 4, r);
+      } else {
+        reinterpret_cast<float4*>(pv.o(bk, g, s))[d4] = acc;
+      }
     }
+  }
+  if (S == 1) {
+    // no split to wait for: only the length bookkeeping of the sequence remains
+    if (tid == 0) {
+      const uint32_t old = finish_lengths_begin(a, b, bk, app, 0);
+      finish_lengths_end(a, b, L, app, old, 0);
+    }
+    return;
   }
   if (!arrive_last(a, bk, &s_last)) return;
   if (S <= kRegSplits)
