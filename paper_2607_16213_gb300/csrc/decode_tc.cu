@@ -56,6 +56,12 @@ namespace {
 #ifndef SELKV_DEC_PF_QB
 #define SELKV_DEC_PF_QB 2  // tiles of bias rows (and the group's queries) prefetched into L2 before the wait
 #endif
+#ifndef SELKV_DEC_UNITS
+#define SELKV_DEC_UNITS 1  // persistent unit-walking CTAs when every (b, kv) has one split and they outnumber the SMs
+#endif
+#ifndef SELKV_DEC_UNITS_MAX_ROWS
+#define SELKV_DEC_UNITS_MAX_ROWS 2112  // ... and their capacity is at most this many rows
+#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif
@@ -666,26 +672,439 @@ __global__ __launch_bounds__(kThreads, SELKV_DEC_MINBLOCKS) void decode_tc_kerne
     combine_record<D>(a, b, kv, bk, smem, C::kRingBytes, comb, L, app);
 }
 
+// ---- one split per (b, kv), more units than CTAs: persistent CTAs ------------------------------
+// When the split model gives every (b, kv) a single CTA and there are more of them than SMs,
+// a grid of kUnitsCtas CTAs walks the units instead: CTA p takes units p, p + P, p + 2P, ...
+// in turn.  The producer streams the next unit's tiles while the consumer warps fold the
+// previous one (the ring runs on across units), so the start and drain of a CTA are paid once
+// per CTA instead of once per unit.  Each unit is held whole by one CTA: its fold is its output.
+// The group's queries (and the appended row) are staged in shared memory per unit, so the
+// mma fragments are not held in registers across the tiles.
+template <int D, bool ROWS16>
+struct UCfg {
+  using C = Cfg<D>;
+  static constexpr int kRows = ROWS16 ? 16 : 8;          // group rows a warp state holds
+  static constexpr int kFoldLd = D + 8;
+  static constexpr int kFoldBytes = kConsumers * kRows * kFoldLd * 4;
+  static constexpr int kQLd = D + 8;                     // staged query row stride (bf16)
+  static constexpr int kQBytes = 16 * kQLd * 2 + 2 * D * 2;  // queries (16 rows), k_new, v_new
+  // ring | fold scratch | queries | full, empty, pre [kStages] | abort | warp (max, sum), appended row
+  static constexpr int kSmemBytes =
+      1024 + C::kRingBytes + kFoldBytes + kQBytes + 3 * kStages * 8 + 8 + 2 * (kConsumers + 1) * 16 * 4;
+  static_assert((C::kRingBytes + kFoldBytes) % 16 == 0 && kQBytes % 16 == 0, "query rows 16-byte aligned");
+};
+
+template <int D, bool ROWS16>
+__global__ __launch_bounds__(kThreads, 1) void decode_units_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                                   const __grid_constant__ CUtensorMap tmV,
+                                                                   DecodeArgs a) {
+  using C = Cfg<D>;
+  using U = UCfg<D, ROWS16>;
+  constexpr int NT = D / 8;
+  constexpr int KS = D / 16;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  float* wo = reinterpret_cast<float*>(smem + C::kRingBytes);  // [kConsumers][kRows][kFoldLd]
+  __nv_bfloat16* sq = reinterpret_cast<__nv_bfloat16*>(smem + C::kRingBytes + U::kFoldBytes);  // [16][kQLd]
+  __nv_bfloat16* snew = sq + 16 * U::kQLd;                                                   // [2][D]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kRingBytes + U::kFoldBytes + U::kQBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* pre = empty + kStages;
+  volatile int* s_abort = reinterpret_cast<volatile int*>(pre + kStages);
+  float* wm = reinterpret_cast<float*>(pre + kStages + 1);  // [kConsumers][16]
+  float* wl = wm + kConsumers * 16;                         // [kConsumers][16]
+  float* apm = wl + kConsumers * 16;                        // [16] appended row's logit
+  float* apw = apm + 16;                                    // [16] its weight / the normaliser
+  __shared__ int s_pre_n;
+  __shared__ float s_inv[16];  // 1 / normaliser per query head of the unit
+
+  const int p = blockIdx.x, P = gridDim.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int G = a.G;
+  const int units = a.B * a.Hkv;
+  constexpr int kBar = 1;  // named barrier of the consumer warps
+  constexpr int kCons = kConsumers * 32;
+
+  if (warp == kConsumers && lane == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kConsumers);
+      mbar_init(&pre[i], 1);
+    }
+    *s_abort = 0;
+    fence_mbar_init();
+    prefetch_tensormap(&tmK);
+    prefetch_tensormap(&tmV);
+    // Before griddepcontrol.wait: the first unit's first tiles below its (possibly stale)
+    // length minus one, as in the split kernel; kept after the wait if the length still covers them.
+    int npre = 0;
+    if (p < units) {
+      const int b = p / a.Hkv;
+      const size_t bk = (size_t)p;
+      const int Lg = min(max(ld_relaxed_gpu(a.lengths + b), 0), a.m_cap);
+      const int safe = Lg - 1;
+      const int max_pre = Lg >= SELKV_DEC_PRELOAD_MIN * kTile ? min(kStages, SELKV_DEC_PRELOAD) : 0;
+      for (; npre < max_pre && (npre + 1) * kTile <= safe; ++npre) {
+        unsigned char* base = smem + npre * C::kStageBytes;
+        mbar_arrive_expect_tx(&pre[npre], C::kStageBytes);
+        for (int h = 0; h < kHalves; ++h) {
+          const int y = (int)(bk * a.m_cap) + npre * kTile + h * kBoxRows;
+#pragma unroll
+          for (int bx = 0; bx < C::kBoxes; ++bx)
+            tma_load_2d(base + bx * C::kBoxBytes + h * C::kPieceBytes, &tmK, bx * 64, y, &pre[npre]);
+#pragma unroll
+          for (int bx = 0; bx < C::kBoxes; ++bx)
+            tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &pre[npre]);
+        }
+      }
+      const char* qp = static_cast<const char*>(a.q) + ((size_t)b * a.Hq + (size_t)(p % a.Hkv) * G) * D * 2;
+      for (int off = 0; off < G * D * 2; off += 128) prefetch_l2(qp + off);
+    }
+    s_pre_n = npre;
+  }
+  pdl_wait();
+  pdl_launch_dependents();
+  __syncthreads();
+  const bool has_new = a.k_new != nullptr;
+
+  if (warp == kConsumers) {
+    // ---------------- producer ----------------
+    if (lane == 0) {
+      const int npre = s_pre_n;
+      uint32_t pre_seen = 0u;
+      int issued = 0;  // tiles handed to the consumers so far, over all of this CTA's units
+      bool stop = false;
+      for (int u = p; u < units && !stop; u += P) {
+        const int L = min(max(a.lengths[u / a.Hkv], 0), a.m_cap);
+        const int nt = (L + kTile - 1) / kTile;
+        const int row0 = (int)((size_t)u * a.m_cap);
+        for (int t = 0; t < nt; ++t) {
+          const int tg = issued, st = tg % kStages;
+          if (!mbar_wait(&empty[st], ((tg / kStages) & 1) ^ 1)) {
+            *s_abort = 1;
+            raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+            stop = true;
+            break;
+          }
+          if (*s_abort) {
+            stop = true;
+            break;
+          }
+          if (tg < npre) {
+            // the early load into this stage lands before the stage is released or reloaded
+            if (!mbar_wait(&pre[st], 0)) {
+              *s_abort = 1;
+              raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+              stop = true;
+              break;
+            }
+            pre_seen |= 1u << st;
+            if (u == p && (t + 1) * kTile <= L) {
+              mbar_arrive(&full[st]);  // the tile is already in place
+              issued = tg + 1;
+              continue;
+            }
+          }
+          unsigned char* base = smem + st * C::kStageBytes;
+          const int nh = min(kHalves, (L - t * kTile + kBoxRows - 1) / kBoxRows);
+          mbar_arrive_expect_tx(&full[st], 2 * nh * C::kBoxes * C::kPieceBytes);
+          for (int h = 0; h < nh; ++h) {
+            const int y = row0 + t * kTile + h * kBoxRows;
+#pragma unroll
+            for (int bx = 0; bx < C::kBoxes; ++bx)
+              tma_load_2d(base + bx * C::kBoxBytes + h * C::kPieceBytes, &tmK, bx * 64, y, &full[st]);
+#pragma unroll
+            for (int bx = 0; bx < C::kBoxes; ++bx)
+              tma_load_2d(base + C::kTileBytes + bx * C::kBoxBytes + h * C::kPieceBytes, &tmV, bx * 64, y, &full[st]);
+          }
+          issued = tg + 1;
+        }
+      }
+      for (int tg = max(0, issued - kStages); tg < issued; ++tg) mbar_wait(&full[tg % kStages], (tg / kStages) & 1);
+      for (int st = 0; st < npre; ++st)
+        if (!(pre_seen & (1u << st))) mbar_wait(&pre[st], 0);
+    }
+    return;
+  }
+  // ---------------- consumers ----------------
+  const int g0 = lane >> 2, c2 = (lane & 3) * 2;
+  const float sc = a.scale_log2;
+  int tg = 0;  // tiles consumed so far, in step with the producer
+  for (int u = p; u < units; u += P) {
+    const int b = u / a.Hkv;
+    const size_t bk = (size_t)u;
+    int L = a.lengths[b];
+    if (L < 0 || L > a.m_cap) {
+      if (tid == 0 && u % a.Hkv == 0) raise_flag(a.flags, SELKV_DEVERR_LENGTH);
+      L = L < 0 ? 0 : a.m_cap;
+    }
+    const bool app = has_new && L + 1 <= a.m_cap;
+    const int nt = (L + kTile - 1) / kTile;
+    float o[NT][4];
+    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+#pragma unroll
+    for (int n8 = 0; n8 < NT; ++n8)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[n8][e] = 0.f;
+    {
+      const __nv_bfloat16* qg = static_cast<const __nv_bfloat16*>(a.q) + ((size_t)b * a.Hq + (size_t)(u - b * a.Hkv) * G) * D;
+      for (int i = tid; i < 16 * (D / 8); i += kCons) {
+        const int row = i / (D / 8), c8 = i % (D / 8);
+        const uint4 v = row < G ? *reinterpret_cast<const uint4*>(qg + (size_t)row * D + c8 * 8) : make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4*>(sq + row * U::kQLd + c8 * 8) = v;
+      }
+      if (app) {
+        // the appended row: into shared memory for the fold, and into the cache at row L (no
+        // tile of this launch reads it)
+        for (int i = tid; i < 2 * (D / 8); i += kCons) {
+          const bool isv = i >= D / 8;
+          const int c8 = isv ? i - D / 8 : i;
+          const uint4 v = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(isv ? a.v_new : a.k_new) +
+                                                          bk * D + c8 * 8);
+          *reinterpret_cast<uint4*>(snew + (isv ? D : 0) + c8 * 8) = v;
+          *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(isv ? a.Vc : a.Kc) + (bk * a.m_cap + L) * D + c8 * 8) = v;
+        }
+        if (tid == 0 && a.bias != nullptr) a.bias[bk * a.m_cap + L] = 0.f;
+      }
+    }
+    named_bar_sync(kBar, kCons);
+    const uint32_t qs = smem_u32(sq) + (uint32_t)(((lane & 15) * U::kQLd + (lane >> 4) * 8) * 2);
+    const float* brow = a.bias != nullptr ? a.bias + bk * a.m_cap : nullptr;
+    auto fetch_bias = [&](int t, float (&dst)[2][2]) {
+#pragma unroll
+      for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = t * kTile + warp * 16 + n2 * 8 + c2 + e;
+          dst[n2][e] = (brow != nullptr && key < L) ? __ldg(brow + key) * kLog2e : 0.f;
+        }
+    };
+    float bnext[2][2];
+    if (nt > 0) fetch_bias(0, bnext);
+    for (int t = 0; t < nt; ++t, ++tg) {
+      float bv[2][2];
+#pragma unroll
+      for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) bv[n2][e] = bnext[n2][e];
+      if (t + 1 < nt) fetch_bias(t + 1, bnext);
+      const int st = tg % kStages;
+      if (!__all_sync(0xffffffffu, *s_abort == 0)) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&full[st], (tg / kStages) & 1))) {
+        *s_abort = 1;
+        if (lane == 0) raise_flag(a.flags, SELKV_DEVERR_TIMEOUT);
+        break;
+      }
+      const int key0 = t * kTile + warp * 16;
+      const int nvalid = L - key0;
+      if (nvalid > 0) {
+        const uint32_t Kt = smem_u32(smem + st * C::kStageBytes);
+        const uint32_t Vt = Kt + C::kTileBytes;
+        float sacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+        const int mi = lane >> 3, ri = lane & 7;
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+          const int krow = (mi >> 1) * 8 + ri;
+          const int chunk16 = ks * 2 + (mi & 1);
+          uint32_t kb[4], qf[4];
+          ldmatrix_x4(kb, Kt + (chunk16 >> 3) * C::kBoxBytes + swz128(warp * 16 + krow, chunk16 & 7));
+          ldmatrix_x4(qf, qs + ks * 32);
+          mma_bf16_16816(sacc[0], qf, kb[0], kb[1]);
+          mma_bf16_16816(sacc[1], qf, kb[2], kb[3]);
+        }
+        float tmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+        for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const bool ok = key0 + n2 * 8 + c2 + e < L;
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+              const float v = ok ? fmaf(sacc[n2][r * 2 + e], sc, bv[n2][e]) : -INFINITY;
+              sacc[n2][r * 2 + e] = v;
+              tmax[r] = fmaxf(tmax[r], v);
+            }
+          }
+        float corr[2], mref[2];
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 1));
+          tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 2));
+          const float mn = fmaxf(mrow[r], tmax[r]);
+          mref[r] = mn == -INFINITY ? 0.f : mn;
+          corr[r] = exp2f(mrow[r] - mref[r]);
+          mrow[r] = mn;
+        }
+        float pr[2][4];
+        float psum[2] = {0.f, 0.f};
+#pragma unroll
+        for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            pr[n2][i] = exp2f(sacc[n2][i] - mref[i >> 1]);
+            psum[i >> 1] += pr[n2][i];
+          }
+#pragma unroll
+        for (int r = 0; r < 2; ++r) lrow[r] = lrow[r] * corr[r] + psum[r];
+#pragma unroll
+        for (int n8 = 0; n8 < NT; ++n8) {
+          o[n8][0] *= corr[0];
+          o[n8][1] *= corr[0];
+          o[n8][2] *= corr[1];
+          o[n8][3] *= corr[1];
+        }
+        uint32_t pa[4];
+        pa[0] = pack_bf16(pr[0][0], pr[0][1]);
+        pa[1] = pack_bf16(pr[0][2], pr[0][3]);
+        pa[2] = pack_bf16(pr[1][0], pr[1][1]);
+        pa[3] = pack_bf16(pr[1][2], pr[1][3]);
+        const bool zeroed = nvalid < 16;
+        if (zeroed) {
+          unsigned char* vt = smem + st * C::kStageBytes + C::kTileBytes;
+          for (int i = lane; i < (16 - nvalid) * C::kBoxes * 8; i += 32) {
+            const int r = warp * 16 + nvalid + i / (C::kBoxes * 8);
+            const int rem = i % (C::kBoxes * 8);
+            *reinterpret_cast<uint4*>(vt + (rem >> 3) * C::kBoxBytes + r * 128 + (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+          }
+          __syncwarp();
+        }
+#pragma unroll
+        for (int n8 = 0; n8 < NT; n8 += 2) {
+          const int vrow = (mi & 1) * 8 + ri;
+          const int chunk16 = n8 + (mi >> 1);
+          uint32_t vb[4];
+          ldmatrix_x4_trans(vb, Vt + (chunk16 >> 3) * C::kBoxBytes + swz128(warp * 16 + vrow, chunk16 & 7));
+          mma_bf16_16816(o[n8], pa, vb[0], vb[1]);
+          mma_bf16_16816(o[n8 + 1], pa, vb[2], vb[3]);
+        }
+        if (zeroed) fence_proxy_async_smem();
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+    }
+    // Fold the warp states (and the appended row, bias 0) into the unit's output, among the
+    // consumer warps only: the producer is already loading the next unit.
+    if (app) {
+      for (int g = warp; g < G; g += kConsumers) {
+        float part = 0.f;
+        for (int d = lane; d < D; d += 32)
+          part = fmaf(__bfloat162float(sq[g * U::kQLd + d]), __bfloat162float(snew[d]), part);
+        part = warp_sum(part) * sc;
+        if (lane == 0) apm[g] = part;
+      }
+    }
+    if ((lane & 3) == 0) {
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int g = g0 + r * 8;
+        if (g >= G) continue;
+        wm[warp * 16 + g] = mrow[r];
+        wl[warp * 16 + g] = lrow[r];
+      }
+    }
+    named_bar_sync(kBar, kCons);
+    const bool aborted = *s_abort != 0;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int g = g0 + r * 8;
+      if (g >= G) continue;
+      float M = app ? apm[g] : -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, wm[w * 16 + g]);
+      const float f = M == -INFINITY ? 0.f : exp2f(mrow[r] - M);
+#pragma unroll
+      for (int n8 = 0; n8 < NT; ++n8)
+        *reinterpret_cast<float2*>(wo + (warp * U::kRows + g) * U::kFoldLd + n8 * 8 + c2) =
+            make_float2(o[n8][r * 2] * f, o[n8][r * 2 + 1] * f);
+      if (warp == 0 && (lane & 3) == 0) {
+        float Ls = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+          for (int w = 0; w < kConsumers; ++w) Ls = fmaf(wl[w * 16 + g], exp2f(wm[w * 16 + g] - M), Ls);
+        }
+        const float wa = app ? exp2f(apm[g] - M) : 0.f;  // M >= apm[g] > -inf when app
+        Ls += wa;
+        const float inv = (Ls > 0.f && !aborted) ? 1.f / Ls : 0.f;
+        apw[g] = wa * inv;   // the appended row's share of the output
+        s_inv[g] = inv;
+      }
+    }
+    named_bar_sync(kBar, kCons);
+    {
+      constexpr int D4 = D / 4;
+      for (int i = tid; i < G * D4; i += kCons) {
+        const int g = i / D4, d4 = i % D4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int w = 0; w < kConsumers; ++w) {
+          const float4 v = *reinterpret_cast<const float4*>(wo + (w * U::kRows + g) * U::kFoldLd + d4 * 4);
+          acc.x += v.x;
+          acc.y += v.y;
+          acc.z += v.z;
+          acc.w += v.w;
+        }
+        const float inv = s_inv[g];
+        float r[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+        if (app) {
+          const float wa = apw[g];
+          const __nv_bfloat16* vn = snew + D + d4 * 4;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) r[e] = fmaf(wa, __bfloat162float(vn[e]), r[e]);
+        }
+        store4(static_cast<__nv_bfloat16*>(a.out) + (bk * G + g) * D + d4 * 4, r);
+      }
+    }
+    // The sequence's length advances once all its KV heads are done: each has read it by now.
+    if (tid == 0 && has_new) {
+      if (app) {
+        if (atom_add_acq_rel_gpu(&a.cnt_seq[b], 1u) == (uint32_t)a.Hkv - 1u) {
+          a.lengths[b] = L + 1;
+          a.cnt_seq[b] = 0u;
+        }
+      } else if (u % a.Hkv == 0) {
+        raise_flag(a.flags, SELKV_DEVERR_CAPACITY);
+      }
+    }
+    // the next unit rewrites the staged queries, the warp states and the fold scratch only
+    // after every consumer has passed this barrier
+    named_bar_sync(kBar, kCons);
+  }
+}
+
 template <int D, bool R16>
 cudaError_t launch_tc_t(const DecodeArgs& a, cudaStream_t st) {
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)a.B * a.Hkv * a.m_cap;
   if (!encode_rows_bf16(&tk, a.Kc, rows, D, kBoxRows) || !encode_rows_bf16(&tv, a.Vc, rows, D, kBoxRows))
     return cudaErrorInvalidValue;
-  auto kern = decode_tc_kernel<D, R16>;
-  cudaError_t e = set_smem_once<decode_tc_kernel<D, R16>>(Cfg<D>::kSmemBytes);
-  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.splits, a.Hkv, a.B);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = Cfg<D>::kSmemBytes;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = SELKV_DEC_PDL ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, tk, tv, a);
+  if (SELKV_DEC_UNITS && a.splits == 1 && a.B * a.Hkv > kPlanSMs && a.m_cap <= SELKV_DEC_UNITS_MAX_ROWS) {
+    // one split per (b, kv), more units than SMs, short units: persistent CTAs walk the units
+    // (with longer units the static walk balances worse than the hardware's CTA scheduling)
+    cudaError_t e = set_smem_once<decode_units_kernel<D, R16>>(UCfg<D, R16>::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    cfg.gridDim = dim3(kPlanSMs, 1, 1);
+    cfg.dynamicSmemBytes = UCfg<D, R16>::kSmemBytes;
+    return cudaLaunchKernelEx(&cfg, decode_units_kernel<D, R16>, tk, tv, a);
+  }
+  cudaError_t e = set_smem_once<decode_tc_kernel<D, R16>>(Cfg<D>::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  cfg.gridDim = dim3(a.splits, a.Hkv, a.B);
+  cfg.dynamicSmemBytes = Cfg<D>::kSmemBytes;
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<D, R16>, tk, tv, a);
 }
 
 }  // namespace

@@ -336,6 +336,50 @@ def test_decode_back_to_back_appends_sweep_the_split_slices():
     np.testing.assert_array_equal(cache.lengths.cpu().numpy(), np.array(L0) + T)
 
 
+def test_decode_persistent_units_back_to_back():
+    """More (sequence, KV head) units than SMs, one split each (48 sequences x 4 KV heads): the
+    decode runs as persistent CTAs walking the units.  Ragged lengths with the edge cases of a
+    128-row tile and of the early loads (0, 1, 63-65, 127-129 rows), 40 appending steps enqueued
+    back to back in bursts; every sequence of every step against exact attention over its rows
+    (bias per row, 0 for appended rows), then the lengths and the error word."""
+    B, Hq, Hkv, d, m_cap = 48, 8, 4, 128, 600
+    g = torch.Generator().manual_seed(33)
+    edge = [0, 1, 63, 64, 65, 127, 128, 129, 255, 256, 257, 511]
+    L0 = edge + [int(x) for x in torch.randint(0, 540, (B - len(edge),), generator=g)]
+    T, burst = 40, 10
+    shape = api.make_shape("bf16", B, Hq, Hkv, d, 32, m_cap, m_cap)
+    cache = api.alloc_compressed(shape)
+    cache.K_c.copy_(torch.randn(cache.K_c.shape, generator=g))
+    cache.V_c.copy_(torch.randn(cache.V_c.shape, generator=g))
+    cache.bias.copy_(0.5 * torch.rand(cache.bias.shape, generator=g))
+    cache.lengths.copy_(torch.tensor(L0, dtype=torch.int32))
+    qs = torch.randn((T, B, Hq, d), generator=g).to(torch.bfloat16).cuda()
+    ks = torch.randn((T, B, Hkv, d), generator=g).to(torch.bfloat16).cuda()
+    vs = torch.randn((T, B, Hkv, d), generator=g).to(torch.bfloat16).cuda()
+    outs = torch.empty((burst, B, Hq, d), dtype=torch.bfloat16, device="cuda")
+    Kh = cache.K_c.double().cpu().numpy()
+    Vh = cache.V_c.double().cpu().numpy()
+    bh = cache.bias.double().cpu().numpy()
+    qh, kh, vh = (x.double().cpu().numpy() for x in (qs, ks, vs))
+    ws = api.Workspace(S.selkv_decode_workspace_size(shape))
+    for t0 in range(0, T, burst):
+        for i in range(burst):
+            api.decode(cache, qs[t0 + i], ks[t0 + i], vs[t0 + i], out=outs[i], workspace=ws)
+        got = outs.float().cpu().numpy()
+        for i in range(burst):
+            t = t0 + i
+            for b in range(B):
+                L = L0[b] + t
+                Kh[b, :, L] = kh[t, b]
+                Vh[b, :, L] = vh[t, b]
+                bh[b, :, L] = 0.0
+                want = O.decode(qh[t, b], Kh[b], Vh[b], bh[b], L + 1)
+                check_decode(got[i, b], want, "bf16", "step %d seq %d" % (t, b))
+    torch.cuda.synchronize()
+    assert ws.errors() == 0
+    np.testing.assert_array_equal(cache.lengths.cpu().numpy(), np.array(L0) + T)
+
+
 def test_repeat_runs_are_bitwise_identical():
     wl = SMALL["bf16_ragged"]
     x = synth.gen_layer(wl, 5)
