@@ -154,7 +154,7 @@ DecodePlan plan_decode(const selkv_shape& s) {
     off += round256(bytes);
     return o;
   };
-  p.splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs);
+  p.splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs, s.dtype == SELKV_BF16);
   p.cnt_head = take((size_t)s.batch * s.num_kv_heads * 4);
   p.cnt_seq = take((size_t)s.batch * 4);
   p.partial = take((size_t)s.batch * s.num_kv_heads *

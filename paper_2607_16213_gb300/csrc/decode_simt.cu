@@ -152,7 +152,7 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 #define SELKV_DEC_CTAS_PER_SM 1  // decode CTAs planned per SM when splitting the rows
 #endif
 #ifndef SELKV_DEC_FILL_ROWS
-#define SELKV_DEC_FILL_ROWS 512  // a CTA's fixed cost in the split model, in rows streamed
+#define SELKV_DEC_FILL_ROWS 256  // a CTA's fixed cost in the split model, in rows streamed
 #endif
 #ifndef SELKV_DEC_MAX_SPLITS
 #define SELKV_DEC_MAX_SPLITS 64  // most splits of one (sequence, KV head)
@@ -160,11 +160,13 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 
 // Split count of each (sequence, KV head).  The B * Hkv * S CTAs run in waves of
 // CTAS_PER_SM * num_sms; a wave lasts about as long as streaming one CTA's rows plus a fixed
-// fill-and-fold cost worth kFillRows rows (about 5 us at one SM's share of HBM bandwidth, the
-// fixed cost measured per launch).  S minimises waves * (rows per CTA + kFillRows) over the
-// capacity m_cap, fewest splits on ties.  (Batch 4 x 8k compressed rows: 512 picks 4 splits,
-// 29.0 us per launch; 192 picked 9 splits in two waves, 31.2 us.  Batch 1 x 25k: 19 either way.)
-int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
+// fill-and-fold cost worth kFillRows rows.  S minimises waves * (rows per CTA + kFillRows) over
+// the capacity m_cap, fewest splits on ties.  With `unit_walk` (the tensor-core decode), one
+// split over more units than slots with at most SELKV_DEC_UNITS_MAX_ROWS rows runs as
+// persistent CTAs that pay the fixed cost once: waves * rows + kFillRows.  (Serving sweep,
+// batch 8 x 32k at 50%: 256 rows of fixed cost pick more splits than 512 did, 85.7 -> 71.0 us
+// per launch; batch 4 x 8k: 4 splits either way.)
+int decode_splits(int B, int Hkv, int m_cap, int num_sms, bool unit_walk) {
   constexpr long kFillRows = SELKV_DEC_FILL_ROWS;
   const long units = (long)B * Hkv;
   const long slots = std::max(1L, (long)SELKV_DEC_CTAS_PER_SM * num_sms);
@@ -174,7 +176,8 @@ int decode_splits(int B, int Hkv, int m_cap, int num_sms) {
   for (int S = 1; S <= smax; ++S) {
     const long waves = (units * S + slots - 1) / slots;
     const long rows = ((long)(m_cap + S - 1) / S + 63) / 64 * 64;
-    const long cost = waves * (rows + kFillRows);
+    const bool walk = unit_walk && S == 1 && units > slots && m_cap <= SELKV_DEC_UNITS_MAX_ROWS;
+    const long cost = walk ? waves * rows + kFillRows : waves * (rows + kFillRows);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
       best = S;

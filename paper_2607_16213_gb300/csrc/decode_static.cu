@@ -106,7 +106,7 @@ extern "C" SELKV_API selkv_status selkv_decode_attn_static(
   if (flags_out != nullptr && (reinterpret_cast<uintptr_t>(flags_out) & 3u) != 0) return SELKV_ERR_INVALID_ARG;
 
   // Scratch layout: error word | per-(b, kv) counters | per-b counters | split partials.
-  const int splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs);
+  const int splits = decode_splits(s.batch, s.num_kv_heads, s.m_cap, kPlanSMs, s.dtype == SELKV_BF16);
   const size_t off_head = 256;
   const size_t off_seq = off_head + round256((size_t)s.batch * s.num_kv_heads * 4);
   const size_t off_part = off_seq + round256((size_t)s.batch * 4);

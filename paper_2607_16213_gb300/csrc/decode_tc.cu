@@ -59,9 +59,6 @@ namespace {
 #ifndef SELKV_DEC_UNITS
 #define SELKV_DEC_UNITS 1  // persistent unit-walking CTAs when every (b, kv) has one split and they outnumber the SMs
 #endif
-#ifndef SELKV_DEC_UNITS_MAX_ROWS
-#define SELKV_DEC_UNITS_MAX_ROWS 2112  // ... and their capacity is at most this many rows
-#endif
 #ifndef SELKV_DEC_MINBLOCKS
 #define SELKV_DEC_MINBLOCKS 1  // CTAs resident per SM (register / shared-memory budget)
 #endif

@@ -341,7 +341,12 @@ bool merge_copies_kept_rows(const CompressArgs& a);
 // SELKV_ERR_CUDA, with `e` kept for selkv_last_cuda_error on this thread.
 selkv_status cuda_fail(cudaError_t e);
 
-int decode_splits(int B, int Hkv, int m_cap, int num_sms);
+#ifndef SELKV_DEC_UNITS_MAX_ROWS
+#define SELKV_DEC_UNITS_MAX_ROWS 2112  // persistent unit-walking decode: most rows of a unit
+#endif
+// Splits per (b, kv) of a decode launch; unit_walk: the tensor-core decode, which walks many
+// short one-split units with persistent CTAs.
+int decode_splits(int B, int Hkv, int m_cap, int num_sms, bool unit_walk);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);     // dispatch by dtype
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);  // bf16: TMA + tensor cores
 
