@@ -336,16 +336,18 @@ def test_decode_back_to_back_appends_sweep_the_split_slices():
     np.testing.assert_array_equal(cache.lengths.cpu().numpy(), np.array(L0) + T)
 
 
-def test_decode_persistent_units_back_to_back():
-    """More (sequence, KV head) units than SMs, one split each (48 sequences x 4 KV heads): the
-    decode runs as persistent CTAs walking the units.  Ragged lengths with the edge cases of a
-    128-row tile and of the early loads (0, 1, 63-65, 127-129 rows), 40 appending steps enqueued
-    back to back in bursts; every sequence of every step against exact attention over its rows
-    (bias per row, 0 for appended rows), then the lengths and the error word."""
-    B, Hq, Hkv, d, m_cap = 48, 8, 4, 128, 600
-    g = torch.Generator().manual_seed(33)
+@pytest.mark.parametrize("B,Hq,Hkv", [(48, 8, 4), (20, 128, 8)])
+def test_decode_persistent_units_back_to_back(B, Hq, Hkv):
+    """More (sequence, KV head) units than SMs, one split each (48 sequences x 4 KV heads, and
+    20 x 8 with 16-head groups): the decode runs as persistent CTAs walking the units.  Ragged
+    lengths with the edge cases of a 128-row tile and of the early loads (0, 1, 63-65, 127-129
+    rows), 40 appending steps enqueued back to back in bursts; every sequence of every step
+    against exact attention over its rows (bias per row, 0 for appended rows), then the lengths
+    and the error word."""
+    d, m_cap = 128, 600
+    g = torch.Generator().manual_seed(33 + B)
     edge = [0, 1, 63, 64, 65, 127, 128, 129, 255, 256, 257, 511]
-    L0 = edge + [int(x) for x in torch.randint(0, 540, (B - len(edge),), generator=g)]
+    L0 = (edge + [int(x) for x in torch.randint(0, 540, (max(0, B - len(edge)),), generator=g)])[:B]
     T, burst = 40, 10
     shape = api.make_shape("bf16", B, Hq, Hkv, d, 32, m_cap, m_cap)
     cache = api.alloc_compressed(shape)
