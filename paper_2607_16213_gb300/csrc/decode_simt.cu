@@ -154,6 +154,12 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 #ifndef SELKV_DEC_FILL_ROWS
 #define SELKV_DEC_FILL_ROWS 256  // a CTA's fixed cost in the split model, in rows streamed
 #endif
+#ifndef SELKV_DEC_BACKFILL_WAVES
+#define SELKV_DEC_BACKFILL_WAVES 3  // one split over at least this many waves of units ...
+#endif
+#ifndef SELKV_DEC_BACKFILL_MAX_ROWS
+#define SELKV_DEC_BACKFILL_MAX_ROWS 8192  // ... of at most this many rows: fractional waves
+#endif
 #ifndef SELKV_DEC_MAX_SPLITS
 #define SELKV_DEC_MAX_SPLITS 64  // most splits of one (sequence, KV head)
 #endif
@@ -163,9 +169,14 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t st) {
 // fill-and-fold cost worth kFillRows rows.  S minimises waves * (rows per CTA + kFillRows) over
 // the capacity m_cap, fewest splits on ties.  With `unit_walk` (the tensor-core decode), one
 // split over more units than slots with at most SELKV_DEC_UNITS_MAX_ROWS rows runs as
-// persistent CTAs that pay the fixed cost once: waves * rows + kFillRows.  (Serving sweep,
-// batch 8 x 32k at 50%: 256 rows of fixed cost pick more splits than 512 did, 85.7 -> 71.0 us
-// per launch; batch 4 x 8k: 4 splits either way.)
+// persistent CTAs that pay the fixed cost once: waves * rows + kFillRows.  There too, one split
+// over at least BACKFILL_WAVES waves of units of at most BACKFILL_MAX_ROWS rows counts its waves as
+// units / slots: the block scheduler starts each unit as a slot frees, so ragged units pack
+// (batch 64 x 8k at 50%: 151.0 -> 144.0 us per launch, 64 x 32k at 10%: 129.6 -> 120.7; with
+// longer units the last ones started leave a tail: 64 x 32k at 50% 490 -> 496, 64 x 128k at
+// 25% 924 -> 972, so those keep their splits).  (Serving sweep, batch 8 x 32k at 50%: 256
+// rows of fixed cost pick more splits than 512 did, 85.7 -> 71.0 us per launch; batch 4 x 8k:
+// 4 splits either way.)
 int decode_splits(int B, int Hkv, int m_cap, int num_sms, bool unit_walk) {
   constexpr long kFillRows = SELKV_DEC_FILL_ROWS;
   const long units = (long)B * Hkv;
@@ -174,10 +185,14 @@ int decode_splits(int B, int Hkv, int m_cap, int num_sms, bool unit_walk) {
   int best = 1;
   long best_cost = -1;
   for (int S = 1; S <= smax; ++S) {
-    const long waves = (units * S + slots - 1) / slots;
+    // costs in units of rows x slots, so that fractional waves stay integral
+    const long waves = (units * S + slots - 1) / slots * slots;
     const long rows = ((long)(m_cap + S - 1) / S + 63) / 64 * 64;
     const bool walk = unit_walk && S == 1 && units > slots && m_cap <= SELKV_DEC_UNITS_MAX_ROWS;
-    const long cost = walk ? waves * rows + kFillRows : waves * (rows + kFillRows);
+    const bool backfill = unit_walk && S == 1 && !walk && units >= (long)SELKV_DEC_BACKFILL_WAVES * slots &&
+                          m_cap <= SELKV_DEC_BACKFILL_MAX_ROWS;
+    const long cost = walk ? waves * rows + kFillRows * slots
+                           : (backfill ? units : waves) * (rows + kFillRows);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
       best = S;

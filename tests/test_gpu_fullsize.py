@@ -79,7 +79,7 @@ def test_llama_32l_b4_layers(layer, seq):
     _decode_sampled(wl, cache, layer, [seq, (seq + 1) % wl.batch], steps=2)
 
 
-SWEEP = [(1, 8192, 0.10), (8, 8192, 0.50), (64, 8192, 0.25), (8, 32768, 0.25),
+SWEEP = [(1, 8192, 0.10), (8, 8192, 0.50), (64, 8192, 0.25), (64, 8192, 0.50), (8, 32768, 0.25),
          (32, 8192, 0.10), (1, 131072, 0.25), (1, 32768, 0.50)]
 
 
