@@ -99,16 +99,14 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ oracle arm
 def _oracle_unit(job):
-    """One unit of the oracle baseline: generate layer `layer` of sequence 0 (on job[4]
-    threads, default 1), compress it with the fp64 oracle, then decode `tokens` tokens over
-    the compressed cache (each appending a row).  Returns the times and the process's CPU
-    time."""
-    wl, layer, tokens, per_head = job[:4]
-    gen_threads = job[4] if len(job) > 4 else 1
+    """One unit of the oracle baseline: generate layer `layer` of sequence 0, compress it with
+    the fp64 oracle, then decode `tokens` tokens over the compressed cache (each appending a
+    row).  Returns the times and the process's CPU time."""
+    wl, layer, tokens, per_head = job
     from oracle import selkv_oracle as O
     cpu0 = time.process_time()
     one = wl.with_(batch=1)
-    x = synth.gen_layer(one, layer, threads=gen_threads)
+    x = synth.gen_layer(one, layer, threads=1)
     n = int(x["n_len"][0])
     K, V, Q = (x[k][0].astype(np.float64) for k in ("K", "V", "Q_obs"))
     t0 = time.perf_counter()
@@ -128,13 +126,12 @@ def _oracle_unit(job):
             "cpu_s": time.process_time() - cpu0}
 
 
-def _single_threaded_blas():
-    """Environment for worker processes: one BLAS / OpenMP thread each (the pool supplies the
-    parallelism)."""
+def _blas_threads_env(threads: int):
+    """Environment for worker processes: `threads` BLAS / OpenMP threads each."""
     keys = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS")
     old = {k: os.environ.get(k) for k in keys}
     for k in keys:
-        os.environ[k] = "1"
+        os.environ[k] = str(threads)
     return old
 
 
@@ -146,41 +143,81 @@ def _restore_env(old):
             os.environ[k] = v
 
 
-def oracle_sample(wl: synth.Workload, per_head: bool = False, decode_tokens: int = 2,
-                  single_thread_refs: bool = True) -> dict:
-    """The fp64 oracle on the host's cores, parallel over independent units: one worker process
-    per core (spawned, single-threaded BLAS), each compressing one layer of sequence 0 (layers
-    0 .. P-1) and decoding `decode_tokens` tokens over it; all P run at once, so each unit's
-    time is taken under the memory contention of a full machine.  The step estimate schedules
-    the step's B x L (sequence, layer) units on the P cores: ceil(B L / P) rounds of the mean
-    unit time (compression + decode_steps decode tokens).  With single_thread_refs, the tiny
-    and the 16k single-layer workloads are also timed alone on one core (compression and
-    decode per layer)."""
-    import multiprocessing as mp
-    P = os.cpu_count() or 1
-    jobs = [(wl, layer % wl.layers, decode_tokens, per_head) for layer in range(P)]
-    refs = [(synth.WORKLOADS["tiny"], 0, 16, False), (synth.WORKLOADS["llama_layer"], 0, 2, False)]
-    old = _single_threaded_blas()
-    try:
-        ctx = mp.get_context("spawn")   # no fork of a process that holds a CUDA context
-        with ctx.Pool(P) as pool:
-            t0 = time.perf_counter()
-            res = pool.map(_oracle_unit, jobs, chunksize=1)
-            wall = time.perf_counter() - t0
-            single = pool.map(_oracle_unit, refs, chunksize=1) if single_thread_refs else None
-    finally:
-        _restore_env(old)
+class _OraclePool:
+    """P spawned worker processes with `blas_threads` BLAS threads each; spawned, not forked,
+    so that no worker inherits a CUDA context."""
+
+    def __init__(self, P: int, blas_threads: int = 1):
+        self.P = P
+        self.blas_threads = blas_threads
+
+    @classmethod
+    def for_step(cls, wl):
+        """As many workers as the step has (sequence, layer) units, at most one per core, and
+        the cores shared out among them as BLAS threads (one each when the units outnumber the
+        cores; all of them for a one-unit step)."""
+        cores = os.cpu_count() or 1
+        P = max(1, min(cores, wl.batch * wl.layers))
+        return cls(P, max(1, cores // P))
+
+    def __enter__(self):
+        import multiprocessing as mp
+        old = _blas_threads_env(self.blas_threads)
+        try:
+            self.pool = mp.get_context("spawn").Pool(self.P)
+        finally:
+            _restore_env(old)
+        return self
+
+    def __exit__(self, *exc):
+        self.pool.terminate()
+        self.pool.join()
+
+    def units(self, wl, first_layer: int, tokens: int, per_head: bool):
+        """P units at once: worker i compresses layer (first_layer + i) mod L of sequence 0 and
+        decodes `tokens` tokens over it.  Returns the units' results and the wall time."""
+        jobs = [(wl, (first_layer + i) % wl.layers, tokens, per_head) for i in range(self.P)]
+        t0 = time.perf_counter()
+        res = self.pool.map(_oracle_unit, jobs, chunksize=1)
+        return res, time.perf_counter() - t0
+
+
+def _step_rate(wl, res, P: int):
+    """Tokens per second of the workload's step from a sample of (sequence, layer) units run P
+    at once: the step's B x L units take ceil(B L / P) rounds of the mean unit (compression +
+    decode_steps decode tokens).  Returns (rate, rounds)."""
     unit_s = statistics.mean(r["compress_s"] + wl.decode_steps * r["decode_s_per_token"] for r in res)
     rounds = math.ceil(wl.batch * wl.layers / P)
-    step_s = rounds * unit_s
-    tokens = wl.batch * wl.decode_steps
+    return wl.batch * wl.decode_steps / (rounds * unit_s), rounds
+
+
+def oracle_sample(wl: synth.Workload, per_head: bool = False, decode_tokens: int = 2,
+                  single_thread_refs: bool = True) -> dict:
+    """The fp64 oracle on the host's cores, parallel over independent units: one spawned worker
+    process per (sequence, layer) unit of the step up to one per core (single-threaded BLAS
+    when the units outnumber the cores, the cores shared out as BLAS threads otherwise), each
+    compressing one layer of sequence 0 (layers 0 .. P-1) and decoding `decode_tokens` tokens
+    over it; all P run at once, so each unit's time is taken under the memory contention of a
+    full machine.  The step estimate schedules the step's B x L units on the P workers:
+    ceil(B L / P) rounds of the mean unit time (compression + decode_steps decode tokens).
+    With single_thread_refs, the tiny and the 16k single-layer workloads are also timed alone
+    on one core each (compression and decode per layer)."""
+    refs = [(synth.WORKLOADS["tiny"], 0, 16, False), (synth.WORKLOADS["llama_layer"], 0, 2, False)]
+    with _OraclePool.for_step(wl) as pool:
+        res, wall = pool.units(wl, 0, decode_tokens, per_head)
+    P, threads = pool.P, pool.blas_threads
+    single = None
+    if single_thread_refs:
+        with _OraclePool(len(refs), 1) as rp:
+            single = rp.pool.map(_oracle_unit, refs, chunksize=1)
+    value, rounds = _step_rate(wl, res, P)
     busy = sum(r["cpu_s"] for r in res) / wall
-    out = {"value": tokens / step_s, "unit": "tokens/s", "cores": P, "kind": "oracle",
-           "sample": ("fp64 oracle, %d worker processes (one per core, single-threaded BLAS) at once, "
+    out = {"value": value, "unit": "tokens/s", "cores": P * threads, "kind": "oracle",
+           "sample": ("fp64 oracle, %d worker process(es) (%d BLAS thread(s) each) at once, "
                       "each compressing one layer of one sequence (n=%d) and decoding %d token(s); "
                       "the step's %d (sequence, layer) units scheduled as %d round(s) of the mean "
                       "unit (compression + %d decode tokens)")
-           % (P, wl.n, decode_tokens, wl.batch * wl.layers, rounds, wl.decode_steps),
+           % (P, threads, wl.n, decode_tokens, wl.batch * wl.layers, rounds, wl.decode_steps),
            "compress_s_per_layer": statistics.mean(r["compress_s"] for r in res),
            "decode_s_per_layer_token": statistics.mean(r["decode_s_per_token"] for r in res),
            "sample_wall_s": wall, "cores_busy_avg": round(busy, 2)}
@@ -191,15 +228,6 @@ def oracle_sample(wl: synth.Workload, per_head: bool = False, decode_tokens: int
                                                                    + w.decode_steps * r["decode_s_per_token"]))}
             for (w, _, _, _), r in zip(refs, single)}
     return out
-
-
-def oracle_step_sample(wl: synth.Workload, layer: int, decode_tokens: int, per_head: bool = False) -> dict:
-    """One bounded sample of the oracle in this process (BLAS on all cores): compression of
-    layer `layer` of sequence 0 and `decode_tokens` decode tokens, scaled to the step."""
-    r = _oracle_unit((wl, layer, decode_tokens, per_head, os.cpu_count() or 1))
-    step_s = wl.batch * wl.layers * (r["compress_s"] + wl.decode_steps * r["decode_s_per_token"])
-    return {"value": wl.batch * wl.decode_steps / step_s, "compress_s": r["compress_s"],
-            "decode_s_per_token": r["decode_s_per_token"]}
 
 
 # ------------------------------------------------------------------------------ ranks
@@ -976,9 +1004,13 @@ def kernel_revision() -> str:
 
 
 def run_reference(args):
-    """The oracle arm: each step is one bounded sample of the workload's step (compression of
-    one layer, a different layer each step, and 8 decode tokens over it), timed in this process
-    with BLAS on the host's cores and scaled to the step; the line reports the median."""
+    """The oracle arm: the fp64 oracle on the host's cores, parallel over independent units as
+    in the main line's `cpu_baseline` (one spawned worker per (sequence, layer) unit up to one
+    per core, the cores left over shared out as BLAS threads; the pool kept for the whole run).
+    Each step is one bounded sample of the workload's step: the P workers each compress a
+    different layer of sequence 0 (the next P layers every step) and decode 8 tokens over it,
+    all at once; the step's B x L units are scheduled as ceil(B L / P) rounds of the mean unit.
+    Warm-up steps decode one token.  The line reports the median over the steps."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if world > 1 and rank != 0:
@@ -988,25 +1020,27 @@ def run_reference(args):
         wl = wl.with_(decode_steps=args.decode_steps)
     per_head = args.select_mode == "per_head"
     tokens_per_sample = 8
-    for i in range(args.warmup):
-        oracle_step_sample(wl, i % wl.layers, 1, per_head)
-    vals, comp, dec = [], [], []
-    cpu0, t0 = os.times(), time.perf_counter()
-    for k in range(args.steps):
-        r = oracle_step_sample(wl, (args.warmup + k) % wl.layers, tokens_per_sample, per_head)
-        vals.append(r["value"])
-        comp.append(r["compress_s"])
-        dec.append(r["decode_s_per_token"])
-    wall = time.perf_counter() - t0
-    cpu1 = os.times()
-    busy = ((cpu1.user - cpu0.user) + (cpu1.system - cpu0.system)) / max(1e-9, wall)
+    vals, comp, dec, cpu_s, walls = [], [], [], 0.0, 0.0
+    with _OraclePool.for_step(wl) as pool:
+        P, threads = pool.P, pool.blas_threads
+        for i in range(args.warmup):
+            pool.units(wl, i * P, 1, per_head)
+        for k in range(args.steps):
+            res, wall = pool.units(wl, (args.warmup + k) * P, tokens_per_sample, per_head)
+            vals.append(_step_rate(wl, res, P)[0])
+            comp.append(statistics.mean(r["compress_s"] for r in res))
+            dec.append(statistics.mean(r["decode_s_per_token"] for r in res))
+            cpu_s += sum(r["cpu_s"] for r in res)
+            walls += wall
     v = statistics.median(vals)
     tokens = wl.batch * wl.decode_steps
-    sample = ("fp64 oracle, one process with BLAS on the host's cores: per step the compression of "
-              "one layer of one sequence (n=%d; layers %d..%d over the steps) and %d decode tokens "
-              "over it, scaled to %d layers x %d sequences x %d decode steps"
-              % (wl.n, args.warmup % wl.layers, (args.warmup + args.steps - 1) % wl.layers,
-                 tokens_per_sample, wl.layers, wl.batch, wl.decode_steps))
+    rounds = math.ceil(wl.batch * wl.layers / P)
+    sample = ("fp64 oracle, %d worker process(es) (%d BLAS thread(s) each) at once: per step each "
+              "compresses one layer of one sequence (n=%d; %d different layer(s) a step) and decodes "
+              "%d tokens over it; the step's %d (sequence, layer) units scheduled as %d round(s) of the "
+              "mean unit (compression + %d decode tokens)"
+              % (P, threads, wl.n, min(P, wl.layers), tokens_per_sample, wl.batch * wl.layers, rounds,
+                 wl.decode_steps))
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": tokens / v * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
@@ -1015,8 +1049,8 @@ def run_reference(args):
                        "rho": wl.rho, "decode_steps": wl.decode_steps, "q_heads": wl.num_q_heads,
                        "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim, "obs_window": wl.obs_window,
                        "select_mode": args.select_mode},
-            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": sample, "cores_busy_avg": round(busy, 2),
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": P * threads, "kind": "oracle",
+                             "sample": sample, "cores_busy_avg": round(cpu_s / max(1e-9, walls), 2),
                              "compress_s_per_layer": statistics.median(comp),
                              "decode_s_per_layer_token": statistics.median(dec)},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
