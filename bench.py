@@ -506,7 +506,8 @@ def run_gpu(args):
     if os.path.exists(prof):
         with open(prof) as f:
             pj = json.load(f)
-        if pj.get("workload") == wl.name and pj.get("kernel_rev") == kernel_revision():
+        if pj.get("workload") == wl.name and pj.get("kernel_rev") == kernel_revision(
+                S.selkv_decode_workspace_size(L.shape)):
             traffic = pj.get("bytes_per_launch")
 
     score = None if args.no_score else measure_scoring(L, S, api, torch, stream, dev, peaks, peak_src)
@@ -987,19 +988,20 @@ def run_sweep(args, points):
         sys.exit(1)
 
 
-DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "decode_simt.cu", "ptx.cuh", "selkv_internal.cuh",
-                  "tma_host.cu")
+DECODE_SOURCES = ("decode_tc.cu", "decode_common.cuh", "ptx.cuh", "selkv_internal.cuh", "tma_host.cu")
 
 
-def kernel_revision() -> str:
-    """Content hash of the decode kernel's sources: profiler figures recorded for the decode
-    kernel are valid only for this revision."""
+def kernel_revision(plan_bytes: int) -> str:
+    """Content hash of the tensor-core decode kernel's sources and of its launch plan for the
+    workload (the decode workspace size, which grows with the split count the host picks):
+    profiler figures recorded for the decode kernel are valid only for this revision."""
     import hashlib
     h = hashlib.sha256()
     cs = os.path.join(ROOT, "paper_2607_16213_gb300", "csrc")
     for f in DECODE_SOURCES:
         with open(os.path.join(cs, f), "rb") as fh:
             h.update(fh.read())
+    h.update(b"plan:%d" % int(plan_bytes))
     return h.hexdigest()[:16]
 
 
