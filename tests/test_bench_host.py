@@ -2,7 +2,8 @@
 torchrun would, rendezvous on 127.0.0.1); every rank replays its own replica of the workload
 (weak scaling, no collective on the data path), the job's time is the slowest rank's, and the
 rate counts every rank's tokens.  Roofline: the decode kernel's algorithmic bytes per launch,
-checked against a count by hand."""
+checked against a count by hand.  Oracle baseline: the process pool's size and the step's
+schedule of units over it."""
 import os
 import socket
 import subprocess
@@ -78,3 +79,31 @@ def test_decode_bytes_per_launch_by_hand():
     assert bench.decode_bytes_per_launch(wl, [100000], T) == pytest.approx(103047330.0)
     per_head = [8 * (25000 + t + 1) * 516 + 2 * 32 * 256 + 2 * 8 * 256 for t in range(T)]
     assert bench.decode_bytes_per_launch(wl, [100000], T, per_head=True) == pytest.approx(sum(per_head) / T)
+
+
+def test_oracle_pool_sized_by_the_steps_units(monkeypatch):
+    """One worker per (sequence, layer) unit of the step, at most one per core; the cores left
+    over go to the workers as BLAS threads."""
+    import synth
+    monkeypatch.setattr(os, "cpu_count", lambda: 16)
+    wl = synth.WORKLOADS["long_100k"]                      # 32 layers x 1 sequence
+    p = bench._OraclePool.for_step(wl)
+    assert (p.P, p.blas_threads) == (16, 1)
+    p = bench._OraclePool.for_step(synth.WORKLOADS["llama_layer"])   # one unit
+    assert (p.P, p.blas_threads) == (1, 16)
+    p = bench._OraclePool.for_step(wl.with_(layers=5))
+    assert (p.P, p.blas_threads) == (5, 3)
+
+
+def test_step_rate_schedules_units_in_rounds():
+    """B x L units on P workers take ceil(B L / P) rounds of the mean unit (compression +
+    decode_steps tokens); the rate is the step's tokens over that time."""
+    import synth
+    wl = synth.WORKLOADS["long_100k"]                      # 32 units, 256 tokens a step
+    res = [{"compress_s": 8.0, "decode_s_per_token": 0.1}, {"compress_s": 10.0, "decode_s_per_token": 0.1}]
+    rate, rounds = bench._step_rate(wl, res, 16)
+    assert rounds == 2
+    assert rate == pytest.approx(256 / (2 * (9.0 + 256 * 0.1)))
+    rate, rounds = bench._step_rate(wl, res, 12)
+    assert rounds == 3
+    assert rate == pytest.approx(256 / (3 * (9.0 + 256 * 0.1)))
