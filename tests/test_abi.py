@@ -64,6 +64,36 @@ def test_workspace_sizes(lib):
     assert S.selkv_decode_workspace_size(shape(dtype=5)) == 0
 
 
+def _decode_splits(s) -> int:
+    """The split count the host planned for a decode shape, read back from the decode
+    workspace size: a 256-byte header, the per-(b, kv) and per-b arrival counters, and one
+    record per (b, kv) of G S d partial outputs plus G S (max, sum) pairs padded to 16 bytes,
+    each region rounded up to 256 bytes."""
+    r256 = lambda x: (x + 255) // 256 * 256
+    G, units = s.num_q_heads // s.num_kv_heads, s.batch * s.num_kv_heads
+    total = S.selkv_decode_workspace_size(s)
+    for splits in range(1, 65):
+        rec = G * splits * s.head_dim + (G * splits * 2 + 3) // 4 * 4
+        if 256 + r256(units * 4) + r256(s.batch * 4) + r256(units * rec * 4) == total:
+            return splits
+    raise AssertionError("no split count gives %d bytes" % total)
+
+
+@pytest.mark.parametrize("batch,m_cap,splits", [
+    (1, 25280, 19),    # 100k context, 25% kept: one wave of 8 x 19 CTAs
+    (4, 8512, 4),      # batch 4 x 32k at 25%: 4 splits in one wave, not 9 in two
+    (1, 512, 8),       # short cache: splits with a combine beat one CTA streaming alone
+    (32, 8128, 4),     # 256 units (under three waves): the units keep their splits
+    (64, 2048, 1),     # 512 short units: one split each (the persistent walk)
+    (64, 4096, 1),     # 512 units of at most 8192 rows: one split, waves counted fractionally
+    (64, 16256, 2),    # longer units keep their splits
+])
+def test_decode_split_plan(lib, batch, m_cap, splits):
+    """The split model's choices for the workloads it was tuned on (bf16, 32 query / 8 KV
+    heads, d = 128), as the workspace size shows them."""
+    assert _decode_splits(shape(batch=batch, m_cap=m_cap)) == splits
+
+
 def _compress(s, n_len, rho=0.25, params=None, ptrs=None, ws=FAKE, wsb=1 << 40):
     p = params or S.selkv_params.defaults()
     t = dict(K=FAKE, V=FAKE, Q=FAKE, Kc=FAKE, Vc=FAKE, bias=FAKE, lengths=FAKE)
